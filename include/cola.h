@@ -1,0 +1,164 @@
+/*
+ * cola.h -- C ABI of the GB300 (sm_103a) CoLA auto-encoder layer library.
+ *
+ * CoLA (arXiv 2502.10940) replaces every full-size projection h = W x of a
+ * LLaMA-style block by the low-rank auto-encoder
+ *
+ *     h = B sigma(A x),   A in R^{r x d_in},  B in R^{d_out x r},  r < min(d_in, d_out)
+ *
+ * (Sec. 3.2, Eq. (main-fwd)).  This library runs its forward pass and its full
+ * backward pass (Sec. 3.4: the "2x rule" grad_x = W^T grad_h,
+ * grad_W = grad_h x^T applied to both products, chain rule through sigma) on
+ * the tensor cores, in the two modes of the paper: CoLA, which saves both
+ * rank-r activations A x and sigma(A x), and CoLA-M (Sec. 4.2, App. C), which
+ * saves only A x and recomputes sigma(A x) in the backward.
+ *
+ * Storage (row-major, token-major; row t = token t, n tokens):
+ *   X  [n x d_in]    layer input,              row pitch ld_x  (also dX)
+ *   A  [r x d_in]    down-projection factor,    row pitch ld_a  (also dA)
+ *   B  [d_out x r]   up-projection factor,      row pitch r     (also dB)
+ *   Z  [n x r]       Z = X A^T  (the rank-r activation A x), pitch r
+ *   H  [n x r]       H = sigma(Z), pitch r
+ *   Y  [n x d_out]   Y = H B^T,   row pitch ld_y (also dY)
+ * The paper writes X column-wise (X in R^{d_in x n}, Sec. 3.3); token-major
+ * storage is its transpose, and A, B keep the nn.Linear weight layouts.
+ *
+ * Numerics: every tensor is bf16 (IEEE bfloat16) in device memory; products
+ * accumulate in fp32; Z is rounded to bf16 once and H = bf16(sigma(bf16 Z)),
+ * so CoLA-M's recomputed H is bit-identical to CoLA's saved H; the gradient at
+ * Z is dZ = bf16(fp32(dY B) * sigma'(Z)).  Weight gradients reduce their token
+ * split in a fixed order: every result is deterministic.
+ *
+ * Conventions shared by every entry point:
+ *   - All pointers are DEVICE pointers of the current device, owned by the
+ *     caller and at least 16-byte aligned.  The library never allocates,
+ *     frees or synchronises (cola_check_status excepted).
+ *   - Calls are asynchronous on `stream` (0 = legacy default stream).
+ *     Argument errors are detected before any launch and return without
+ *     touching memory.  A launch failure returns COLA_ERR_LAUNCH.
+ *   - Sizes: n, d_in, d_out >= 1; r >= 64 and r % 64 == 0 (else
+ *     COLA_ERR_UNSUPPORTED); row pitches (ld_*) are in elements, >= the
+ *     logical width and a multiple of 8 (16 bytes); 0 selects the logical
+ *     width.  Every extent must stay below 2^31 elements per row/column.
+ *   - `ws` is a caller-owned device workspace of at least
+ *     cola_workspace_size() bytes, 256-byte aligned; its first 256 bytes hold
+ *     the device status word and must be zeroed once with
+ *     cola_workspace_init() before first use.  One workspace must not be
+ *     used by two calls that may run concurrently.
+ *   - Every wait inside the kernels is bounded (about 2 s).  A wait that runs
+ *     out records a code in the workspace status word and the kernel returns
+ *     early (its outputs are then undefined); cola_check_status() reports it.
+ */
+#ifndef COLA_H
+#define COLA_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    COLA_OK = 0,
+    COLA_ERR_INVALID = 1,        /* null pointer, non-positive size, bad pitch or enum */
+    COLA_ERR_ALIGN = 2,          /* a pointer not 16-byte aligned (ws: 256-byte) */
+    COLA_ERR_UNSUPPORTED = 3,    /* r not a positive multiple of 64, extent too large, no sm_103 device */
+    COLA_ERR_WORKSPACE = 4,      /* ws_bytes below cola_workspace_size() */
+    COLA_ERR_LAUNCH = 5,         /* a CUDA launch or driver call failed */
+    COLA_ERR_DEVICE_TIMEOUT = 6  /* a bounded device-side wait ran out (see cola_check_status) */
+} cola_status_t;
+
+typedef enum {
+    COLA_SIGMA_IDENTITY = 0,     /* sigma(z) = z: the plain low-rank product B A x */
+    COLA_SIGMA_SILU = 1,         /* Swish / SiLU, z / (1 + e^-z) (LLaMA, Sec. 5) */
+    COLA_SIGMA_GELU = 2          /* GELU, erf form z * Phi(z) (BERT, Sec. 5.3) */
+} cola_sigma_t;
+
+typedef enum {
+    COLA_MODE_COLA = 0,          /* forward stores Z and H; backward reads both */
+    COLA_MODE_COLA_M = 1         /* forward stores Z only; backward recomputes H = sigma(Z) */
+} cola_mode_t;
+
+/* The layer of Eq. (main-fwd) as the paper states it: (d_in, d_out, rank r,
+ * sigma) applied to n tokens. */
+typedef struct {
+    int64_t n;          /* tokens (sequences x sequence length) */
+    int64_t d_in;       /* input width */
+    int64_t d_out;      /* output width */
+    int64_t r;          /* rank, r % 64 == 0 */
+    int64_t ld_x;       /* row pitch of X and dX in elements (0: d_in) */
+    int64_t ld_y;       /* row pitch of Y and dY in elements (0: d_out) */
+    int64_t ld_a;       /* row pitch of A and dA in elements (0: d_in) */
+    int32_t sigma;      /* cola_sigma_t */
+    int32_t mode;       /* cola_mode_t */
+    int32_t wgrad_fp32; /* 0: dA, dB are bf16 and overwritten; 1: dA, dB are fp32 and
+                           accumulated into (dA += ..., dB += ...), row pitches as above */
+    int32_t reserved;   /* must be 0 */
+} cola_desc_t;
+
+/* Bytes of workspace that cola_fwd / cola_bwd (fused_qkv = 0) or the fused
+ * q/k/v entry points (fused_qkv = 1) need for `desc` on the current device.
+ * The value depends on n, r, d_in, d_out, the mode and the device's SM count
+ * (it sizes the weight-gradient split over tokens). */
+cola_status_t cola_workspace_size(const cola_desc_t* desc, int fused_qkv, size_t* bytes);
+
+/* Zero the workspace status word (first 256 bytes of ws), asynchronously. */
+cola_status_t cola_workspace_init(void* ws, void* stream);
+
+/* Forward, Eq. (main-fwd):  Z = X A^T,  H = sigma(Z),  Y = H B^T.
+ *   X [n x d_in] (ld_x), A [r x d_in] (ld_a), B [d_out x r]: inputs.
+ *   Y [n x d_out] (ld_y): output.
+ *   Z_save [n x r]: output, saved for the backward (both modes).
+ *   H_save [n x r]: output under COLA_MODE_COLA; must be NULL under COLA_M
+ *                   (H is then formed in the workspace and not kept).
+ * Two tensor-core GEMMs: Z/H (sigma fused in the epilogue), then Y. */
+cola_status_t cola_fwd(const cola_desc_t* desc, const void* X, const void* A, const void* B, void* Y,
+                       void* Z_save, void* H_save, void* ws, size_t ws_bytes, void* stream);
+
+/* Backward, Sec. 3.4 (two GEMMs per forward GEMM, chain rule through sigma):
+ *   dZ = (dY B) * sigma'(Z)      [n x r]    (workspace)
+ *   dB = dY^T H                  [d_out x r]
+ *   dA = dZ^T X                  [r x d_in] (ld_a)
+ *   dX = dZ A                    [n x d_in] (ld_x)
+ * Inputs X, A, B, dY [n x d_out] (ld_y), Z_save; H_save under COLA (must be
+ * NULL under COLA_M, where H = sigma(Z_save) is recomputed into the
+ * workspace).  Outputs dX (bf16), dA and dB (bf16, or fp32 accumulated when
+ * desc->wgrad_fp32).  The result does not depend on the mode, bit for bit. */
+cola_status_t cola_bwd(const cola_desc_t* desc, const void* X, const void* A, const void* B, const void* dY,
+                       const void* Z_save, const void* H_save, void* dX, void* dA, void* dB, void* ws,
+                       size_t ws_bytes, void* stream);
+
+/* Fused q/k/v forward (Fig. 4: the q, k and v auto-encoders read the same x).
+ * desc->d_out is the width of each projection; desc->r the rank of each.
+ *   A_qkv [3r x d_in] (ld_a) = [A_q; A_k; A_v] stacked by rows: one GEMM with
+ *   N = 3r reads X once and writes Z_qkv [n x 3r] = [Z_q Z_k Z_v] and (COLA)
+ *   H_qkv [n x 3r]; then Y_j = H_j B_j^T for j in q, k, v (Y_j pitch ld_y).
+ * H_qkv must be NULL under COLA_M. */
+cola_status_t cola_fwd_qkv_fused(const cola_desc_t* desc, const void* X, const void* A_qkv, const void* B_q,
+                                 const void* B_k, const void* B_v, void* Y_q, void* Y_k, void* Y_v,
+                                 void* Z_qkv, void* H_qkv, void* ws, size_t ws_bytes, void* stream);
+
+/* Fused q/k/v backward: three dZ_j = (dY_j B_j) * sigma'(Z_j) into one
+ * [n x 3r] buffer, then one GEMM with M = 3r gives dA_qkv [3r x d_in] (ld_a),
+ * one GEMM with K = 3r gives dX = sum_j dZ_j A_j (ld_x), and dB_j = dY_j^T H_j.
+ * H_qkv must be NULL under COLA_M. */
+cola_status_t cola_bwd_qkv_fused(const cola_desc_t* desc, const void* X, const void* A_qkv, const void* B_q,
+                                 const void* B_k, const void* B_v, const void* dY_q, const void* dY_k,
+                                 const void* dY_v, const void* Z_qkv, const void* H_qkv, void* dX, void* dA_qkv,
+                                 void* dB_q, void* dB_k, void* dB_v, void* ws, size_t ws_bytes, void* stream);
+
+/* Synchronise `stream`, read and clear the workspace status word.
+ * Returns COLA_OK, or COLA_ERR_DEVICE_TIMEOUT if a kernel that used this
+ * workspace gave up on a wait since the last check (*code_out, if not NULL,
+ * receives the raw status bits), or COLA_ERR_LAUNCH on a CUDA error. */
+cola_status_t cola_check_status(void* ws, void* stream, uint32_t* code_out);
+
+/* Static description of a status code. */
+const char* cola_status_string(cola_status_t status);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* COLA_H */

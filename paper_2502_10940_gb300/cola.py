@@ -1,0 +1,177 @@
+"""Thin ctypes binding of libcola.so (include/cola.h), same names as the C ABI.
+
+Argument marshalling only: tensors become device pointers, the stream
+defaults to torch's current CUDA stream, and a non-OK status raises
+ColaError.  Every step of the layer runs in the library's kernels; there is
+no fallback of any kind -- if libcola.so is missing or cannot load, every
+call raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import torch
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libcola.so")
+
+SIGMA = {"identity": 0, "silu": 1, "gelu": 2}
+MODE = {"cola": 0, "cola_m": 1}
+STATUS = {0: "COLA_OK", 1: "COLA_ERR_INVALID", 2: "COLA_ERR_ALIGN", 3: "COLA_ERR_UNSUPPORTED",
+          4: "COLA_ERR_WORKSPACE", 5: "COLA_ERR_LAUNCH", 6: "COLA_ERR_DEVICE_TIMEOUT"}
+
+# the entry points include/cola.h declares
+SYMBOLS = ("cola_workspace_size", "cola_workspace_init", "cola_fwd", "cola_bwd", "cola_fwd_qkv_fused",
+           "cola_bwd_qkv_fused", "cola_check_status", "cola_status_string")
+
+
+class ColaError(RuntimeError):
+    def __init__(self, status: int, where: str):
+        self.status = int(status)
+        super().__init__(f"{where}: {STATUS.get(self.status, self.status)} ({_status_text(self.status)})")
+
+
+class cola_desc_t(ctypes.Structure):
+    _fields_ = [("n", ctypes.c_int64), ("d_in", ctypes.c_int64), ("d_out", ctypes.c_int64),
+                ("r", ctypes.c_int64), ("ld_x", ctypes.c_int64), ("ld_y", ctypes.c_int64),
+                ("ld_a", ctypes.c_int64), ("sigma", ctypes.c_int32), ("mode", ctypes.c_int32),
+                ("wgrad_fp32", ctypes.c_int32), ("reserved", ctypes.c_int32)]
+
+
+_lib = None
+_vp = ctypes.c_void_p
+
+
+def lib():
+    """Load libcola.so (once).  Raises if it is missing: there is no fallback."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(LIB_PATH):
+            raise RuntimeError(f"{LIB_PATH} is missing: build it with paper_2502_10940_gb300.build.build()")
+        l = ctypes.CDLL(LIB_PATH)
+        D = ctypes.POINTER(cola_desc_t)
+        st = ctypes.c_int
+        l.cola_workspace_size.argtypes = [D, ctypes.c_int, ctypes.POINTER(ctypes.c_size_t)]
+        l.cola_workspace_size.restype = st
+        l.cola_workspace_init.argtypes = [_vp, _vp]
+        l.cola_workspace_init.restype = st
+        l.cola_fwd.argtypes = [D] + [_vp] * 7 + [ctypes.c_size_t, _vp]
+        l.cola_fwd.restype = st
+        l.cola_bwd.argtypes = [D] + [_vp] * 10 + [ctypes.c_size_t, _vp]
+        l.cola_bwd.restype = st
+        l.cola_fwd_qkv_fused.argtypes = [D] + [_vp] * 11 + [ctypes.c_size_t, _vp]
+        l.cola_fwd_qkv_fused.restype = st
+        l.cola_bwd_qkv_fused.argtypes = [D] + [_vp] * 16 + [ctypes.c_size_t, _vp]
+        l.cola_bwd_qkv_fused.restype = st
+        l.cola_check_status.argtypes = [_vp, _vp, ctypes.POINTER(ctypes.c_uint32)]
+        l.cola_check_status.restype = st
+        l.cola_status_string.argtypes = [ctypes.c_int]
+        l.cola_status_string.restype = ctypes.c_char_p
+        _lib = l
+    return _lib
+
+
+def _status_text(status: int) -> str:
+    try:
+        return lib().cola_status_string(int(status)).decode()
+    except Exception:  # noqa: BLE001 -- only used to word an error message
+        return "?"
+
+
+def _check(status: int, where: str):
+    if status != 0:
+        raise ColaError(status, where)
+
+
+def desc(n, d_in, d_out, r, ld_x=0, ld_y=0, ld_a=0, sigma="silu", mode="cola", wgrad_fp32=False):
+    d = cola_desc_t()
+    d.n, d.d_in, d.d_out, d.r = int(n), int(d_in), int(d_out), int(r)
+    d.ld_x, d.ld_y, d.ld_a = int(ld_x), int(ld_y), int(ld_a)
+    d.sigma = SIGMA[sigma] if isinstance(sigma, str) else int(sigma)
+    d.mode = MODE[mode] if isinstance(mode, str) else int(mode)
+    d.wgrad_fp32 = int(bool(wgrad_fp32))
+    d.reserved = 0
+    return d
+
+
+def _ptr(t):
+    if t is None:
+        return None
+    if isinstance(t, int):
+        return t
+    return t.data_ptr()
+
+
+def _stream(s):
+    if s is None:
+        return torch.cuda.current_stream().cuda_stream
+    if isinstance(s, int):
+        return s
+    return s.cuda_stream
+
+
+def _nbytes(ws):
+    return ws.numel() * ws.element_size()
+
+
+def cola_workspace_size(d: cola_desc_t, fused_qkv: int = 0) -> int:
+    out = ctypes.c_size_t(0)
+    _check(lib().cola_workspace_size(ctypes.byref(d), int(fused_qkv), ctypes.byref(out)), "cola_workspace_size")
+    return int(out.value)
+
+
+def cola_workspace_init(ws, stream=None):
+    _check(lib().cola_workspace_init(_ptr(ws), _stream(stream)), "cola_workspace_init")
+
+
+def cola_fwd(d, X, A, B, Y, Z_save, H_save, ws, stream=None):
+    _check(lib().cola_fwd(ctypes.byref(d), _ptr(X), _ptr(A), _ptr(B), _ptr(Y), _ptr(Z_save), _ptr(H_save),
+                          _ptr(ws), _nbytes(ws), _stream(stream)), "cola_fwd")
+
+
+def cola_bwd(d, X, A, B, dY, Z_save, H_save, dX, dA, dB, ws, stream=None):
+    _check(lib().cola_bwd(ctypes.byref(d), _ptr(X), _ptr(A), _ptr(B), _ptr(dY), _ptr(Z_save), _ptr(H_save),
+                          _ptr(dX), _ptr(dA), _ptr(dB), _ptr(ws), _nbytes(ws), _stream(stream)), "cola_bwd")
+
+
+def cola_fwd_qkv_fused(d, X, A_qkv, B_q, B_k, B_v, Y_q, Y_k, Y_v, Z_qkv, H_qkv, ws, stream=None):
+    _check(lib().cola_fwd_qkv_fused(ctypes.byref(d), _ptr(X), _ptr(A_qkv), _ptr(B_q), _ptr(B_k), _ptr(B_v),
+                                    _ptr(Y_q), _ptr(Y_k), _ptr(Y_v), _ptr(Z_qkv), _ptr(H_qkv), _ptr(ws),
+                                    _nbytes(ws), _stream(stream)), "cola_fwd_qkv_fused")
+
+
+def cola_bwd_qkv_fused(d, X, A_qkv, B_q, B_k, B_v, dY_q, dY_k, dY_v, Z_qkv, H_qkv, dX, dA_qkv, dB_q, dB_k, dB_v,
+                       ws, stream=None):
+    _check(lib().cola_bwd_qkv_fused(ctypes.byref(d), _ptr(X), _ptr(A_qkv), _ptr(B_q), _ptr(B_k), _ptr(B_v),
+                                    _ptr(dY_q), _ptr(dY_k), _ptr(dY_v), _ptr(Z_qkv), _ptr(H_qkv), _ptr(dX),
+                                    _ptr(dA_qkv), _ptr(dB_q), _ptr(dB_k), _ptr(dB_v), _ptr(ws), _nbytes(ws),
+                                    _stream(stream)), "cola_bwd_qkv_fused")
+
+
+def cola_check_status(ws, stream=None):
+    """Returns (status, raw code); does not raise on a device timeout."""
+    code = ctypes.c_uint32(0)
+    st = lib().cola_check_status(_ptr(ws), _stream(stream), ctypes.byref(code))
+    return int(st), int(code.value)
+
+
+def cola_status_string(status: int) -> str:
+    return lib().cola_status_string(int(status)).decode()
+
+
+# ---------------------------------------------------------------- helpers
+def ld_of(t) -> int:
+    """Row pitch (elements) of a 2-D row-major tensor view."""
+    assert t.dim() == 2 and t.stride(1) == 1
+    return int(t.stride(0))
+
+
+def workspace(d: cola_desc_t, fused_qkv: int = 0, device="cuda"):
+    """A zero-initialised workspace tensor for `d` (allocated by torch)."""
+    nbytes = cola_workspace_size(d, fused_qkv)
+    ws = torch.empty(nbytes + 256, dtype=torch.uint8, device=device)
+    off = (-ws.data_ptr()) % 256
+    ws = ws[off:off + nbytes]
+    cola_workspace_init(ws)
+    return ws

@@ -1,0 +1,16 @@
+// Backward activation-gradient GEMMs: dZ = (dY B) * sigma'(Z) (EPI_DSIGMA) and
+// dX = dZ A (EPI_STORE); A operand K-major, B operand (a weight read
+// transposed) MN-major.
+#define COLA_DEFINE_LAUNCHERS
+#include "gemm_launch.cuh"
+
+namespace cola {
+template cudaError_t launch_gemm<128, false, true, EPI_DSIGMA>(const CUtensorMap&, const CUtensorMap&,
+                                                               const GemmParams&, int, cudaStream_t);
+template cudaError_t launch_gemm<256, false, true, EPI_DSIGMA>(const CUtensorMap&, const CUtensorMap&,
+                                                               const GemmParams&, int, cudaStream_t);
+template cudaError_t launch_gemm<128, false, true, EPI_STORE>(const CUtensorMap&, const CUtensorMap&,
+                                                              const GemmParams&, int, cudaStream_t);
+template cudaError_t launch_gemm<256, false, true, EPI_STORE>(const CUtensorMap&, const CUtensorMap&,
+                                                              const GemmParams&, int, cudaStream_t);
+}  // namespace cola

@@ -1,0 +1,15 @@
+// Forward GEMMs: Z/H = sigma-epilogue of X A^T (EPI_ZH) and Y = H B^T (EPI_STORE);
+// both operands K-major.
+#define COLA_DEFINE_LAUNCHERS
+#include "gemm_launch.cuh"
+
+namespace cola {
+template cudaError_t launch_gemm<128, false, false, EPI_ZH>(const CUtensorMap&, const CUtensorMap&,
+                                                            const GemmParams&, int, cudaStream_t);
+template cudaError_t launch_gemm<256, false, false, EPI_ZH>(const CUtensorMap&, const CUtensorMap&,
+                                                            const GemmParams&, int, cudaStream_t);
+template cudaError_t launch_gemm<128, false, false, EPI_STORE>(const CUtensorMap&, const CUtensorMap&,
+                                                               const GemmParams&, int, cudaStream_t);
+template cudaError_t launch_gemm<256, false, false, EPI_STORE>(const CUtensorMap&, const CUtensorMap&,
+                                                               const GemmParams&, int, cudaStream_t);
+}  // namespace cola

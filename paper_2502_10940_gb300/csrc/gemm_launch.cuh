@@ -1,0 +1,40 @@
+// gemm_launch.cuh -- host-side launcher of the GEMM kernel template.  The
+// kernel translation units (gemm_*.cu) instantiate it explicitly; the ABI
+// translation unit only sees the declarations.
+#pragma once
+#include <cuda_runtime.h>
+
+#include "gemm.cuh"
+
+namespace cola {
+
+template <int BN, bool A_MN, bool B_MN, int EPI>
+cudaError_t launch_gemm(const CUtensorMap& map_a, const CUtensorMap& map_b, const GemmParams& p, int grid,
+                        cudaStream_t stream);
+
+cudaError_t launch_splitk_reduce(const float* part, int splits, long long part_stride, int ldp, int M, int N,
+                                 void* out, long long ldo, int accumulate_f32, int grid, cudaStream_t stream);
+
+#ifdef COLA_DEFINE_LAUNCHERS
+template <int BN, bool A_MN, bool B_MN, int EPI>
+cudaError_t launch_gemm(const CUtensorMap& map_a, const CUtensorMap& map_b, const GemmParams& p, int grid,
+                        cudaStream_t stream)
+{
+    constexpr int smem = GemmCfg<BN>::SMEM_BYTES;
+    auto kern = gemm_kernel<BN, A_MN, B_MN, EPI>;
+    // the opt-in shared-memory size is a per-device function attribute
+    static unsigned long long configured = 0;   // bit d: set on device d
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev >= 64 || !((configured >> dev) & 1ull)) {
+        e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+        if (e != cudaSuccess) return e;
+        if (dev < 64) configured |= 1ull << dev;
+    }
+    kern<<<grid, NUM_THREADS, smem, stream>>>(map_a, map_b, p);
+    return cudaGetLastError();
+}
+#endif
+
+}  // namespace cola
