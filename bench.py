@@ -1,0 +1,568 @@
+#!/usr/bin/env python3
+"""Throughput of the CoLA layer stack (forward + full backward) on GB300.
+
+One step = one pass of the whole hot path over one batch: the forward of all
+seven CoLA layers of a LLaMA-shaped block (q/k/v fused, o, gate, up, down;
+h = B sigma(A x) each, Sec. 3.2 / Fig. 4) followed by their backward
+(Sec. 3.4), every GEMM on the library's tcgen05 kernels through the C ABI.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--workload 60m|350m|1b|7b|60m-q]
+                    [--mode cola|cola_m] [--impl cola|reference]
+
+Prints ONE JSON line (rank 0).  `value` is whole-job TFLOP/s (algorithmic
+6 n r (d_in + d_out) per layer), device-timed with CUDA events, inputs
+resident in HBM; `e2e` is the same metric with each step's inputs copied
+from pinned host memory and the weight gradients copied back inside the
+timed region.  The working set of every block workload is larger than L2
+(129 MB), so no L2 flush is needed between steps.
+
+--impl reference times the fp64 CPU oracle (the only reference there is: the
+paper publishes no implementation) on the host cores, on a bounded sample of
+the same workload.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "CoLA layer fwd+bwd TFLOP/s and % of GB300 dense-BF16 peak; tokens/s per block"
+
+
+def _peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            p = json.load(f)
+        return {"hbm_gbs": float(p["hbm_gbs"]), "bf16_tflops": float(p["bf16_tflops"]),
+                "bf16_tflops_sustained": float(p.get("bf16_tflops_sustained", p["bf16_tflops"])),
+                "source": "measured"}
+    except Exception:  # noqa: BLE001 -- the file is driver-written; fall back to the recipe's figures
+        return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0, "source": "fallback"}
+
+
+# ---------------------------------------------------------------- the block
+class Block:
+    """All tensors of one CoLA block workload, resident on the device."""
+
+    def __init__(self, wl, mode, device, seed=0, sigma="silu"):
+        import torch
+
+        from paper_2502_10940_gb300 import cola
+        from paper_2502_10940_gb300 import inputs as I
+
+        self.torch, self.cola = torch, cola
+        self.wl, self.mode, self.sigma = wl, mode, sigma
+        n = wl.n
+        bf = torch.bfloat16
+        self.X = {}
+        for li, L in enumerate(wl.layers):
+            if L.x not in self.X:
+                self.X[L.x] = I.activation(n, L.d_in, seed, device, layer=100 + len(self.X))
+        names = [L.name for L in wl.layers]
+        self.qkv = wl.fused_qkv and all(k in names for k in ("q", "k", "v"))
+        self.layers = []
+        for li, L in enumerate(wl.layers):
+            t = I.layer_inputs(n, L.d_in, L.d_out, L.r, seed=seed, device=device, layer=li, with_x=False)
+            X = self.X[L.x]
+            st = dict(L=L, X=X, A=t["A"], B=t["B"], dY=t["dY"])
+            ldy = cola.ld_of(t["dY"])
+            st["Y"] = torch.empty((n, ldy), dtype=bf, device=device)[:, :L.d_out]
+            st["desc"] = cola.desc(n, L.d_in, L.d_out, L.r, ld_x=cola.ld_of(X), ld_y=ldy, ld_a=cola.ld_of(t["A"]),
+                                   sigma=sigma, mode=mode)
+            self.layers.append(st)
+        self.ws_bytes = 0
+        self.plain = [s for s in self.layers if not (self.qkv and s["L"].name in ("q", "k", "v"))]
+        for s in self.plain:
+            L = s["L"]
+            s["Z"] = torch.empty((n, L.r), dtype=bf, device=device)
+            s["H"] = torch.empty((n, L.r), dtype=bf, device=device) if mode == "cola" else None
+            ldx = cola.ld_of(s["X"])
+            s["dX"] = torch.empty((n, ldx), dtype=bf, device=device)[:, :L.d_in]
+            s["dA"] = torch.empty((L.r, ldx), dtype=bf, device=device)[:, :L.d_in]
+            s["dB"] = torch.empty((L.d_out, L.r), dtype=bf, device=device)
+            self.ws_bytes = max(self.ws_bytes, cola.cola_workspace_size(s["desc"], 0))
+        if self.qkv:
+            q = [s for s in self.layers if s["L"].name in ("q", "k", "v")]
+            self.q3 = q
+            L = q[0]["L"]
+            r3 = 3 * L.r
+            ldx = cola.ld_of(q[0]["X"])
+            A3 = torch.empty((r3, ldx), dtype=bf, device=device)[:, :L.d_in]
+            for j, s in enumerate(q):
+                A3[j * L.r:(j + 1) * L.r].copy_(s["A"])
+            self.A_qkv = A3
+            self.Z_qkv = torch.empty((n, r3), dtype=bf, device=device)
+            self.H_qkv = torch.empty((n, r3), dtype=bf, device=device) if mode == "cola" else None
+            self.dX_qkv = torch.empty((n, ldx), dtype=bf, device=device)[:, :L.d_in]
+            self.dA_qkv = torch.empty((r3, ldx), dtype=bf, device=device)[:, :L.d_in]
+            for s in q:
+                s["dB"] = torch.empty((L.d_out, L.r), dtype=bf, device=device)
+            self.ws_bytes = max(self.ws_bytes, cola.cola_workspace_size(q[0]["desc"], 1))
+        self.ws = torch.empty(self.ws_bytes, dtype=torch.uint8, device=device)
+        cola.cola_workspace_init(self.ws)
+        self.launches_per_step = None
+
+    # inputs a step consumes from outside (activations + upstream gradients)
+    def step_inputs(self):
+        return list(self.X.values()) + [s["dY"] for s in self.layers]
+
+    def step_results(self):
+        out = [s["dA"] for s in self.plain] + [s["dB"] for s in self.layers]
+        if self.qkv:
+            out.append(self.dA_qkv)
+        return out
+
+    def forward(self):
+        c = self.cola
+        if self.qkv:
+            q, k, v = self.q3
+            c.cola_fwd_qkv_fused(q["desc"], q["X"], self.A_qkv, q["B"], k["B"], v["B"], q["Y"], k["Y"], v["Y"],
+                                 self.Z_qkv, self.H_qkv, self.ws)
+        for s in self.plain:
+            c.cola_fwd(s["desc"], s["X"], s["A"], s["B"], s["Y"], s["Z"], s["H"], self.ws)
+
+    def backward(self):
+        c = self.cola
+        for s in reversed(self.plain):
+            c.cola_bwd(s["desc"], s["X"], s["A"], s["B"], s["dY"], s["Z"], s["H"], s["dX"], s["dA"], s["dB"],
+                       self.ws)
+        if self.qkv:
+            q, k, v = self.q3
+            c.cola_bwd_qkv_fused(q["desc"], q["X"], self.A_qkv, q["B"], k["B"], v["B"], q["dY"], k["dY"], v["dY"],
+                                 self.Z_qkv, self.H_qkv, self.dX_qkv, self.dA_qkv, q["dB"], k["dB"], v["dB"],
+                                 self.ws)
+
+    def step(self):
+        self.forward()
+        self.backward()
+
+    def check(self):
+        st, code = self.cola.cola_check_status(self.ws)
+        if st != 0:
+            raise RuntimeError(f"device status {st} (code {code:#x})")
+
+    def working_set_bytes(self):
+        t = self.torch
+        seen, total = set(), 0
+        for obj in vars(self).values():
+            items = obj if isinstance(obj, list) else [obj]
+            for it in items:
+                vals = it.values() if isinstance(it, dict) else [it]
+                for v in vals:
+                    if isinstance(v, t.Tensor) and v.is_cuda and v.data_ptr() not in seen:
+                        seen.add(v.data_ptr())
+                        total += v.untyped_storage().nbytes()
+        return total
+
+
+# ---------------------------------------------------------------- per-launch accounting
+def launch_cost(kind, m, n, k, splits, flags):
+    """(algorithmic bytes, flops) of one library launch: each operand read once,
+    each result written once, bf16 (2 B); the fp32 token-split partials of the
+    weight gradients are implementation traffic and are not counted."""
+    e = 2
+    if kind == "fwd_zh":
+        return e * (m * k + n * k + m * n * (2 if flags & 1 else 1)), 2.0 * m * n * k
+    if kind == "fwd_y":
+        return e * (m * k + n * k + m * n), 2.0 * m * n * k
+    if kind == "bwd_dz":
+        return e * (m * k + n * k + m * n * (3 if flags & 1 else 2)), 2.0 * m * n * k
+    if kind in ("wgrad_db", "wgrad_da"):
+        return e * (k * m + k * n + m * n), 2.0 * m * n * k
+    if kind == "bwd_dx":
+        return e * (m * k + n * k + m * n), 2.0 * m * n * k
+    if kind == "reduce":
+        return e * m * n, 0.0
+    return 0, 0.0
+
+
+def summarize_trace(records, peaks, ridge):
+    kinds = {}
+    for kind, m, n, k, splits, flags, ms in records:
+        b, f = launch_cost(kind, m, n, k, splits, flags)
+        d = kinds.setdefault(kind, {"launches": 0, "ms": 0.0, "bytes": 0.0, "flops": 0.0})
+        d["launches"] += 1
+        d["ms"] += ms
+        d["bytes"] += b
+        d["flops"] += f
+    total = sum(d["ms"] for d in kinds.values()) or 1.0
+    for d in kinds.values():
+        d["share"] = d["ms"] / total
+    top = max(kinds, key=lambda x: kinds[x]["ms"])
+    d = kinds[top]
+    t = d["ms"] / 1e3
+    intensity = d["flops"] / max(d["bytes"], 1.0)
+    if intensity >= ridge:
+        achieved = d["flops"] / t / 1e12
+        peak = peaks["bf16_tflops_sustained"]
+        roof = {"bound": "tensor", "unit": "TFLOP/s"}
+    else:
+        achieved = d["bytes"] / t / 1e9
+        peak = peaks["hbm_gbs"]
+        roof = {"bound": "hbm", "unit": "GB/s"}
+    roof.update({"kernel": f"gemm {top}", "achieved": round(achieved, 1), "peak": peak,
+                 "frac": round(achieved / peak, 4), "peak_source": peaks["source"],
+                 "launches": d["launches"], "avg_launch_us": round(d["ms"] * 1e3 / d["launches"], 2),
+                 "algorithmic_bytes_per_launch": int(d["bytes"] / d["launches"]),
+                 "flop_per_launch": d["flops"] / d["launches"], "share": round(d["share"], 4)})
+    return roof, {k: {"launches": v["launches"], "share": round(v["share"], 4),
+                      "avg_us": round(v["ms"] * 1e3 / v["launches"], 2),
+                      "gbs": round(v["bytes"] / (v["ms"] / 1e3) / 1e9, 1),
+                      "tflops": round(v["flops"] / (v["ms"] / 1e3) / 1e12, 1)} for k, v in kinds.items()}
+
+
+def traffic_from_profile(kernel_key, workload):
+    """dram bytes per launch from a committed ncu summary, valid only while the
+    kernel sources are unchanged (hash match); else None."""
+    import hashlib
+
+    path = os.path.join(ROOT, "profiles", "ncu_traffic.json")
+    if not os.path.exists(path):
+        return None
+    try:
+        with open(path) as f:
+            rec = json.load(f)
+        h = hashlib.sha256()
+        for name in ("gemm.cuh", "ptx.cuh"):
+            with open(os.path.join(ROOT, "paper_2502_10940_gb300", "csrc", name), "rb") as g:
+                h.update(g.read())
+        entry = rec.get(workload, {}).get(kernel_key)
+        if entry and entry.get("src_sha256") == h.hexdigest():
+            return entry["dram_bytes_per_launch"]
+    except Exception:  # noqa: BLE001 -- a missing or stale summary means "no traffic figure"
+        return None
+    return None
+
+
+# ---------------------------------------------------------------- clocks
+class ClockSampler:
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, device_index):
+        self.proc = None
+        self.dev = device_index
+
+    def start(self):
+        try:
+            import torch
+            uuid = None
+            try:
+                uuid = str(torch.cuda.get_device_properties(self.dev).uuid)
+                if uuid and not uuid.startswith("GPU-"):
+                    uuid = "GPU-" + uuid
+            except Exception:  # noqa: BLE001
+                uuid = None
+            sel = ["-i", uuid] if uuid else []
+            self.proc = subprocess.Popen(["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                                          "-lms", "100"] + sel, stdout=subprocess.PIPE, stderr=subprocess.DEVNULL,
+                                         text=True)
+        except Exception:  # noqa: BLE001 -- no nvidia-smi: clocks are reported as unknown
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"], "samples": 0}
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=5)
+        except Exception:  # noqa: BLE001
+            self.proc.kill()
+            out, _ = self.proc.communicate()
+        sm, mx, pw, reasons = [], [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in out.splitlines():
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 7:
+                continue
+            try:
+                sm.append(float(parts[0]))
+                mx.append(float(parts[1]))
+                pw.append(float(parts[2]))
+            except ValueError:
+                continue
+            for nm, v in zip(names, parts[3:7]):
+                if v.lower().startswith("active"):
+                    reasons.add(nm)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"], "samples": 0}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "power_w_max": max(pw), "samples": len(sm)}
+
+
+# ---------------------------------------------------------------- CPU oracle
+def oracle_block_sample(wl, n_s, seed=0):
+    """The whole block (7 layers, fwd + bwd) through the fp64 oracle on n_s
+    tokens of the same synthetic distribution.  Returns (seconds, flops)."""
+    import oracle
+    from paper_2502_10940_gb300 import inputs as I
+    from paper_2502_10940_gb300.workloads import layer_flops
+
+    xs = {}
+    for L in wl.layers:
+        if L.x not in xs:
+            xs[L.x] = I.activation(n_s, L.d_in, seed, "cpu", layer=100 + len(xs)).float().double().numpy()
+    prepared = []
+    for li, L in enumerate(wl.layers):
+        t = I.layer_inputs(n_s, L.d_in, L.d_out, L.r, seed=seed, device="cpu", layer=li, with_x=False)
+        prepared.append((xs[L.x], t["A"].float().double().numpy(), t["B"].float().double().numpy(),
+                         t["dY"].float().double().numpy()))
+    t0 = time.perf_counter()
+    for X, A, B, dY in prepared:
+        Z, H, Y = oracle.fwd(X, A, B, "silu")
+        oracle.bwd(X, A, B, dY, Z, H, "silu", "cola")
+    dt = time.perf_counter() - t0
+    return dt, float(sum(layer_flops(n_s, L.d_in, L.d_out, L.r) for L in wl.layers))
+
+
+def calibrate_tokens(wl, target_s):
+    n_s, dt = 64, 0.0
+    while True:
+        dt, _ = oracle_block_sample(wl, n_s)
+        if dt >= 0.5 or n_s >= wl.n:
+            break
+        n_s *= 2
+    return max(16, min(wl.n, int(n_s * target_s / max(dt, 1e-6)) // 16 * 16))
+
+
+def cpu_baseline(wl, target_s=10.0):
+    import oracle
+
+    n_s = calibrate_tokens(wl, target_s)
+    dt, fl = oracle_block_sample(wl, n_s)
+    return {"value": round(fl / dt / 1e12, 6), "unit": "TFLOP/s", "cores": oracle.num_threads(), "kind": "oracle",
+            "sample": f"{wl.name} block, all {len(wl.layers)} layers fwd+bwd on {n_s} of {wl.n} tokens "
+                      f"({dt:.1f} s, fp64 loops, OpenMP)"}
+
+
+# ---------------------------------------------------------------- arms
+def run_reference(args, wl):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return 0
+    import oracle
+
+    budget = 150.0  # seconds for warmup + steps
+    per_step = max(0.5, min(10.0, budget / max(1, args.steps + args.warmup)))
+    n_s = calibrate_tokens(wl, per_step)
+    for _ in range(args.warmup):
+        oracle_block_sample(wl, n_s)
+    tot_t, tot_f = 0.0, 0.0
+    for _ in range(args.steps):
+        dt, fl = oracle_block_sample(wl, n_s)
+        tot_t += dt
+        tot_f += fl
+    value = tot_f / tot_t / 1e12
+    sample = f"{wl.name} block, all {len(wl.layers)} layers fwd+bwd on {n_s} of {wl.n} tokens per step"
+    line = {"impl": "reference", "metric": METRIC, "value": round(value, 6), "unit": "TFLOP/s", "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(tot_t / args.steps * 1e3, 3),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "config": {"workload": wl.desc, "n_tokens_sampled": n_s, "mode": "cola"},
+            "cpu_baseline": {"value": round(value, 6), "unit": "TFLOP/s", "cores": oracle.num_threads(),
+                             "kind": "oracle", "sample": sample},
+            "e2e": {"value": round(value, 6), "unit": "TFLOP/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def time_steps(fn, steps, stream, dist=None):
+    import torch
+
+    if dist:
+        dist.barrier()
+    torch.cuda.synchronize()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(steps):
+        fn()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    if dist:
+        dist.barrier()
+    ms = e0.elapsed_time(e1) / steps
+    if dist:
+        t = torch.tensor([ms], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    return ms
+
+
+def full_rank_baseline(wl, device, steps, warmup, seed=0):
+    """Same-shape full-rank layers (fwd Y = X W^T, bwd dX = dY W, dW = dY^T X)
+    with torch.matmul (cuBLAS), q/k/v fused as one N = 3d GEMM."""
+    import torch
+
+    n = wl.n
+    bf = torch.bfloat16
+    g = torch.Generator(device=device).manual_seed(seed + 77)
+    groups = {}
+    for L in wl.layers:
+        key = "qkv" if (wl.fused_qkv and L.name in ("q", "k", "v")) else L.name
+        groups.setdefault(key, []).append(L)
+    bufs = []
+    flops = 0.0
+    for key, Ls in groups.items():
+        d_in = Ls[0].d_in
+        d_out = sum(L.d_out for L in Ls)
+        X = torch.randn((n, d_in), generator=g, device=device, dtype=torch.float32).to(bf)
+        W = (torch.randn((d_out, d_in), generator=g, device=device, dtype=torch.float32) * d_in ** -0.5).to(bf)
+        dY = torch.randn((n, d_out), generator=g, device=device, dtype=torch.float32).to(bf)
+        bufs.append(dict(X=X, W=W, dY=dY, Y=torch.empty((n, d_out), dtype=bf, device=device),
+                         dX=torch.empty((n, d_in), dtype=bf, device=device),
+                         dW=torch.empty((d_out, d_in), dtype=bf, device=device)))
+        flops += 6.0 * n * d_in * d_out
+
+    def step():
+        for b in bufs:
+            torch.matmul(b["X"], b["W"].t(), out=b["Y"])
+        for b in reversed(bufs):
+            torch.matmul(b["dY"], b["W"], out=b["dX"])
+            torch.matmul(b["dY"].t(), b["X"], out=b["dW"])
+
+    for _ in range(warmup):
+        step()
+    ms = time_steps(step, steps, torch.cuda.current_stream())
+    del bufs
+    return {"ms_per_step": round(ms, 4), "tflops": round(flops / (ms / 1e3) / 1e12, 1), "flops": flops,
+            "impl": "torch.matmul (cuBLAS) bf16"}
+
+
+def run_cola(args, wl):
+    import torch
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    dist = None
+    if world > 1:
+        import torch.distributed as dist_mod
+        dist_mod.init_process_group("nccl")
+        dist = dist_mod
+    torch.cuda.set_device(local)
+    device = f"cuda:{local}"
+
+    from paper_2502_10940_gb300 import build
+    from paper_2502_10940_gb300 import cola
+
+    build.build()
+    peaks = _peaks()
+    ridge = peaks["bf16_tflops"] * 1e12 / (peaks["hbm_gbs"] * 1e9)
+    mode = args.mode or wl.modes[0]
+    blk = Block(wl, mode, device, seed=args.seed + rank)
+    stream = torch.cuda.current_stream()
+
+    # launches per step, counted by the library's trace
+    with cola.Trace(512) as tr:
+        blk.step()
+    blk.launches_per_step = tr.count.value
+    blk.check()
+
+    sampler = ClockSampler(local)
+    sampler.start()
+    for _ in range(args.warmup):
+        blk.step()
+    torch.cuda.synchronize()
+    ms = time_steps(blk.step, args.steps, stream, dist)
+    clocks = sampler.stop()
+    blk.check()
+
+    # the same steps again with every launch bracketed by events: per-kernel times
+    cap = blk.launches_per_step * args.steps
+    with cola.Trace(cap) as tr:
+        time_steps(blk.step, args.steps, stream)
+    records = tr.records()
+    roofline, kinds = summarize_trace(records, peaks, ridge)
+    roofline["traffic"] = traffic_from_profile(roofline["kernel"], wl.name)
+
+    flops = wl.flops
+    value = flops * world / (ms / 1e3) / 1e12
+    line = {"metric": METRIC, "value": round(value, 2), "unit": "TFLOP/s", "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": round(ms, 4), "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+            "config": {"workload": wl.desc, "n_tokens": wl.n, "mode": mode, "sigma": "silu",
+                       "layers": [f"{L.name}:{L.d_in}->{L.d_out},r={L.r}" for L in wl.layers],
+                       "fused_qkv": blk.qkv, "parallelism": "replicas" if world > 1 else "single-gpu",
+                       "l2": f"no flush: working set {blk.working_set_bytes() / 1e9:.2f} GB > 129 MB L2"},
+            "tokens_per_s": round(wl.n * world / (ms / 1e3), 1),
+            "pct_dense_bf16_peak": round(100.0 * value / world / peaks["bf16_tflops"], 2),
+            "pct_dense_bf16_peak_sustained": round(100.0 * value / world / peaks["bf16_tflops_sustained"], 2),
+            "roofline": roofline, "kernels": kinds,
+            "gpu_launches": blk.launches_per_step * args.steps, "clocks": clocks}
+
+    if not args.no_extras:
+        # end to end: each step's activations and upstream gradients come from
+        # pinned host memory; the weight gradients go back to pinned host memory
+        def full_rows(t):   # the whole padded row-major buffer behind a view
+            return torch.as_strided(t, (t.shape[0], t.stride(0)), (t.stride(0), 1))
+
+        ins = [full_rows(t) for t in blk.step_inputs()]
+        outs = [full_rows(t) for t in blk.step_results()]
+        h_in = [torch.empty(t.shape, dtype=t.dtype, pin_memory=True) for t in ins]
+        for h, t in zip(h_in, ins):
+            h.copy_(t)
+        h_out = [torch.empty(t.shape, dtype=t.dtype, pin_memory=True) for t in outs]
+
+        def e2e_step():
+            for h, t in zip(h_in, ins):
+                t.copy_(h, non_blocking=True)
+            blk.step()
+            for h, t in zip(h_out, outs):
+                h.copy_(t, non_blocking=True)
+
+        for _ in range(max(1, args.warmup // 2)):
+            e2e_step()
+        e2e_steps = max(3, args.steps // 2)
+        ms_e2e = time_steps(e2e_step, e2e_steps, stream, dist)
+        blk.check()
+        bi = sum(t.numel() * t.element_size() for t in ins)
+        bo = sum(t.numel() * t.element_size() for t in outs)
+        line["e2e"] = {"value": round(flops * world / (ms_e2e / 1e3) / 1e12, 2), "unit": "TFLOP/s",
+                       "ms_per_step": round(ms_e2e, 4), "steps": e2e_steps, "h2d_bytes_per_step": bi,
+                       "d2h_bytes_per_step": bo}
+        del h_in, h_out
+        if rank == 0 and world == 1:
+            fr = full_rank_baseline(wl, device, max(3, args.steps // 2), 2, seed=args.seed)
+            fr["speedup_cola_vs_full_rank"] = round(fr["ms_per_step"] / ms, 3)
+            line["full_rank"] = fr
+            line["cpu_baseline"] = cpu_baseline(wl)
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if dist:
+        dist.destroy_process_group()
+    return 0
+
+
+def main(argv=None):
+    from paper_2502_10940_gb300.workloads import WORKLOADS
+
+    ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="cola", choices=["cola", "reference"])
+    ap.add_argument("--workload", default="60m", choices=sorted(WORKLOADS))
+    ap.add_argument("--mode", default=None, choices=["cola", "cola_m"])
+    ap.add_argument("--seed", type=int, default=0)
+    ap.add_argument("--no-extras", action="store_true", help="skip e2e, full-rank and CPU baselines")
+    args = ap.parse_args(argv)
+    args.warmup = max(3, args.warmup)   # at least 3 untimed warm-up steps, always
+    args.steps = max(1, args.steps)
+    wl = WORKLOADS[args.workload]
+    if args.impl == "reference":
+        return run_reference(args, wl)
+    return run_cola(args, wl)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -23,7 +23,9 @@ STATUS = {0: "COLA_OK", 1: "COLA_ERR_INVALID", 2: "COLA_ERR_ALIGN", 3: "COLA_ERR
 
 # the entry points include/cola.h declares
 SYMBOLS = ("cola_workspace_size", "cola_workspace_init", "cola_fwd", "cola_bwd", "cola_fwd_qkv_fused",
-           "cola_bwd_qkv_fused", "cola_check_status", "cola_status_string")
+           "cola_bwd_qkv_fused", "cola_check_status", "cola_trace_attach", "cola_trace_detach",
+           "cola_status_string")
+KERNELS = {0: "fwd_zh", 1: "fwd_y", 2: "bwd_dz", 3: "wgrad_db", 4: "wgrad_da", 5: "reduce", 6: "bwd_dx"}
 
 
 class ColaError(RuntimeError):
@@ -37,6 +39,12 @@ class cola_desc_t(ctypes.Structure):
                 ("r", ctypes.c_int64), ("ld_x", ctypes.c_int64), ("ld_y", ctypes.c_int64),
                 ("ld_a", ctypes.c_int64), ("sigma", ctypes.c_int32), ("mode", ctypes.c_int32),
                 ("wgrad_fp32", ctypes.c_int32), ("reserved", ctypes.c_int32)]
+
+
+class cola_trace_slot_t(ctypes.Structure):
+    _fields_ = [("start", ctypes.c_void_p), ("stop", ctypes.c_void_p), ("kernel", ctypes.c_int32),
+                ("m", ctypes.c_int32), ("n", ctypes.c_int32), ("k", ctypes.c_int32), ("splits", ctypes.c_int32),
+                ("flags", ctypes.c_int32)]
 
 
 _lib = None
@@ -66,6 +74,11 @@ def lib():
         l.cola_bwd_qkv_fused.restype = st
         l.cola_check_status.argtypes = [_vp, _vp, ctypes.POINTER(ctypes.c_uint32)]
         l.cola_check_status.restype = st
+        l.cola_trace_attach.argtypes = [ctypes.POINTER(cola_trace_slot_t), ctypes.c_int32,
+                                        ctypes.POINTER(ctypes.c_int32)]
+        l.cola_trace_attach.restype = st
+        l.cola_trace_detach.argtypes = []
+        l.cola_trace_detach.restype = st
         l.cola_status_string.argtypes = [ctypes.c_int]
         l.cola_status_string.restype = ctypes.c_char_p
         _lib = l
@@ -158,6 +171,52 @@ def cola_check_status(ws, stream=None):
 
 def cola_status_string(status: int) -> str:
     return lib().cola_status_string(int(status)).decode()
+
+
+def cola_trace_attach(slots, capacity: int, count):
+    _check(lib().cola_trace_attach(slots, int(capacity), ctypes.byref(count)), "cola_trace_attach")
+
+
+def cola_trace_detach():
+    _check(lib().cola_trace_detach(), "cola_trace_detach")
+
+
+class Trace:
+    """Context manager: while active, every library launch is bracketed by a
+    pair of torch CUDA events (timing enabled) recorded on its stream."""
+
+    def __init__(self, capacity: int):
+        self.capacity = int(capacity)
+        self.events = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+                       for _ in range(self.capacity)]
+        for a, b in self.events:        # events are created lazily on first record
+            a.record()
+            b.record()
+        self.slots = (cola_trace_slot_t * max(self.capacity, 1))()
+        for i, (a, b) in enumerate(self.events):
+            self.slots[i].start = a.cuda_event
+            self.slots[i].stop = b.cuda_event
+        self.count = ctypes.c_int32(0)
+
+    def __enter__(self):
+        torch.cuda.synchronize()
+        cola_trace_attach(self.slots, self.capacity, self.count)
+        return self
+
+    def __exit__(self, *exc):
+        cola_trace_detach()
+        return False
+
+    def records(self):
+        """[(kernel name, m, n, k, splits, flags, ms)] of the recorded launches."""
+        torch.cuda.synchronize()
+        out = []
+        for i in range(self.count.value):
+            s_ = self.slots[i]
+            a, b = self.events[i]
+            out.append((KERNELS.get(s_.kernel, str(s_.kernel)), s_.m, s_.n, s_.k, s_.splits, s_.flags,
+                        a.elapsed_time(b)))
+        return out
 
 
 # ---------------------------------------------------------------- helpers

@@ -225,6 +225,37 @@ cola_status_t check_ws(const cola_desc_t& d, int fused, int sms, void* ws, size_
 
 inline cola_status_t launched(cudaError_t e) { return e == cudaSuccess ? COLA_OK : COLA_ERR_LAUNCH; }
 
+// ------------------------------------------------------------ launch tracing
+struct TraceState {
+    cola_trace_slot_t* slots = nullptr;
+    int32_t capacity = 0;
+    int32_t* count = nullptr;
+};
+TraceState g_trace;
+
+// Launch through `fn`, bracketed by the next free trace slot's events.
+template <class Fn>
+cudaError_t traced(int kind, int64_t m, int64_t n, int64_t k, int splits, int flags, cudaStream_t st, Fn&& fn)
+{
+    cola_trace_slot_t* slot = nullptr;
+    if (g_trace.slots && g_trace.count && *g_trace.count >= 0 && *g_trace.count < g_trace.capacity)
+        slot = &g_trace.slots[*g_trace.count];
+    cudaError_t e;
+    if (slot && (e = cudaEventRecord(static_cast<cudaEvent_t>(slot->start), st)) != cudaSuccess) return e;
+    if ((e = fn()) != cudaSuccess) return e;
+    if (slot) {
+        if ((e = cudaEventRecord(static_cast<cudaEvent_t>(slot->stop), st)) != cudaSuccess) return e;
+        slot->kernel = kind;
+        slot->m = static_cast<int32_t>(m);
+        slot->n = static_cast<int32_t>(n);
+        slot->k = static_cast<int32_t>(k);
+        slot->splits = splits;
+        slot->flags = flags;
+        ++*g_trace.count;
+    }
+    return cudaSuccess;
+}
+
 #define COLA_TRY(expr)                          \
     do {                                        \
         cola_status_t _st = (expr);             \
@@ -255,7 +286,8 @@ cola_status_t run_f1(const Shape& s, int sigma, int64_t N, const void* X, const 
     p.ldd2 = ldz;
     p.sigma = sigma;
     p.status = status;
-    return launched(dispatch<false, false, EPI_ZH>(bn, ma, mb, p, sms, st));
+    return launched(traced(COLA_KERNEL_FWD_ZH, s.n, N, s.d_in, 1, H != nullptr, st,
+                           [&] { return dispatch<false, false, EPI_ZH>(bn, ma, mb, p, sms, st); }));
 }
 
 // F2: Y = H B^T  (H [n x r] with pitch ldh)
@@ -270,7 +302,8 @@ cola_status_t run_f2(const Shape& s, const void* H, int64_t ldh, const void* B, 
     p.D = Y;
     p.ldd = s.ld_y;
     p.status = status;
-    return launched(dispatch<false, false, EPI_STORE>(bn, ma, mb, p, sms, st));
+    return launched(traced(COLA_KERNEL_FWD_Y, s.n, s.d_out, s.r, 1, 0, st,
+                           [&] { return dispatch<false, false, EPI_STORE>(bn, ma, mb, p, sms, st); }));
 }
 
 // B1: dZ = (dY B) * sigma'(Z), and H = sigma(Z) when Hout != null (CoLA-M)
@@ -290,12 +323,13 @@ cola_status_t run_b1(const Shape& s, int sigma, const void* dY, const void* B, c
     p.ldz = ldz;
     p.sigma = sigma;
     p.status = status;
-    return launched(dispatch<false, true, EPI_DSIGMA>(bn, ma, mb, p, sms, st));
+    return launched(traced(COLA_KERNEL_BWD_DZ, s.n, s.r, s.d_out, 1, Hout != nullptr, st,
+                           [&] { return dispatch<false, true, EPI_DSIGMA>(bn, ma, mb, p, sms, st); }));
 }
 
 // Weight gradient D[M x N] = sum_t P[t, m] Q[t, n] over the n tokens, both
 // operands token-major (MN-major): split over tokens, fixed-order reduce.
-cola_status_t run_wgrad(int64_t ntok, int64_t M, int64_t N, const void* P, int64_t ldp, const void* Q,
+cola_status_t run_wgrad(int kind, int64_t ntok, int64_t M, int64_t N, const void* P, int64_t ldp, const void* Q,
                         int64_t ldq, void* out, int64_t ldo, int accumulate_f32, float* part, size_t part_bytes,
                         unsigned int* status, int sms, cudaStream_t st)
 {
@@ -310,9 +344,12 @@ cola_status_t run_wgrad(int64_t ntok, int64_t M, int64_t N, const void* P, int64
     p.ldd = p.n_tiles * bn;
     p.part_stride = slab;
     p.status = status;
-    COLA_TRY(launched(dispatch<true, true, EPI_F32>(bn, ma, mb, p, sms, st)));
-    return launched(launch_splitk_reduce(part, p.splits, slab, p.n_tiles * bn, static_cast<int>(M),
-                                         static_cast<int>(N), out, ldo, accumulate_f32, sms * 4, st));
+    COLA_TRY(launched(traced(kind, M, N, ntok, p.splits, 0, st,
+                             [&] { return dispatch<true, true, EPI_F32>(bn, ma, mb, p, sms, st); })));
+    return launched(traced(COLA_KERNEL_REDUCE, M, N, p.splits, p.splits, 0, st, [&] {
+        return launch_splitk_reduce(part, p.splits, slab, p.n_tiles * bn, static_cast<int>(M), static_cast<int>(N),
+                                    out, ldo, accumulate_f32, sms * 4, st);
+    }));
 }
 
 // B4: dX = dZ A  (dZ [n x K] pitch ldz, A [K x d_in] pitch ld_a; K = r or 3r)
@@ -327,7 +364,8 @@ cola_status_t run_b4(const Shape& s, int64_t K, const void* dZ, int64_t ldz, con
     p.D = dX;
     p.ldd = s.ld_x;
     p.status = status;
-    return launched(dispatch<false, true, EPI_STORE>(bn, ma, mb, p, sms, st));
+    return launched(traced(COLA_KERNEL_BWD_DX, s.n, s.d_in, K, 1, 0, st,
+                           [&] { return dispatch<false, true, EPI_STORE>(bn, ma, mb, p, sms, st); }));
 }
 
 }  // namespace
@@ -399,8 +437,8 @@ cola_status_t cola_bwd(const cola_desc_t* desc, const void* X, const void* A, co
 
     COLA_TRY(run_b1(s, desc->sigma, dY, B, Z_save, s.r, dZ, Hrec, status, sms, st));
     const void* Hsrc = cola_m ? Hrec : H_save;
-    COLA_TRY(run_wgrad(s.n, s.d_out, s.r, dY, s.ld_y, Hsrc, s.r, dB, s.r, acc, part, part_bytes, status, sms, st));
-    COLA_TRY(run_wgrad(s.n, s.r, s.d_in, dZ, s.r, X, s.ld_x, dA, s.ld_a, acc, part, part_bytes, status, sms, st));
+    COLA_TRY(run_wgrad(COLA_KERNEL_WGRAD_DB, s.n, s.d_out, s.r, dY, s.ld_y, Hsrc, s.r, dB, s.r, acc, part, part_bytes, status, sms, st));
+    COLA_TRY(run_wgrad(COLA_KERNEL_WGRAD_DA, s.n, s.r, s.d_in, dZ, s.r, X, s.ld_x, dA, s.ld_a, acc, part, part_bytes, status, sms, st));
     return run_b4(s, s.r, dZ, s.r, A, dX, status, sms, st);
 }
 
@@ -462,10 +500,10 @@ cola_status_t cola_bwd_qkv_fused(const cola_desc_t* desc, const void* X, const v
     for (int j = 0; j < 3; ++j) {
         COLA_TRY(run_b1(s, desc->sigma, dYs[j], Bs[j], Zb + j * slice, R, dZ + j * slice,
                         Hrec ? Hrec + j * slice : nullptr, status, sms, st));
-        COLA_TRY(run_wgrad(s.n, s.d_out, s.r, dYs[j], s.ld_y, Hsrc + j * slice, R, dBs[j], s.r, acc, part,
+        COLA_TRY(run_wgrad(COLA_KERNEL_WGRAD_DB, s.n, s.d_out, s.r, dYs[j], s.ld_y, Hsrc + j * slice, R, dBs[j], s.r, acc, part,
                            part_bytes, status, sms, st));
     }
-    COLA_TRY(run_wgrad(s.n, R, s.d_in, dZ, R, X, s.ld_x, dA_qkv, s.ld_a, acc, part, part_bytes, status, sms, st));
+    COLA_TRY(run_wgrad(COLA_KERNEL_WGRAD_DA, s.n, R, s.d_in, dZ, R, X, s.ld_x, dA_qkv, s.ld_a, acc, part, part_bytes, status, sms, st));
     return run_b4(s, R, dZ, R, A_qkv, dX, status, sms, st);
 }
 
@@ -481,6 +519,23 @@ cola_status_t cola_check_status(void* ws, void* stream, uint32_t* code_out)
         if (cudaMemset(ws, 0, sizeof code) != cudaSuccess) return COLA_ERR_LAUNCH;
         return COLA_ERR_DEVICE_TIMEOUT;
     }
+    return COLA_OK;
+}
+
+cola_status_t cola_trace_attach(cola_trace_slot_t* slots, int32_t capacity, int32_t* count)
+{
+    if (!slots || !count || capacity < 0) return COLA_ERR_INVALID;
+    for (int32_t i = 0; i < capacity; ++i)
+        if (!slots[i].start || !slots[i].stop) return COLA_ERR_INVALID;
+    g_trace.slots = slots;
+    g_trace.capacity = capacity;
+    g_trace.count = count;
+    return COLA_OK;
+}
+
+cola_status_t cola_trace_detach(void)
+{
+    g_trace = TraceState{};
     return COLA_OK;
 }
 
