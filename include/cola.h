@@ -154,6 +154,42 @@ cola_status_t cola_bwd_qkv_fused(const cola_desc_t* desc, const void* X, const v
  * receives the raw status bits), or COLA_ERR_LAUNCH on a CUDA error. */
 cola_status_t cola_check_status(void* ws, void* stream, uint32_t* code_out);
 
+/* ---- weight gradient without any workspace or allocation ----
+ * The paper has no counterpart to this entry point.  It serves callers that
+ * cannot allocate device memory: an operator or plugin interface that hands
+ * the library its inputs and outputs but no workspace, or a process whose
+ * device memory is fixed at start-up by another allocator, where any later
+ * cudaMalloc would fail or break its budget.
+ *
+ *   D[M x N] = sum over t < n_tokens of P[t, m] * Q[t, n]
+ *
+ * i.e. dB = dY^T H (P = dY [n x d_out], Q = H [n x r]) or dA = dZ^T X
+ * (P = dZ [n x r], Q = X [n x d_in]), the token-reduction GEMM of cola_bwd
+ * on the same kernels.  P, Q: bf16, token-major, row pitches ld_p, ld_q
+ * (elements, multiples of 8).  D: bf16 (overwritten) or, with
+ * accumulate_f32 = 1, fp32 accumulated into (D += ...); row pitch ld_d.
+ * All pointers are device pointers, 16-byte aligned; async on `stream`.
+ *
+ * The token-split partial sums live in one static device array of
+ * COLA_STATIC_SCRATCH_BYTES inside libcola.so, which every GPU that loads
+ * the array holds until the process exits.  The entry point calls no
+ * cudaMalloc, cudaFree or other allocating routine.  A problem whose fp32
+ * partial tile grid (M and N rounded up to the tile size) does not fit the
+ * array even without a token split returns COLA_ERR_WORKSPACE before any
+ * launch.  The first call on each device fetches the array's device address
+ * (cudaGetSymbolAddress, which may load the library's device module): make
+ * that first call before any stream capture begins on the device.  Every
+ * call shares the one array, so calls that may overlap on the GPU (other
+ * streams, other host threads) race and must be serialised by the caller.
+ * Nothing in the array needs to start at zero: each call overwrites the
+ * partials it reads.  A device-side wait that runs out leaves D undefined
+ * and is not reported here (there is no workspace status word). */
+#define COLA_STATIC_SCRATCH_BYTES (64u * 1024u * 1024u)
+
+cola_status_t cola_wgrad_static_scratch(int64_t n_tokens, int64_t M, int64_t N, const void* P, int64_t ld_p,
+                                        const void* Q, int64_t ld_q, void* D, int64_t ld_d, int32_t accumulate_f32,
+                                        void* stream);
+
 /* ---- launch tracing (optional; for measurement) ----
  * While a slot array is attached, every kernel the library launches is
  * bracketed by two CUDA events recorded on the launch stream: slot

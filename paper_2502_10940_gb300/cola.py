@@ -23,8 +23,9 @@ STATUS = {0: "COLA_OK", 1: "COLA_ERR_INVALID", 2: "COLA_ERR_ALIGN", 3: "COLA_ERR
 
 # the entry points include/cola.h declares
 SYMBOLS = ("cola_workspace_size", "cola_workspace_init", "cola_fwd", "cola_bwd", "cola_fwd_qkv_fused",
-           "cola_bwd_qkv_fused", "cola_check_status", "cola_trace_attach", "cola_trace_detach",
-           "cola_status_string")
+           "cola_bwd_qkv_fused", "cola_check_status", "cola_wgrad_static_scratch", "cola_trace_attach",
+           "cola_trace_detach", "cola_status_string")
+STATIC_SCRATCH_BYTES = 64 * 1024 * 1024
 KERNELS = {0: "fwd_zh", 1: "fwd_y", 2: "bwd_dz", 3: "wgrad_db", 4: "wgrad_da", 5: "reduce", 6: "bwd_dx"}
 
 
@@ -74,6 +75,9 @@ def lib():
         l.cola_bwd_qkv_fused.restype = st
         l.cola_check_status.argtypes = [_vp, _vp, ctypes.POINTER(ctypes.c_uint32)]
         l.cola_check_status.restype = st
+        i64 = ctypes.c_int64
+        l.cola_wgrad_static_scratch.argtypes = [i64, i64, i64, _vp, i64, _vp, i64, _vp, i64, ctypes.c_int32, _vp]
+        l.cola_wgrad_static_scratch.restype = st
         l.cola_trace_attach.argtypes = [ctypes.POINTER(cola_trace_slot_t), ctypes.c_int32,
                                         ctypes.POINTER(ctypes.c_int32)]
         l.cola_trace_attach.restype = st
@@ -171,6 +175,15 @@ def cola_check_status(ws, stream=None):
 
 def cola_status_string(status: int) -> str:
     return lib().cola_status_string(int(status)).decode()
+
+
+def cola_wgrad_static_scratch(n_tokens, M, N, P, ld_p, Q, ld_q, D, ld_d, accumulate_f32=False, stream=None):
+    """D[M x N] = P[:n_tokens, :M]^T Q[:n_tokens, :N] with the library's static
+    device scratch: no workspace, no allocation.  For callers that cannot
+    allocate device memory (see include/cola.h)."""
+    _check(lib().cola_wgrad_static_scratch(int(n_tokens), int(M), int(N), _ptr(P), int(ld_p), _ptr(Q), int(ld_q),
+                                           _ptr(D), int(ld_d), int(bool(accumulate_f32)), _stream(stream)),
+           "cola_wgrad_static_scratch")
 
 
 def cola_trace_attach(slots, capacity: int, count):

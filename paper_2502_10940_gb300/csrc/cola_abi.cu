@@ -10,6 +10,7 @@
 
 #include "../../include/cola.h"
 #include "gemm_launch.cuh"
+#include "host_plan.cuh"
 
 namespace cola {
 namespace {
@@ -43,101 +44,6 @@ cola_status_t device_info(int* sms)
     if (d.ok != 1) return COLA_ERR_UNSUPPORTED;
     *sms = d.sms;
     return COLA_OK;
-}
-
-// ------------------------------------------------------------ tensor maps
-using EncodeFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
-                              const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
-                              CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
-
-EncodeFn encode_fn()
-{
-    static EncodeFn fn = nullptr;
-    static std::once_flag once;
-    std::call_once(once, [] {
-        void* p = nullptr;
-        cudaDriverEntryPointQueryResult q = cudaDriverEntryPointSymbolNotFound;
-        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
-                cudaSuccess &&
-            q == cudaDriverEntryPointSuccess)
-            fn = reinterpret_cast<EncodeFn>(p);
-    });
-    return fn;
-}
-
-// 2-D bf16 matrix [outer x inner] with row pitch ld (elements), 128-byte
-// swizzle, box = {64 inner, box_outer}.  Out-of-range box parts read as zero.
-bool make_map(CUtensorMap* m, const void* base, int64_t inner, int64_t outer, int64_t ld, int box_outer)
-{
-    EncodeFn fn = encode_fn();
-    if (!fn) return false;
-    cuuint64_t dims[2] = {static_cast<cuuint64_t>(inner), static_cast<cuuint64_t>(outer)};
-    cuuint64_t strides[1] = {static_cast<cuuint64_t>(ld) * 2};
-    cuuint32_t box[2] = {64u, static_cast<cuuint32_t>(box_outer)};
-    cuuint32_t estr[2] = {1u, 1u};
-    CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
-                    CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-                    CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-    return r == CUDA_SUCCESS;
-}
-
-// K-major operand: rows are the M (or N) index, k contiguous: box {64, rows_per_tile}.
-// MN-major operand: rows are k, the M (or N) index contiguous: box {64, 64}.
-bool map_kmajor(CUtensorMap* m, const void* base, int64_t k_extent, int64_t mn_extent, int64_t ld, int tile_rows)
-{
-    return make_map(m, base, k_extent, mn_extent, ld, tile_rows);
-}
-
-bool map_mnmajor(CUtensorMap* m, const void* base, int64_t mn_extent, int64_t k_extent, int64_t ld)
-{
-    return make_map(m, base, mn_extent, k_extent, ld, 64);
-}
-
-// ------------------------------------------------------------ planning
-int choose_bn(int64_t N)
-{
-    if (N <= 128) return 128;
-    const int64_t pad256 = (N + 255) / 256 * 256;
-    const int64_t pad128 = (N + 127) / 128 * 128;
-    return pad256 <= pad128 ? 256 : 128;
-}
-
-GemmParams plan(int64_t M, int64_t N, int64_t K, int bn, int sms, bool split_k)
-{
-    GemmParams p;
-    std::memset(&p, 0, sizeof p);
-    p.M = static_cast<int>(M);
-    p.N = static_cast<int>(N);
-    p.k_blocks = static_cast<int>((K + BK - 1) / BK);
-    p.m_tiles = static_cast<int>((M + BM - 1) / BM);
-    p.n_tiles = static_cast<int>((N + bn - 1) / bn);
-    const int tiles = p.m_tiles * p.n_tiles;
-    int S = 1;
-    if (split_k) {
-        S = sms / tiles;
-        const int max_s = p.k_blocks / 4;     // at least 4 k-blocks (256 tokens) per split
-        if (S > max_s) S = max_s;
-        if (S < 1) S = 1;
-    }
-    p.kb_per_split = (p.k_blocks + S - 1) / S;
-    p.splits = (p.k_blocks + p.kb_per_split - 1) / p.kb_per_split;
-    p.units = tiles * p.splits;
-    return p;
-}
-
-int64_t partial_elems(const GemmParams& p, int bn)
-{
-    return static_cast<int64_t>(p.m_tiles) * BM * p.n_tiles * bn;
-}
-
-int grid_for(const GemmParams& p, int sms) { return p.units < sms ? p.units : sms; }
-
-template <bool A_MN, bool B_MN, int EPI>
-cudaError_t dispatch(int bn, const CUtensorMap& ma, const CUtensorMap& mb, const GemmParams& p, int sms,
-                     cudaStream_t s)
-{
-    if (bn == 256) return launch_gemm<256, A_MN, B_MN, EPI>(ma, mb, p, grid_for(p, sms), s);
-    return launch_gemm<128, A_MN, B_MN, EPI>(ma, mb, p, grid_for(p, sms), s);
 }
 
 // ------------------------------------------------------------ workspace
