@@ -245,59 +245,104 @@ def traffic_from_profile(kernel_key, workload):
 
 # ---------------------------------------------------------------- clocks
 class ClockSampler:
-    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
-              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
-              "clocks_event_reasons.sw_power_cap")
+    """SM clock, power and clock-event reasons sampled every 10 ms on a
+    background thread while the timed region runs (NVML read-only queries
+    through the driver's libnvidia-ml; falls back to nvidia-smi)."""
+
+    REASONS = {0x4: "sw_power_cap", 0x8: "hw_slowdown", 0x20: "sw_thermal_slowdown",
+               0x40: "hw_thermal_slowdown", 0x80: "hw_power_brake_slowdown"}
 
     def __init__(self, device_index):
-        self.proc = None
         self.dev = device_index
+        self.samples = []
+        self.max_mhz = None
+        self._stop = None
+        self._thread = None
+        self._nvml = None
+        self._h = None
+        self._smi = None
+
+    def _open_nvml(self):
+        import ctypes
+
+        import torch
+        lib = ctypes.CDLL("libnvidia-ml.so.1")
+        if lib.nvmlInit_v2() != 0:
+            raise RuntimeError("nvmlInit failed")
+        h = ctypes.c_void_p()
+        uuid = str(torch.cuda.get_device_properties(self.dev).uuid)
+        uuid = uuid if uuid.startswith("GPU-") else "GPU-" + uuid
+        if lib.nvmlDeviceGetHandleByUUID(uuid.encode(), ctypes.byref(h)) != 0:
+            if lib.nvmlDeviceGetHandleByIndex_v2(self.dev, ctypes.byref(h)) != 0:
+                raise RuntimeError("no NVML handle")
+        mx = ctypes.c_uint()
+        if lib.nvmlDeviceGetMaxClockInfo(h, 1, ctypes.byref(mx)) == 0:
+            self.max_mhz = float(mx.value)
+        self._reasons_fn = getattr(lib, "nvmlDeviceGetCurrentClocksEventReasons", None) or \
+            getattr(lib, "nvmlDeviceGetCurrentClocksThrottleReasons")
+        self._nvml, self._h = lib, h
+
+    def _sample_nvml(self):
+        import ctypes
+        c = ctypes.c_uint()
+        r = ctypes.c_ulonglong()
+        pw = ctypes.c_uint()
+        if self._nvml.nvmlDeviceGetClockInfo(self._h, 1, ctypes.byref(c)) != 0:
+            return
+        self._reasons_fn(self._h, ctypes.byref(r))
+        self._nvml.nvmlDeviceGetPowerUsage(self._h, ctypes.byref(pw))
+        self.samples.append((float(c.value), int(r.value), pw.value / 1000.0))
 
     def start(self):
+        import threading
         try:
-            import torch
-            uuid = None
+            self._open_nvml()
+        except Exception:  # noqa: BLE001 -- no NVML: use nvidia-smi instead
+            self._nvml = None
+        if self._nvml is None:
             try:
-                uuid = str(torch.cuda.get_device_properties(self.dev).uuid)
-                if uuid and not uuid.startswith("GPU-"):
-                    uuid = "GPU-" + uuid
+                self._smi = subprocess.Popen(
+                    ["nvidia-smi", "--query-gpu=clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active",
+                     "--format=csv,noheader,nounits", "-lms", "100", "-i", str(self.dev)],
+                    stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
             except Exception:  # noqa: BLE001
-                uuid = None
-            sel = ["-i", uuid] if uuid else []
-            self.proc = subprocess.Popen(["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
-                                          "-lms", "100"] + sel, stdout=subprocess.PIPE, stderr=subprocess.DEVNULL,
-                                         text=True)
-        except Exception:  # noqa: BLE001 -- no nvidia-smi: clocks are reported as unknown
-            self.proc = None
+                self._smi = None
+            return
+        self._stop = threading.Event()
+
+        def loop():
+            while not self._stop.is_set():
+                self._sample_nvml()
+                self._stop.wait(0.01)
+
+        self._thread = threading.Thread(target=loop, daemon=True)
+        self._thread.start()
 
     def stop(self):
-        if self.proc is None:
-            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"], "samples": 0}
-        self.proc.terminate()
-        try:
-            out, _ = self.proc.communicate(timeout=5)
-        except Exception:  # noqa: BLE001
-            self.proc.kill()
-            out, _ = self.proc.communicate()
-        sm, mx, pw, reasons = [], [], [], set()
-        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
-        for line in out.splitlines():
-            parts = [p.strip() for p in line.split(",")]
-            if len(parts) < 7:
-                continue
-            try:
-                sm.append(float(parts[0]))
-                mx.append(float(parts[1]))
-                pw.append(float(parts[2]))
-            except ValueError:
-                continue
-            for nm, v in zip(names, parts[3:7]):
-                if v.lower().startswith("active"):
+        if self._thread is not None:
+            self._stop.set()
+            self._thread.join()
+            self._sample_nvml()
+        elif self._smi is not None:
+            self._smi.terminate()
+            out, _ = self._smi.communicate()
+            for line in out.splitlines():
+                parts = [p.strip() for p in line.split(",")]
+                try:
+                    self.samples.append((float(parts[0]), int(parts[3], 16), float(parts[2])))
+                    self.max_mhz = float(parts[1])
+                except (ValueError, IndexError):
+                    continue
+        if not self.samples:
+            return {"sm_mhz": None, "sm_max_mhz": self.max_mhz, "reasons": ["no clock samples"], "samples": 0}
+        reasons = set()
+        for _, bits, _ in self.samples:
+            for b, nm in self.REASONS.items():
+                if bits & b:
                     reasons.add(nm)
-        if not sm:
-            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"], "samples": 0}
-        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
-                "power_w_max": max(pw), "samples": len(sm)}
+        return {"sm_mhz": statistics.median(x[0] for x in self.samples), "sm_max_mhz": self.max_mhz,
+                "reasons": sorted(reasons), "power_w_max": round(max(x[2] for x in self.samples), 1),
+                "samples": len(self.samples), "source": "nvml" if self._nvml is not None else "nvidia-smi"}
 
 
 # ---------------------------------------------------------------- CPU oracle
@@ -468,11 +513,11 @@ def run_cola(args, wl):
     blk.launches_per_step = tr.count.value
     blk.check()
 
-    sampler = ClockSampler(local)
-    sampler.start()
     for _ in range(args.warmup):
         blk.step()
     torch.cuda.synchronize()
+    sampler = ClockSampler(local)
+    sampler.start()
     ms = time_steps(blk.step, args.steps, stream, dist)
     clocks = sampler.stop()
     blk.check()

@@ -183,17 +183,17 @@ cola_status_t run_f1(const Shape& s, int sigma, int64_t N, const void* X, const 
 {
     const int bn = choose_bn(N);
     GemmParams p = plan(s.n, N, s.d_in, bn, sms, false);
-    CUtensorMap ma, mb;
+    CUtensorMap ma, mb, md, md2;
     COLA_MAP(map_kmajor(&ma, X, s.d_in, s.n, s.ld_x, BM));
     COLA_MAP(map_kmajor(&mb, A, s.d_in, N, s.ld_a, bn));
-    p.D = Z;
-    p.ldd = ldz;
-    p.D2 = static_cast<__nv_bfloat16*>(H);
-    p.ldd2 = ldz;
+    COLA_MAP(map_box32(&md, Z, N, s.n, ldz));
+    if (H) COLA_MAP(map_box32(&md2, H, N, s.n, ldz));
+    p.has_d2 = H != nullptr;
     p.sigma = sigma;
     p.status = status;
-    return launched(traced(COLA_KERNEL_FWD_ZH, s.n, N, s.d_in, 1, H != nullptr, st,
-                           [&] { return dispatch<false, false, EPI_ZH>(bn, ma, mb, p, sms, st); }));
+    return launched(traced(COLA_KERNEL_FWD_ZH, s.n, N, s.d_in, 1, H != nullptr, st, [&] {
+        return dispatch<false, false, EPI_ZH>(bn, ma, mb, md, H ? md2 : md, p, sms, st);
+    }));
 }
 
 // F2: Y = H B^T  (H [n x r] with pitch ldh)
@@ -202,14 +202,16 @@ cola_status_t run_f2(const Shape& s, const void* H, int64_t ldh, const void* B, 
 {
     const int bn = choose_bn(s.d_out);
     GemmParams p = plan(s.n, s.d_out, s.r, bn, sms, false);
-    CUtensorMap ma, mb;
+    CUtensorMap ma, mb, md;
     COLA_MAP(map_kmajor(&ma, H, s.r, s.n, ldh, BM));
     COLA_MAP(map_kmajor(&mb, B, s.r, s.d_out, s.r, bn));
-    p.D = Y;
-    p.ldd = s.ld_y;
+    COLA_MAP(map_box32(&md, Y, s.d_out, s.n, s.ld_y));
+    p.d_ptr = static_cast<__nv_bfloat16*>(Y);
+    p.d_ld = s.ld_y;
     p.status = status;
-    return launched(traced(COLA_KERNEL_FWD_Y, s.n, s.d_out, s.r, 1, 0, st,
-                           [&] { return dispatch<false, false, EPI_STORE>(bn, ma, mb, p, sms, st); }));
+    return launched(traced(COLA_KERNEL_FWD_Y, s.n, s.d_out, s.r, 1, 0, st, [&] {
+        return dispatch<false, false, EPI_STORE>(bn, ma, mb, md, md, p, sms, st);
+    }));
 }
 
 // B1: dZ = (dY B) * sigma'(Z), and H = sigma(Z) when Hout != null (CoLA-M)
@@ -218,19 +220,19 @@ cola_status_t run_b1(const Shape& s, int sigma, const void* dY, const void* B, c
 {
     const int bn = choose_bn(s.r);
     GemmParams p = plan(s.n, s.r, s.d_out, bn, sms, false);
-    CUtensorMap ma, mb;
+    CUtensorMap ma, mb, md, md2;
     COLA_MAP(map_kmajor(&ma, dY, s.d_out, s.n, s.ld_y, BM));
     COLA_MAP(map_mnmajor(&mb, B, s.r, s.d_out, s.r));
-    p.D = dZ;
-    p.ldd = ldz;
-    p.D2 = static_cast<__nv_bfloat16*>(Hout);
-    p.ldd2 = ldz;
-    p.Zin = static_cast<const __nv_bfloat16*>(Z);
-    p.ldz = ldz;
+    COLA_MAP(map_box32(&md, dZ, s.r, s.n, ldz));
+    if (Hout) COLA_MAP(map_box32(&md2, Hout, s.r, s.n, ldz));
+    p.has_d2 = Hout != nullptr;
+    p.z_ptr = static_cast<const __nv_bfloat16*>(Z);
+    p.z_ld = ldz;
     p.sigma = sigma;
     p.status = status;
-    return launched(traced(COLA_KERNEL_BWD_DZ, s.n, s.r, s.d_out, 1, Hout != nullptr, st,
-                           [&] { return dispatch<false, true, EPI_DSIGMA>(bn, ma, mb, p, sms, st); }));
+    return launched(traced(COLA_KERNEL_BWD_DZ, s.n, s.r, s.d_out, 1, Hout != nullptr, st, [&] {
+        return dispatch<false, true, EPI_DSIGMA>(bn, ma, mb, md, Hout ? md2 : md, p, sms, st);
+    }));
 }
 
 // Weight gradient D[M x N] = sum_t P[t, m] Q[t, n] over the n tokens, both
@@ -251,7 +253,7 @@ cola_status_t run_wgrad(int kind, int64_t ntok, int64_t M, int64_t N, const void
     p.part_stride = slab;
     p.status = status;
     COLA_TRY(launched(traced(kind, M, N, ntok, p.splits, 0, st,
-                             [&] { return dispatch<true, true, EPI_F32>(bn, ma, mb, p, sms, st); })));
+                             [&] { return dispatch<true, true, EPI_F32>(bn, ma, mb, ma, ma, p, sms, st); })));
     return launched(traced(COLA_KERNEL_REDUCE, M, N, p.splits, p.splits, 0, st, [&] {
         return launch_splitk_reduce(part, p.splits, slab, p.n_tiles * bn, static_cast<int>(M), static_cast<int>(N),
                                     out, ldo, accumulate_f32, sms * 4, st);
@@ -264,14 +266,16 @@ cola_status_t run_b4(const Shape& s, int64_t K, const void* dZ, int64_t ldz, con
 {
     const int bn = choose_bn(s.d_in);
     GemmParams p = plan(s.n, s.d_in, K, bn, sms, false);
-    CUtensorMap ma, mb;
+    CUtensorMap ma, mb, md;
     COLA_MAP(map_kmajor(&ma, dZ, K, s.n, ldz, BM));
     COLA_MAP(map_mnmajor(&mb, A, s.d_in, K, s.ld_a));
-    p.D = dX;
-    p.ldd = s.ld_x;
+    COLA_MAP(map_box32(&md, dX, s.d_in, s.n, s.ld_x));
+    p.d_ptr = static_cast<__nv_bfloat16*>(dX);
+    p.d_ld = s.ld_x;
     p.status = status;
-    return launched(traced(COLA_KERNEL_BWD_DX, s.n, s.d_in, K, 1, 0, st,
-                           [&] { return dispatch<false, true, EPI_STORE>(bn, ma, mb, p, sms, st); }));
+    return launched(traced(COLA_KERNEL_BWD_DX, s.n, s.d_in, K, 1, 0, st, [&] {
+        return dispatch<false, true, EPI_STORE>(bn, ma, mb, md, md, p, sms, st);
+    }));
 }
 
 }  // namespace

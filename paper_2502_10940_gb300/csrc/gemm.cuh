@@ -8,12 +8,16 @@
 // swizzled shared memory and consumed by tcgen05.mma directly, so no
 // operand is ever transposed in memory.
 //
-// Warp roles (192 threads, one CTA per SM, persistent over output tiles):
+// Warp roles (320 threads, one CTA per SM, persistent over output tiles):
 //   warp 0      TMA producer: fills a STAGES-deep ring of (A, B) k-blocks.
 //   warp 1      MMA issuer:  tcgen05.mma M=128, N=BN, K=16 into one of two
 //               TMEM accumulators (double buffered, so the epilogue of tile
 //               i overlaps the main loop of tile i+1); allocates TMEM.
-//   warps 2..5  epilogue: tcgen05.ld -> fused elementwise -> global stores.
+//   warps 2..9  epilogue, two warps per TMEM lane quarter taking alternate
+//               32-column chunks: tcgen05.ld -> fused elementwise -> 32x32
+//               boxes staged in shared memory (64-byte swizzle, bank-conflict
+//               free) -> TMA bulk tensor stores, which are coalesced,
+//               asynchronous and clipped to the tensor's extents in hardware.
 //
 // Epilogues (the elementwise parts of the layer, fused so that the rank-r
 // intermediate makes no extra HBM round trip):
@@ -39,7 +43,8 @@ namespace cola {
 constexpr int BM = 128;              // UMMA M (cta_group::1): one row per TMEM lane
 constexpr int BK = 64;               // k-block: one 128-byte swizzle row of bf16
 constexpr int UMMA_K = 16;           // K of one kind::f16 MMA
-constexpr int NUM_THREADS = 192;
+constexpr int NUM_EPI_WARPS = 8;     // two per TMEM lane quarter
+constexpr int NUM_THREADS = 64 + 32 * NUM_EPI_WARPS;
 constexpr uint64_t WAIT_LIMIT_NS = 2000000000ull;   // 2 s
 
 // bits recorded in the status word when a wait gives up
@@ -59,16 +64,28 @@ struct GemmParams {
     int m_tiles, n_tiles;
     int splits, kb_per_split;
     int units;             // m_tiles * n_tiles * splits
-    void* D;               // bf16 output, or fp32 partial slabs (EPI_F32)
-    long long ldd;         // row pitch of D in elements
-    __nv_bfloat16* D2;     // H output (EPI_ZH / EPI_DSIGMA), may be null
-    long long ldd2;
-    const __nv_bfloat16* Zin;  // saved Z (EPI_DSIGMA)
-    long long ldz;
+    void* D;               // EPI_F32: fp32 partial slabs (bf16 outputs go through map_d / map_d2)
+    long long ldd;         // EPI_F32: row pitch of a slab in elements
     long long part_stride; // EPI_F32: elements per split slab
+    int has_d2;            // EPI_ZH / EPI_DSIGMA: also store H through map_d2
+    // The bf16 output behind map_d, for the one 32-column chunk per row block
+    // that holds a ragged right edge (N % 8 != 0): a TMA store clips at
+    // 16-byte granularity and would write the row padding past column N, so
+    // that chunk is stored with masked direct stores instead.
+    __nv_bfloat16* d_ptr;
+    long long d_ld;
+    const __nv_bfloat16* z_ptr;  // EPI_DSIGMA: the saved Z (same extents as the output)
+    long long z_ld;
     int sigma;
     unsigned int* status;
 };
+
+// Epilogue staging: per epilogue warp two 2 KB boxes of 32 rows x 32 bf16
+// columns (64-byte rows, 64-byte TMA swizzle), used as a ring of output boxes.
+constexpr int EPI_BOX_BYTES = 32 * 32 * 2;
+constexpr int EPI_OUT_BOXES = 2;
+constexpr int EPI_WARP_BYTES = EPI_OUT_BOXES * EPI_BOX_BYTES;
+constexpr int EPI_SMEM_BYTES = NUM_EPI_WARPS * EPI_WARP_BYTES;
 
 template <int BN>
 struct GemmCfg {
@@ -76,16 +93,27 @@ struct GemmCfg {
     static constexpr int A_BYTES = BM * BK * 2;
     static constexpr int B_BYTES = BN * BK * 2;
     static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
-    static constexpr int STAGES = (200 * 1024) / STAGE_BYTES > 8 ? 8 : (200 * 1024) / STAGE_BYTES;
-    static constexpr int TMEM_COLS = (2 * BN <= 128) ? 128 : (2 * BN <= 256 ? 256 : 512);
     static constexpr int BAR_BYTES = 256;
-    static constexpr int SMEM_BYTES = 1024 + STAGES * STAGE_BYTES + BAR_BYTES;
+    static constexpr int SMEM_LIMIT = 232448;   // opt-in maximum per CTA
+    static constexpr int STAGES_FIT = (SMEM_LIMIT - 1024 - BAR_BYTES - EPI_SMEM_BYTES) / STAGE_BYTES;
+    static constexpr int STAGES = STAGES_FIT > 8 ? 8 : STAGES_FIT;
+    static constexpr int TMEM_COLS = (2 * BN <= 128) ? 128 : (2 * BN <= 256 ? 256 : 512);
+    static constexpr int SMEM_BYTES = 1024 + STAGES * STAGE_BYTES + EPI_SMEM_BYTES + BAR_BYTES;
+    static_assert(SMEM_BYTES <= SMEM_LIMIT, "shared memory budget");
 };
 
 // ------------------------------------------------------------ activations
+// logistic(z) with the fast exponential and divide (a few ulp of fp32, far
+// below the bf16 rounding every result goes through); exactly 0 below -87,
+// where e^{-z} would leave the range of the fast divide.
+__device__ __forceinline__ float logistic_fast(float z)
+{
+    return z < -87.0f ? 0.0f : __fdividef(1.0f, 1.0f + __expf(-z));
+}
+
 __device__ __forceinline__ float act_sigma(int kind, float z)
 {
-    if (kind == SIG_SILU) return z / (1.0f + __expf(-z));
+    if (kind == SIG_SILU) return z * logistic_fast(z);
     if (kind == SIG_GELU) return 0.5f * z * erfcf(-z * 0.70710678118654752f);
     return z;
 }
@@ -93,7 +121,7 @@ __device__ __forceinline__ float act_sigma(int kind, float z)
 __device__ __forceinline__ float act_dsigma(int kind, float z)
 {
     if (kind == SIG_SILU) {
-        const float s = 1.0f / (1.0f + __expf(-z));
+        const float s = logistic_fast(z);
         return s * (1.0f + z * (1.0f - s));
     }
     if (kind == SIG_GELU) {
@@ -146,23 +174,35 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi)
 __device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
 __device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
 
-// Store 32 packed bf16 (16 words) at dst[0..31], clipped to `valid` columns.
-__device__ __forceinline__ void store_row32_bf16(__nv_bfloat16* dst, const uint32_t (&w)[16], int valid)
+// Byte offset of 16-byte chunk j of row i inside a 32 x 32 bf16 box laid out
+// with the TMA 64-byte swizzle (chunk bits 4-5 XOR address bits 7-8).
+__device__ __forceinline__ uint32_t box64_off(int i, int j) { return i * 64 + ((j ^ ((i >> 1) & 3)) << 4); }
+
+__device__ __forceinline__ void st_shared_v4(uint32_t addr, uint32_t a, uint32_t b, uint32_t c, uint32_t d)
 {
-    if (valid >= 32) {
-        uint4* d4 = reinterpret_cast<uint4*>(dst);
+    asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(a), "r"(b), "r"(c), "r"(d) : "memory");
+}
+
+__device__ __forceinline__ uint4 ld_shared_v4(uint32_t addr)
+{
+    uint4 v;
+    asm volatile("ld.shared.v4.b32 {%0, %1, %2, %3}, [%4];" : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(addr)
+                 : "memory");
+    return v;
+}
+
+// Write this thread's 32 packed bf16 (row `lane` of the box) into a staging box.
+__device__ __forceinline__ void stage_row(uint32_t box, int lane, const uint32_t (&w)[16])
+{
 #pragma unroll
-        for (int q = 0; q < 4; ++q) d4[q] = make_uint4(w[4 * q], w[4 * q + 1], w[4 * q + 2], w[4 * q + 3]);
-    } else {
-        uint16_t* d = reinterpret_cast<uint16_t*>(dst);
-        for (int j = 0; j < valid; ++j) d[j] = static_cast<uint16_t>((j & 1) ? (w[j >> 1] >> 16) : (w[j >> 1] & 0xFFFFu));
-    }
+    for (int j = 0; j < 4; ++j) st_shared_v4(box + box64_off(lane, j), w[4 * j], w[4 * j + 1], w[4 * j + 2], w[4 * j + 3]);
 }
 
 // ------------------------------------------------------------ the kernel
 template <int BN, bool A_MN, bool B_MN, int EPI>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
     gemm_kernel(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUtensorMap map_b,
+                const __grid_constant__ CUtensorMap map_d, const __grid_constant__ CUtensorMap map_d2,
                 const GemmParams p)
 {
     using C = GemmCfg<BN>;
@@ -171,7 +211,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint8_t* smem_a = smem;                              // STAGES x A_BYTES
     uint8_t* smem_b = smem + STAGES * C::A_BYTES;        // STAGES x B_BYTES
-    uint64_t* bars = reinterpret_cast<uint64_t*>(smem + STAGES * C::STAGE_BYTES);
+    uint8_t* smem_epi = smem + STAGES * C::STAGE_BYTES;  // NUM_EPI_WARPS x EPI_WARP_BYTES
+    uint64_t* bars = reinterpret_cast<uint64_t*>(smem_epi + EPI_SMEM_BYTES);
     uint64_t* full_bar = bars;                 // [STAGES]
     uint64_t* empty_bar = bars + STAGES;       // [STAGES]
     uint64_t* tfull_bar = bars + 2 * STAGES;   // [2]
@@ -191,13 +232,14 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(&tfull_bar[b], 1);
-            mbar_init(&tempty_bar[b], 4 * 32);
+            mbar_init(&tempty_bar[b], NUM_EPI_WARPS * 32);
         }
         mbar_init(drain_bar, 1);
         *abort_flag = 0;
         fence_mbar_init();
         tma_prefetch_desc(&map_a);
         tma_prefetch_desc(&map_b);
+        if (EPI != EPI_F32) tma_prefetch_desc(&map_d);
     }
     if (warp == 1) {
         tmem_alloc(tmem_slot, C::TMEM_COLS);
@@ -341,27 +383,62 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             }
         }
     } else {
-        // ------------------------------------------------ epilogue (warps 2..5)
+        // ------------------------------------------------ epilogue (warps 2..9)
         const int q = warp & 3;                 // TMEM lane quarter this warp may access
+        const int half = (warp - 2) >> 2;       // the two warps of a quarter take alternate chunks
         const int row_in_tile = q * 32 + lane;
+        const uint32_t ep = smem_u32(smem_epi + (warp - 2) * EPI_WARP_BYTES);
+        int out_slot = 0;                       // next output box of the ring
         int buf = 0;
         uint32_t bphase = 0;
+
+        // stage one output box (this thread's row) and hand it to the TMA engine
+        auto emit = [&](const CUtensorMap* map, const uint32_t (&w)[16], int x, int y) {
+            if (y >= p.M) return;               // whole box below the last row: nothing to store
+            const uint32_t box = ep + out_slot * EPI_BOX_BYTES;
+            if (lane == 0) bulk_wait_group_read<EPI_OUT_BOXES - 1>();   // its previous store has read it
+            __syncwarp();
+            stage_row(box, lane, w);
+            fence_proxy_async_smem();
+            __syncwarp();
+            if (lane == 0) {
+                tma_store_2d(map, box, x, y);
+                bulk_commit_group();
+            }
+            if (++out_slot == EPI_OUT_BOXES) out_slot = 0;
+        };
+
         for (int u = blockIdx.x; u < p.units; u += gridDim.x) {
             int m_blk, n_blk, split, kb0, kb1;
             decode_unit(p, u, m_blk, n_blk, split, kb0, kb1);
+            const int row0 = m_blk * BM + q * 32;
+            const int row = row0 + lane;
+            int nch = BN / 32;                  // chunks of 32 columns that hold valid output
+            if (n_blk * BN + BN > p.N) nch = (p.N - n_blk * BN + 31) / 32;
+            if (EPI != EPI_F32 && row0 >= p.M) nch = 0;   // this warp's 32 rows are all past the end
             if (!wait_bounded(&tfull_bar[buf], bphase, wc, ST_TIMEOUT_EPILOGUE)) break;
             tc_fence_after();
-            const int row = m_blk * BM + row_in_tile;
             const uint32_t tbase = tmem_base + (static_cast<uint32_t>(q * 32) << 16) + static_cast<uint32_t>(buf * BN);
 #pragma unroll 1
-            for (int c = 0; c < BN / 32; ++c) {
+            for (int c = half; c < (EPI == EPI_F32 ? BN / 32 : nch); c += 2) {
+                const int col0 = n_blk * BN + c * 32;
+                uint4 zq[4];
+                if (EPI == EPI_DSIGMA) {        // the saved Z of this row's chunk, in flight during the TMEM load
+                    if (row < p.M) {
+                        const uint4* zs = reinterpret_cast<const uint4*>(p.z_ptr + row * p.z_ld + col0);
+#pragma unroll
+                        for (int j = 0; j < 4; ++j) zq[j] = __ldg(zs + j);
+                    } else {
+#pragma unroll
+                        for (int j = 0; j < 4; ++j) zq[j] = make_uint4(0u, 0u, 0u, 0u);
+                    }
+                }
                 uint32_t v[32];
                 tmem_ld_32x32b_x32(tbase + c * 32, v);
                 tmem_ld_wait();
-                const int col0 = n_blk * BN + c * 32;
                 if (EPI == EPI_F32) {
                     float* dst = reinterpret_cast<float*>(p.D) + split * p.part_stride +
-                                 static_cast<long long>(m_blk * BM + row_in_tile) * (p.n_tiles * BN) + col0;
+                                 static_cast<long long>(m_blk * BM + row_in_tile) * p.ldd + col0;
                     float4* d4 = reinterpret_cast<float4*>(dst);
 #pragma unroll
                     for (int j = 0; j < 8; ++j)
@@ -369,51 +446,45 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                                             __uint_as_float(v[4 * j + 2]), __uint_as_float(v[4 * j + 3]));
                     continue;
                 }
-                if (row >= p.M || col0 >= p.N) continue;
-                const int valid = min(32, p.N - col0);
                 uint32_t w[16];
                 if (EPI == EPI_STORE) {
 #pragma unroll
                     for (int j = 0; j < 16; ++j)
                         w[j] = pack_bf16x2(__uint_as_float(v[2 * j]), __uint_as_float(v[2 * j + 1]));
-                    store_row32_bf16(reinterpret_cast<__nv_bfloat16*>(p.D) + row * p.ldd + col0, w, valid);
+                    if ((p.N & 7) != 0 && col0 + 32 > p.N) {
+                        // ragged right edge: masked per-element stores, padding untouched
+                        if (row < p.M) {
+                            uint16_t* d = reinterpret_cast<uint16_t*>(p.d_ptr + row * p.d_ld + col0);
+                            for (int j = 0; j < p.N - col0; ++j)
+                                d[j] = static_cast<uint16_t>((j & 1) ? (w[j >> 1] >> 16) : (w[j >> 1] & 0xFFFFu));
+                        }
+                        continue;
+                    }
+                    emit(&map_d, w, col0, row0);
                 } else if (EPI == EPI_ZH) {
 #pragma unroll
                     for (int j = 0; j < 16; ++j)
                         w[j] = pack_bf16x2(__uint_as_float(v[2 * j]), __uint_as_float(v[2 * j + 1]));
-                    store_row32_bf16(reinterpret_cast<__nv_bfloat16*>(p.D) + row * p.ldd + col0, w, valid);
-                    if (p.D2 != nullptr) {
-                        uint32_t h[16];
+                    emit(&map_d, w, col0, row0);
+                    if (p.has_d2) {
 #pragma unroll
                         for (int j = 0; j < 16; ++j)
-                            h[j] = pack_bf16x2(act_sigma(p.sigma, bf16_lo(w[j])), act_sigma(p.sigma, bf16_hi(w[j])));
-                        store_row32_bf16(p.D2 + row * p.ldd2 + col0, h, valid);
+                            w[j] = pack_bf16x2(act_sigma(p.sigma, bf16_lo(w[j])), act_sigma(p.sigma, bf16_hi(w[j])));
+                        emit(&map_d2, w, col0, row0);
                     }
                 } else if (EPI == EPI_DSIGMA) {
-                    // Z has the same (row, col) extent as dZ: N = r is a multiple of 64.
-                    uint32_t z[16];
-                    const uint4* zs = reinterpret_cast<const uint4*>(p.Zin + row * p.ldz + col0);
+                    const uint32_t z[16] = {zq[0].x, zq[0].y, zq[0].z, zq[0].w, zq[1].x, zq[1].y, zq[1].z, zq[1].w,
+                                            zq[2].x, zq[2].y, zq[2].z, zq[2].w, zq[3].x, zq[3].y, zq[3].z, zq[3].w};
 #pragma unroll
-                    for (int qd = 0; qd < 4; ++qd) {
-                        const uint4 t = zs[qd];
-                        z[4 * qd] = t.x;
-                        z[4 * qd + 1] = t.y;
-                        z[4 * qd + 2] = t.z;
-                        z[4 * qd + 3] = t.w;
-                    }
-#pragma unroll
-                    for (int j = 0; j < 16; ++j) {
-                        const float z0 = bf16_lo(z[j]), z1 = bf16_hi(z[j]);
-                        w[j] = pack_bf16x2(__uint_as_float(v[2 * j]) * act_dsigma(p.sigma, z0),
-                                           __uint_as_float(v[2 * j + 1]) * act_dsigma(p.sigma, z1));
-                    }
-                    store_row32_bf16(reinterpret_cast<__nv_bfloat16*>(p.D) + row * p.ldd + col0, w, valid);
-                    if (p.D2 != nullptr) {
-                        uint32_t h[16];
+                    for (int j = 0; j < 16; ++j)
+                        w[j] = pack_bf16x2(__uint_as_float(v[2 * j]) * act_dsigma(p.sigma, bf16_lo(z[j])),
+                                           __uint_as_float(v[2 * j + 1]) * act_dsigma(p.sigma, bf16_hi(z[j])));
+                    emit(&map_d, w, col0, row0);
+                    if (p.has_d2) {
 #pragma unroll
                         for (int j = 0; j < 16; ++j)
-                            h[j] = pack_bf16x2(act_sigma(p.sigma, bf16_lo(z[j])), act_sigma(p.sigma, bf16_hi(z[j])));
-                        store_row32_bf16(p.D2 + row * p.ldd2 + col0, h, valid);
+                            w[j] = pack_bf16x2(act_sigma(p.sigma, bf16_lo(z[j])), act_sigma(p.sigma, bf16_hi(z[j])));
+                        emit(&map_d2, w, col0, row0);
                     }
                 }
             }
@@ -424,6 +495,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                 bphase ^= 1u;
             }
         }
+        if (lane == 0) bulk_wait_group_all();   // every output store has landed
     }
 
     tc_fence_before();

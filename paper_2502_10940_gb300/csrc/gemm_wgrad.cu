@@ -46,10 +46,12 @@ __global__ void splitk_reduce_kernel(const float* __restrict__ part, int splits,
 }
 
 
-template cudaError_t launch_gemm<128, true, true, EPI_F32>(const CUtensorMap&, const CUtensorMap&,
-                                                           const GemmParams&, int, cudaStream_t);
-template cudaError_t launch_gemm<256, true, true, EPI_F32>(const CUtensorMap&, const CUtensorMap&,
-                                                           const GemmParams&, int, cudaStream_t);
+template cudaError_t launch_gemm<128, true, true, EPI_F32>(const CUtensorMap&, const CUtensorMap&, const CUtensorMap&,
+                                                           const CUtensorMap&, const GemmParams&, int,
+                                                            cudaStream_t);
+template cudaError_t launch_gemm<256, true, true, EPI_F32>(const CUtensorMap&, const CUtensorMap&, const CUtensorMap&,
+                                                           const CUtensorMap&, const GemmParams&, int,
+                                                            cudaStream_t);
 
 cudaError_t launch_splitk_reduce(const float* part, int splits, long long part_stride, int ldp, int M, int N,
                                  void* out, long long ldo, int accumulate_f32, int grid, cudaStream_t stream)

@@ -34,32 +34,41 @@ EncodeFn encode_fn()
     return fn;
 }
 
-// 2-D bf16 matrix [outer x inner] with row pitch ld (elements), 128-byte
-// swizzle, box = {64 inner, box_outer}.  Out-of-range box parts read as zero.
-bool make_map(CUtensorMap* m, const void* base, int64_t inner, int64_t outer, int64_t ld, int box_outer)
+// 2-D bf16 matrix [outer x inner] with row pitch ld (elements) and box
+// {box_inner, box_outer}.  Loads read zeros outside the extents; stores are
+// clipped to them.
+bool make_map(CUtensorMap* m, const void* base, int64_t inner, int64_t outer, int64_t ld, int box_inner,
+              int box_outer, CUtensorMapSwizzle swz)
 {
     EncodeFn fn = encode_fn();
     if (!fn) return false;
     cuuint64_t dims[2] = {static_cast<cuuint64_t>(inner), static_cast<cuuint64_t>(outer)};
     cuuint64_t strides[1] = {static_cast<cuuint64_t>(ld) * 2};
-    cuuint32_t box[2] = {64u, static_cast<cuuint32_t>(box_outer)};
+    cuuint32_t box[2] = {static_cast<cuuint32_t>(box_inner), static_cast<cuuint32_t>(box_outer)};
     cuuint32_t estr[2] = {1u, 1u};
     CUresult r = fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
-                    CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                    CU_TENSOR_MAP_INTERLEAVE_NONE, swz, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                     CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     return r == CUDA_SUCCESS;
+}
+
+// Epilogue box of 32 rows x 32 columns (64-byte rows, 64-byte swizzle): the
+// unit in which the GEMM epilogue stores bf16 outputs and reads the saved Z.
+bool map_box32(CUtensorMap* m, const void* base, int64_t cols, int64_t rows, int64_t ld)
+{
+    return make_map(m, base, cols, rows, ld, 32, 32, CU_TENSOR_MAP_SWIZZLE_64B);
 }
 
 // K-major operand: rows are the M (or N) index, k contiguous: box {64, rows_per_tile}.
 // MN-major operand: rows are k, the M (or N) index contiguous: box {64, 64}.
 bool map_kmajor(CUtensorMap* m, const void* base, int64_t k_extent, int64_t mn_extent, int64_t ld, int tile_rows)
 {
-    return make_map(m, base, k_extent, mn_extent, ld, tile_rows);
+    return make_map(m, base, k_extent, mn_extent, ld, 64, tile_rows, CU_TENSOR_MAP_SWIZZLE_128B);
 }
 
 bool map_mnmajor(CUtensorMap* m, const void* base, int64_t mn_extent, int64_t k_extent, int64_t ld)
 {
-    return make_map(m, base, mn_extent, k_extent, ld, 64);
+    return make_map(m, base, mn_extent, k_extent, ld, 64, 64, CU_TENSOR_MAP_SWIZZLE_128B);
 }
 
 // ------------------------------------------------------------ planning
@@ -102,11 +111,11 @@ int64_t partial_elems(const GemmParams& p, int bn)
 int grid_for(const GemmParams& p, int sms) { return p.units < sms ? p.units : sms; }
 
 template <bool A_MN, bool B_MN, int EPI>
-cudaError_t dispatch(int bn, const CUtensorMap& ma, const CUtensorMap& mb, const GemmParams& p, int sms,
-                     cudaStream_t s)
+cudaError_t dispatch(int bn, const CUtensorMap& ma, const CUtensorMap& mb, const CUtensorMap& md,
+                     const CUtensorMap& md2, const GemmParams& p, int sms, cudaStream_t s)
 {
-    if (bn == 256) return launch_gemm<256, A_MN, B_MN, EPI>(ma, mb, p, grid_for(p, sms), s);
-    return launch_gemm<128, A_MN, B_MN, EPI>(ma, mb, p, grid_for(p, sms), s);
+    if (bn == 256) return launch_gemm<256, A_MN, B_MN, EPI>(ma, mb, md, md2, p, grid_for(p, sms), s);
+    return launch_gemm<128, A_MN, B_MN, EPI>(ma, mb, md, md2, p, grid_for(p, sms), s);
 }
 
 }  // namespace
