@@ -8,7 +8,7 @@
 #include <cstring>
 #include <mutex>
 
-#include "../../include/cola.h"
+#include "cola.h"
 #include "gemm_launch.cuh"
 #include "host_plan.cuh"
 
@@ -192,7 +192,7 @@ cola_status_t run_f1(const Shape& s, int sigma, int64_t N, const void* X, const 
     p.sigma = sigma;
     p.status = status;
     return launched(traced(COLA_KERNEL_FWD_ZH, s.n, N, s.d_in, 1, H != nullptr, st, [&] {
-        return dispatch<false, false, EPI_ZH>(bn, ma, mb, md, H ? md2 : md, p, sms, st);
+        return dispatch<false, false, EPI_ZH>(bn, ma, mb, md, H ? md2 : md, md, p, sms, st);
     }));
 }
 
@@ -210,7 +210,7 @@ cola_status_t run_f2(const Shape& s, const void* H, int64_t ldh, const void* B, 
     p.d_ld = s.ld_y;
     p.status = status;
     return launched(traced(COLA_KERNEL_FWD_Y, s.n, s.d_out, s.r, 1, 0, st, [&] {
-        return dispatch<false, false, EPI_STORE>(bn, ma, mb, md, md, p, sms, st);
+        return dispatch<false, false, EPI_STORE>(bn, ma, mb, md, md, md, p, sms, st);
     }));
 }
 
@@ -220,18 +220,17 @@ cola_status_t run_b1(const Shape& s, int sigma, const void* dY, const void* B, c
 {
     const int bn = choose_bn(s.r);
     GemmParams p = plan(s.n, s.r, s.d_out, bn, sms, false);
-    CUtensorMap ma, mb, md, md2;
+    CUtensorMap ma, mb, md, md2, mz;
     COLA_MAP(map_kmajor(&ma, dY, s.d_out, s.n, s.ld_y, BM));
     COLA_MAP(map_mnmajor(&mb, B, s.r, s.d_out, s.r));
     COLA_MAP(map_box32(&md, dZ, s.r, s.n, ldz));
+    COLA_MAP(map_box32(&mz, Z, s.r, s.n, ldz));
     if (Hout) COLA_MAP(map_box32(&md2, Hout, s.r, s.n, ldz));
     p.has_d2 = Hout != nullptr;
-    p.z_ptr = static_cast<const __nv_bfloat16*>(Z);
-    p.z_ld = ldz;
     p.sigma = sigma;
     p.status = status;
     return launched(traced(COLA_KERNEL_BWD_DZ, s.n, s.r, s.d_out, 1, Hout != nullptr, st, [&] {
-        return dispatch<false, true, EPI_DSIGMA>(bn, ma, mb, md, Hout ? md2 : md, p, sms, st);
+        return dispatch<false, true, EPI_DSIGMA>(bn, ma, mb, md, Hout ? md2 : md, mz, p, sms, st);
     }));
 }
 
@@ -248,12 +247,21 @@ cola_status_t run_wgrad(int kind, int64_t ntok, int64_t M, int64_t N, const void
     CUtensorMap ma, mb;
     COLA_MAP(map_mnmajor(&ma, P, M, ntok, ldp));
     COLA_MAP(map_mnmajor(&mb, Q, N, ntok, ldq));
+    p.status = status;
+    if (p.splits == 1 && !accumulate_f32) {
+        // no token split: the epilogue writes the bf16 gradient directly
+        CUtensorMap md;
+        COLA_MAP(map_box32(&md, out, N, M, ldo));
+        p.d_ptr = static_cast<__nv_bfloat16*>(out);
+        p.d_ld = ldo;
+        return launched(traced(kind, M, N, ntok, 1, 0, st,
+                               [&] { return dispatch<true, true, EPI_STORE>(bn, ma, mb, md, md, md, p, sms, st); }));
+    }
     p.D = part;
     p.ldd = p.n_tiles * bn;
     p.part_stride = slab;
-    p.status = status;
     COLA_TRY(launched(traced(kind, M, N, ntok, p.splits, 0, st,
-                             [&] { return dispatch<true, true, EPI_F32>(bn, ma, mb, ma, ma, p, sms, st); })));
+                             [&] { return dispatch<true, true, EPI_F32>(bn, ma, mb, ma, ma, ma, p, sms, st); })));
     return launched(traced(COLA_KERNEL_REDUCE, M, N, p.splits, p.splits, 0, st, [&] {
         return launch_splitk_reduce(part, p.splits, slab, p.n_tiles * bn, static_cast<int>(M), static_cast<int>(N),
                                     out, ldo, accumulate_f32, sms * 4, st);
@@ -274,7 +282,7 @@ cola_status_t run_b4(const Shape& s, int64_t K, const void* dZ, int64_t ldz, con
     p.d_ld = s.ld_x;
     p.status = status;
     return launched(traced(COLA_KERNEL_BWD_DX, s.n, s.d_in, K, 1, 0, st, [&] {
-        return dispatch<false, true, EPI_STORE>(bn, ma, mb, md, md, p, sms, st);
+        return dispatch<false, true, EPI_STORE>(bn, ma, mb, md, md, md, p, sms, st);
     }));
 }
 

@@ -18,7 +18,7 @@
 #include <cstdint>
 #include <mutex>
 
-#include "../../include/cola.h"
+#include "cola.h"
 #include "gemm_launch.cuh"
 #include "host_plan.cuh"
 
@@ -106,7 +106,7 @@ extern "C" cola_status_t cola_wgrad_static_scratch(int64_t n_tokens, int64_t M, 
     p.part_stride = slab;
     p.status = nullptr;   // no workspace to report a device-side timeout through
     cudaStream_t st = static_cast<cudaStream_t>(stream);
-    if (dispatch<true, true, EPI_F32>(bn, ma, mb, ma, ma, p, sms, st) != cudaSuccess) return COLA_ERR_LAUNCH;
+    if (dispatch<true, true, EPI_F32>(bn, ma, mb, ma, ma, ma, p, sms, st) != cudaSuccess) return COLA_ERR_LAUNCH;
     if (launch_splitk_reduce(part, p.splits, slab, p.n_tiles * bn, static_cast<int>(M), static_cast<int>(N), D, ld_d,
                              accumulate_f32, sms * 4, st) != cudaSuccess)
         return COLA_ERR_LAUNCH;

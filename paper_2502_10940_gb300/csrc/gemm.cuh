@@ -74,14 +74,15 @@ struct GemmParams {
     // that chunk is stored with masked direct stores instead.
     __nv_bfloat16* d_ptr;
     long long d_ld;
-    const __nv_bfloat16* z_ptr;  // EPI_DSIGMA: the saved Z (same extents as the output)
-    long long z_ld;
     int sigma;
     unsigned int* status;
 };
 
 // Epilogue staging: per epilogue warp two 2 KB boxes of 32 rows x 32 bf16
-// columns (64-byte rows, 64-byte TMA swizzle), used as a ring of output boxes.
+// columns (64-byte rows, 64-byte TMA swizzle).  EPI_STORE / EPI_ZH use them as
+// a ring of output boxes.  EPI_DSIGMA uses them as a double buffer for the
+// saved Z: the box of the warp's next chunk is TMA-loaded while the current
+// one is processed, and dZ is computed in place and TMA-stored from the box.
 constexpr int EPI_BOX_BYTES = 32 * 32 * 2;
 constexpr int EPI_OUT_BOXES = 2;
 constexpr int EPI_WARP_BYTES = EPI_OUT_BOXES * EPI_BOX_BYTES;
@@ -111,25 +112,45 @@ __device__ __forceinline__ float logistic_fast(float z)
     return z < -87.0f ? 0.0f : __fdividef(1.0f, 1.0f + __expf(-z));
 }
 
-__device__ __forceinline__ float act_sigma(int kind, float z)
+template <int SIG>
+__device__ __forceinline__ float act_sigma(float z)
 {
-    if (kind == SIG_SILU) return z * logistic_fast(z);
-    if (kind == SIG_GELU) return 0.5f * z * erfcf(-z * 0.70710678118654752f);
+    if (SIG == SIG_SILU) return z * logistic_fast(z);
+    if (SIG == SIG_GELU) return 0.5f * z * erfcf(-z * 0.70710678118654752f);
     return z;
 }
 
-__device__ __forceinline__ float act_dsigma(int kind, float z)
+template <int SIG>
+__device__ __forceinline__ float act_dsigma(float z)
 {
-    if (kind == SIG_SILU) {
+    if (SIG == SIG_SILU) {
         const float s = logistic_fast(z);
         return s * (1.0f + z * (1.0f - s));
     }
-    if (kind == SIG_GELU) {
+    if (SIG == SIG_GELU) {
         const float Phi = 0.5f * erfcf(-z * 0.70710678118654752f);
         const float phi = 0.39894228040143268f * __expf(-0.5f * z * z);
         return Phi + z * phi;
     }
     return 1.0f;
+}
+
+template <int SIG>
+struct SigTag {
+    static constexpr int value = SIG;
+};
+
+// Run fn(SigTag<sigma>{}) with sigma fixed at compile time, so the unrolled
+// elementwise loops carry no per-element branch on the activation kind.
+template <class Fn>
+__device__ __forceinline__ void with_sigma(int sigma, Fn&& fn)
+{
+    if (sigma == SIG_SILU)
+        fn(SigTag<SIG_SILU>{});
+    else if (sigma == SIG_GELU)
+        fn(SigTag<SIG_GELU>{});
+    else
+        fn(SigTag<SIG_IDENTITY>{});
 }
 
 // --------------------------------------------------------- bounded waits
@@ -203,7 +224,7 @@ template <int BN, bool A_MN, bool B_MN, int EPI>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
     gemm_kernel(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUtensorMap map_b,
                 const __grid_constant__ CUtensorMap map_d, const __grid_constant__ CUtensorMap map_d2,
-                const GemmParams p)
+                const __grid_constant__ CUtensorMap map_z, const GemmParams p)
 {
     using C = GemmCfg<BN>;
     constexpr int STAGES = C::STAGES;
@@ -218,7 +239,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     uint64_t* tfull_bar = bars + 2 * STAGES;   // [2]
     uint64_t* tempty_bar = tfull_bar + 2;      // [2]
     uint64_t* drain_bar = tempty_bar + 2;      // [1]
-    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain_bar + 1);
+    uint64_t* zfull_bar = drain_bar + 1;       // [NUM_EPI_WARPS][2]  Z boxes (EPI_DSIGMA)
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(zfull_bar + 2 * NUM_EPI_WARPS);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
     const int warp = threadIdx.x >> 5;
@@ -235,11 +257,13 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             mbar_init(&tempty_bar[b], NUM_EPI_WARPS * 32);
         }
         mbar_init(drain_bar, 1);
+        for (int j = 0; j < 2 * NUM_EPI_WARPS; ++j) mbar_init(&zfull_bar[j], 1);
         *abort_flag = 0;
         fence_mbar_init();
         tma_prefetch_desc(&map_a);
         tma_prefetch_desc(&map_b);
         if (EPI != EPI_F32) tma_prefetch_desc(&map_d);
+        if (EPI == EPI_DSIGMA) tma_prefetch_desc(&map_z);
     }
     if (warp == 1) {
         tmem_alloc(tmem_slot, C::TMEM_COLS);
@@ -387,12 +411,33 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         const int q = warp & 3;                 // TMEM lane quarter this warp may access
         const int half = (warp - 2) >> 2;       // the two warps of a quarter take alternate chunks
         const int row_in_tile = q * 32 + lane;
-        const uint32_t ep = smem_u32(smem_epi + (warp - 2) * EPI_WARP_BYTES);
-        int out_slot = 0;                       // next output box of the ring
+        uint8_t* ep_gen = smem_epi + (warp - 2) * EPI_WARP_BYTES;
+        const uint32_t ep = smem_u32(ep_gen);
+        uint64_t* zbar = zfull_bar + 2 * (warp - 2);
+        int out_slot = 0;                       // next output box of the ring (EPI_STORE / EPI_ZH)
         int buf = 0;
         uint32_t bphase = 0;
+        bool ok = true;
 
-        // stage one output box (this thread's row) and hand it to the TMA engine
+        // 32-column chunks of tile u that hold output rows of this warp
+        auto chunk_count = [&](int u) {
+            int m_blk, n_blk, split, kb0, kb1;
+            decode_unit(p, u, m_blk, n_blk, split, kb0, kb1);
+            if (EPI == EPI_F32) return BN / 32;
+            if (m_blk * BM + q * 32 >= p.M) return 0;   // this warp's 32 rows are all past the end
+            const int left = p.N - n_blk * BN;
+            return left >= BN ? BN / 32 : (left + 31) / 32;
+        };
+
+        // hand box `box` (already staged, fenced) to the TMA engine
+        auto store_box = [&](const CUtensorMap* map, uint32_t box, int x, int y) {
+            __syncwarp();
+            if (lane == 0) {
+                tma_store_2d(map, box, x, y);
+                bulk_commit_group();
+            }
+        };
+        // stage one output box (this thread's row) from the ring and store it
         auto emit = [&](const CUtensorMap* map, const uint32_t (&w)[16], int x, int y) {
             if (y >= p.M) return;               // whole box below the last row: nothing to store
             const uint32_t box = ep + out_slot * EPI_BOX_BYTES;
@@ -400,39 +445,52 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             __syncwarp();
             stage_row(box, lane, w);
             fence_proxy_async_smem();
-            __syncwarp();
-            if (lane == 0) {
-                tma_store_2d(map, box, x, y);
-                bulk_commit_group();
-            }
+            store_box(map, box, x, y);
             if (++out_slot == EPI_OUT_BOXES) out_slot = 0;
         };
 
-        for (int u = blockIdx.x; u < p.units; u += gridDim.x) {
+        // EPI_DSIGMA: Z boxes run one (tile, chunk) item ahead of their use
+        int zu = blockIdx.x, zc = half;         // next item whose Z box is to be loaded
+        uint32_t zphase = 0;                    // bit b: parity of the next wait on zbar[b]
+        int zload = 0, zuse = 0;
+        auto z_advance = [&]() {                // move (zu, zc) to the next item that has a chunk
+            while (zu < p.units && zc >= chunk_count(zu)) {
+                zu += gridDim.x;
+                zc = half;
+            }
+        };
+        auto z_issue = [&]() {                  // load the Z box of item (zu, zc), then step past it
+            if (zu >= p.units) return;
+            int m_blk, n_blk, split, kb0, kb1;
+            decode_unit(p, zu, m_blk, n_blk, split, kb0, kb1);
+            const int b = zload & 1;
+            if (lane == 0) {
+                bulk_wait_group_read<0>();      // the stores that last read box b are done with it
+                mbar_arrive_expect_tx(&zbar[b], EPI_BOX_BYTES);
+                tma_load_2d(&map_z, &zbar[b], ep_gen + b * EPI_BOX_BYTES, n_blk * BN + zc * 32, m_blk * BM + q * 32);
+            }
+            ++zload;
+            zc += 2;
+            z_advance();
+        };
+        if (EPI == EPI_DSIGMA) {
+            z_advance();
+            z_issue();
+        }
+
+        for (int u = blockIdx.x; u < p.units && ok; u += gridDim.x) {
             int m_blk, n_blk, split, kb0, kb1;
             decode_unit(p, u, m_blk, n_blk, split, kb0, kb1);
             const int row0 = m_blk * BM + q * 32;
             const int row = row0 + lane;
-            int nch = BN / 32;                  // chunks of 32 columns that hold valid output
-            if (n_blk * BN + BN > p.N) nch = (p.N - n_blk * BN + 31) / 32;
-            if (EPI != EPI_F32 && row0 >= p.M) nch = 0;   // this warp's 32 rows are all past the end
+            const int nch = chunk_count(u);
             if (!wait_bounded(&tfull_bar[buf], bphase, wc, ST_TIMEOUT_EPILOGUE)) break;
             tc_fence_after();
             const uint32_t tbase = tmem_base + (static_cast<uint32_t>(q * 32) << 16) + static_cast<uint32_t>(buf * BN);
 #pragma unroll 1
-            for (int c = half; c < (EPI == EPI_F32 ? BN / 32 : nch); c += 2) {
+            for (int c = half; c < nch; c += 2) {
                 const int col0 = n_blk * BN + c * 32;
-                uint4 zq[4];
-                if (EPI == EPI_DSIGMA) {        // the saved Z of this row's chunk, in flight during the TMEM load
-                    if (row < p.M) {
-                        const uint4* zs = reinterpret_cast<const uint4*>(p.z_ptr + row * p.z_ld + col0);
-#pragma unroll
-                        for (int j = 0; j < 4; ++j) zq[j] = __ldg(zs + j);
-                    } else {
-#pragma unroll
-                        for (int j = 0; j < 4; ++j) zq[j] = make_uint4(0u, 0u, 0u, 0u);
-                    }
-                }
+                if (EPI == EPI_DSIGMA) z_issue();   // the next item's Z box, while this one is processed
                 uint32_t v[32];
                 tmem_ld_32x32b_x32(tbase + c * 32, v);
                 tmem_ld_wait();
@@ -455,8 +513,11 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                         // ragged right edge: masked per-element stores, padding untouched
                         if (row < p.M) {
                             uint16_t* d = reinterpret_cast<uint16_t*>(p.d_ptr + row * p.d_ld + col0);
-                            for (int j = 0; j < p.N - col0; ++j)
-                                d[j] = static_cast<uint16_t>((j & 1) ? (w[j >> 1] >> 16) : (w[j >> 1] & 0xFFFFu));
+                            const int valid = p.N - col0;
+#pragma unroll
+                            for (int j = 0; j < 32; ++j)   // fully unrolled: w stays in registers
+                                if (j < valid)
+                                    d[j] = static_cast<uint16_t>((j & 1) ? (w[j >> 1] >> 16) : (w[j >> 1] & 0xFFFFu));
                         }
                         continue;
                     }
@@ -467,24 +528,55 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                         w[j] = pack_bf16x2(__uint_as_float(v[2 * j]), __uint_as_float(v[2 * j + 1]));
                     emit(&map_d, w, col0, row0);
                     if (p.has_d2) {
+                        with_sigma(p.sigma, [&](auto tag) {
+                            constexpr int S = decltype(tag)::value;
 #pragma unroll
-                        for (int j = 0; j < 16; ++j)
-                            w[j] = pack_bf16x2(act_sigma(p.sigma, bf16_lo(w[j])), act_sigma(p.sigma, bf16_hi(w[j])));
+                            for (int j = 0; j < 16; ++j)
+                                w[j] = pack_bf16x2(act_sigma<S>(bf16_lo(w[j])), act_sigma<S>(bf16_hi(w[j])));
+                        });
                         emit(&map_d2, w, col0, row0);
                     }
                 } else if (EPI == EPI_DSIGMA) {
-                    const uint32_t z[16] = {zq[0].x, zq[0].y, zq[0].z, zq[0].w, zq[1].x, zq[1].y, zq[1].z, zq[1].w,
-                                            zq[2].x, zq[2].y, zq[2].z, zq[2].w, zq[3].x, zq[3].y, zq[3].z, zq[3].w};
+                    const int b = zuse & 1;
+                    const bool zok = wait_bounded(&zbar[b], (zphase >> b) & 1u, wc, ST_TIMEOUT_EPILOGUE);
+                    zphase ^= 1u << b;
+                    ++zuse;
+                    if (!zok) {
+                        ok = false;
+                        break;
+                    }
+                    const uint32_t box = ep + b * EPI_BOX_BYTES;
+                    uint32_t z[16];
 #pragma unroll
-                    for (int j = 0; j < 16; ++j)
-                        w[j] = pack_bf16x2(__uint_as_float(v[2 * j]) * act_dsigma(p.sigma, bf16_lo(z[j])),
-                                           __uint_as_float(v[2 * j + 1]) * act_dsigma(p.sigma, bf16_hi(z[j])));
-                    emit(&map_d, w, col0, row0);
-                    if (p.has_d2) {
+                    for (int j = 0; j < 4; ++j) {
+                        const uint4 t = ld_shared_v4(box + box64_off(lane, j));
+                        z[4 * j] = t.x;
+                        z[4 * j + 1] = t.y;
+                        z[4 * j + 2] = t.z;
+                        z[4 * j + 3] = t.w;
+                    }
+                    with_sigma(p.sigma, [&](auto tag) {
+                        constexpr int S = decltype(tag)::value;
 #pragma unroll
                         for (int j = 0; j < 16; ++j)
-                            w[j] = pack_bf16x2(act_sigma(p.sigma, bf16_lo(z[j])), act_sigma(p.sigma, bf16_hi(z[j])));
-                        emit(&map_d2, w, col0, row0);
+                            w[j] = pack_bf16x2(__uint_as_float(v[2 * j]) * act_dsigma<S>(bf16_lo(z[j])),
+                                               __uint_as_float(v[2 * j + 1]) * act_dsigma<S>(bf16_hi(z[j])));
+                    });
+                    stage_row(box, lane, w);        // dZ in place of this row's Z
+                    fence_proxy_async_smem();
+                    store_box(&map_d, box, col0, row0);
+                    if (p.has_d2) {                 // CoLA-M: H = sigma(Z) through the same box
+                        with_sigma(p.sigma, [&](auto tag) {
+                            constexpr int S = decltype(tag)::value;
+#pragma unroll
+                            for (int j = 0; j < 16; ++j)
+                                w[j] = pack_bf16x2(act_sigma<S>(bf16_lo(z[j])), act_sigma<S>(bf16_hi(z[j])));
+                        });
+                        if (lane == 0) bulk_wait_group_read<0>();
+                        __syncwarp();
+                        stage_row(box, lane, w);
+                        fence_proxy_async_smem();
+                        store_box(&map_d2, box, col0, row0);
                     }
                 }
             }
@@ -494,6 +586,19 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                 buf = 0;
                 bphase ^= 1u;
             }
+        }
+        // Z boxes still in flight (issued ahead, or for items the loop left early)
+        while (zuse < zload) {
+            const int b = zuse & 1;
+            const uint64_t t0 = global_timer_ns();
+            while (!mbar_try_wait(&zbar[b], (zphase >> b) & 1u)) {
+                if (global_timer_ns() - t0 > WAIT_LIMIT_NS) {
+                    if (p.status) atomicOr(p.status, ST_TIMEOUT_DRAIN);
+                    break;
+                }
+            }
+            zphase ^= 1u << b;
+            ++zuse;
         }
         if (lane == 0) bulk_wait_group_all();   // every output store has landed
     }

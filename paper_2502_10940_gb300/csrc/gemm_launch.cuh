@@ -8,11 +8,12 @@
 
 namespace cola {
 
-// map_d / map_d2: bf16 output boxes {32, 32} (64-byte swizzle).  Maps an
-// epilogue does not use may be any valid map.
+// map_d / map_d2: bf16 output boxes {32, 32} (64-byte swizzle); map_z: the
+// saved Z that EPI_DSIGMA reads, same box geometry.  Maps an epilogue does
+// not use may be any valid map.
 template <int BN, bool A_MN, bool B_MN, int EPI>
 cudaError_t launch_gemm(const CUtensorMap& map_a, const CUtensorMap& map_b, const CUtensorMap& map_d,
-                        const CUtensorMap& map_d2, const GemmParams& p, int grid,
+                        const CUtensorMap& map_d2, const CUtensorMap& map_z, const GemmParams& p, int grid,
                         cudaStream_t stream);
 
 cudaError_t launch_splitk_reduce(const float* part, int splits, long long part_stride, int ldp, int M, int N,
@@ -21,7 +22,7 @@ cudaError_t launch_splitk_reduce(const float* part, int splits, long long part_s
 #ifdef COLA_DEFINE_LAUNCHERS
 template <int BN, bool A_MN, bool B_MN, int EPI>
 cudaError_t launch_gemm(const CUtensorMap& map_a, const CUtensorMap& map_b, const CUtensorMap& map_d,
-                        const CUtensorMap& map_d2, const GemmParams& p, int grid,
+                        const CUtensorMap& map_d2, const CUtensorMap& map_z, const GemmParams& p, int grid,
                         cudaStream_t stream)
 {
     constexpr int smem = GemmCfg<BN>::SMEM_BYTES;
@@ -36,7 +37,7 @@ cudaError_t launch_gemm(const CUtensorMap& map_a, const CUtensorMap& map_b, cons
         if (e != cudaSuccess) return e;
         if (dev < 64) configured |= 1ull << dev;
     }
-    kern<<<grid, NUM_THREADS, smem, stream>>>(map_a, map_b, map_d, map_d2, p);
+    kern<<<grid, NUM_THREADS, smem, stream>>>(map_a, map_b, map_d, map_d2, map_z, p);
     return cudaGetLastError();
 }
 #endif

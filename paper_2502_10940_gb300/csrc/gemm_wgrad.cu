@@ -8,55 +8,92 @@
 namespace cola {
 
 // ------------------------------------------------ split-K reduction
-// out[i, j] = sum over s = 0..splits-1 (in that order) of part[s][i][j];
-// bf16 store, or fp32 accumulate (out += sum) when accumulate_f32.
-__global__ void splitk_reduce_kernel(const float* __restrict__ part, int splits, long long part_stride,
-                                     int ldp, int M, int N, void* out, long long ldo, int accumulate_f32)
+// out[i, j] = sum over s = 0..splits-1 of part[s][i][j], bf16 store or fp32
+// accumulate (out += sum).  One block covers 32 groups of 4 consecutive
+// columns; its `ways` = min(8, splits) warps take the splits s = w, w + ways,
+// ... (one warp reads 512 contiguous bytes of a slab per split), and the
+// per-warp sums of a group are added in the fixed order w = 0..ways-1.  Every
+// run adds the same numbers in the same order: the result is deterministic.
+constexpr int RED_GROUPS = 32;
+constexpr int RED_WAYS = 8;
+
+__global__ void __launch_bounds__(RED_GROUPS * RED_WAYS)
+    splitk_reduce_kernel(const float* __restrict__ part, int splits, long long part_stride, int ldp, int M, int N,
+                         void* out, long long ldo, int accumulate_f32)
 {
-    const int groups = (N + 3) / 4;
-    const long long total = static_cast<long long>(M) * groups;
-    for (long long g = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x; g < total;
-         g += static_cast<long long>(gridDim.x) * blockDim.x) {
-        const int i = static_cast<int>(g / groups);
-        const int j = static_cast<int>(g - static_cast<long long>(i) * groups) * 4;
+    __shared__ float4 red[RED_WAYS][RED_GROUPS];
+    const int ways = blockDim.x >> 5;
+    const int gl = threadIdx.x & 31;
+    const int way = threadIdx.x >> 5;
+    const int groups_per_row = (N + 3) / 4;
+    const long long total = static_cast<long long>(M) * groups_per_row;
+    const long long g = static_cast<long long>(blockIdx.x) * RED_GROUPS + gl;
+    int i = 0, j = 0;
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (g < total) {
+        i = static_cast<int>(g / groups_per_row);
+        j = static_cast<int>(g - static_cast<long long>(i) * groups_per_row) * 4;
         const float* src = part + static_cast<long long>(i) * ldp + j;
-        float4 acc = *reinterpret_cast<const float4*>(src);
-        for (int s = 1; s < splits; ++s) {
-            const float4 t = *reinterpret_cast<const float4*>(src + s * part_stride);
+#pragma unroll 4
+        for (int sp = way; sp < splits; sp += ways) {
+            const float4 t = __ldg(reinterpret_cast<const float4*>(src + sp * part_stride));
             acc.x += t.x;
             acc.y += t.y;
             acc.z += t.z;
             acc.w += t.w;
         }
-        const float a[4] = {acc.x, acc.y, acc.z, acc.w};
-        const int valid = min(4, N - j);
-        if (accumulate_f32) {
-            float* o = reinterpret_cast<float*>(out) + static_cast<long long>(i) * ldo + j;
-            for (int e = 0; e < valid; ++e) o[e] += a[e];
+    }
+    if (ways > 1) {
+        red[way][gl] = acc;
+        __syncthreads();
+        if (way != 0) return;
+        acc = red[0][gl];
+        for (int w = 1; w < ways; ++w) {
+            const float4 t = red[w][gl];
+            acc.x += t.x;
+            acc.y += t.y;
+            acc.z += t.z;
+            acc.w += t.w;
+        }
+    }
+    if (g >= total) return;
+    const float v[4] = {acc.x, acc.y, acc.z, acc.w};
+    const int valid = min(4, N - j);
+    if (accumulate_f32) {
+        float* o = reinterpret_cast<float*>(out) + static_cast<long long>(i) * ldo + j;
+        for (int e = 0; e < valid; ++e) o[e] += v[e];
+    } else {
+        __nv_bfloat16* o = reinterpret_cast<__nv_bfloat16*>(out) + static_cast<long long>(i) * ldo + j;
+        if (valid == 4 && ((reinterpret_cast<uintptr_t>(o) & 7) == 0)) {
+            *reinterpret_cast<uint2*>(o) = make_uint2(pack_bf16x2(v[0], v[1]), pack_bf16x2(v[2], v[3]));
         } else {
-            __nv_bfloat16* o = reinterpret_cast<__nv_bfloat16*>(out) + static_cast<long long>(i) * ldo + j;
-            if (valid == 4 && ((reinterpret_cast<uintptr_t>(o) & 7) == 0)) {
-                uint2 pk = make_uint2(pack_bf16x2(a[0], a[1]), pack_bf16x2(a[2], a[3]));
-                *reinterpret_cast<uint2*>(o) = pk;
-            } else {
-                for (int e = 0; e < valid; ++e) o[e] = __float2bfloat16_rn(a[e]);
-            }
+            for (int e = 0; e < valid; ++e) o[e] = __float2bfloat16_rn(v[e]);
         }
     }
 }
 
-
+template cudaError_t launch_gemm<128, true, true, EPI_STORE>(const CUtensorMap&, const CUtensorMap&, const CUtensorMap&,
+                                                             const CUtensorMap&, const CUtensorMap&, const GemmParams&,
+                                                             int, cudaStream_t);
+template cudaError_t launch_gemm<256, true, true, EPI_STORE>(const CUtensorMap&, const CUtensorMap&, const CUtensorMap&,
+                                                             const CUtensorMap&, const CUtensorMap&, const GemmParams&,
+                                                             int, cudaStream_t);
 template cudaError_t launch_gemm<128, true, true, EPI_F32>(const CUtensorMap&, const CUtensorMap&, const CUtensorMap&,
-                                                           const CUtensorMap&, const GemmParams&, int,
+                                                           const CUtensorMap&, const CUtensorMap&, const GemmParams&, int,
                                                             cudaStream_t);
 template cudaError_t launch_gemm<256, true, true, EPI_F32>(const CUtensorMap&, const CUtensorMap&, const CUtensorMap&,
-                                                           const CUtensorMap&, const GemmParams&, int,
+                                                           const CUtensorMap&, const CUtensorMap&, const GemmParams&, int,
                                                             cudaStream_t);
 
 cudaError_t launch_splitk_reduce(const float* part, int splits, long long part_stride, int ldp, int M, int N,
                                  void* out, long long ldo, int accumulate_f32, int grid, cudaStream_t stream)
 {
-    splitk_reduce_kernel<<<grid, 256, 0, stream>>>(part, splits, part_stride, ldp, M, N, out, ldo, accumulate_f32);
+    (void)grid;   // one block per 32 column groups
+    const long long groups = static_cast<long long>(M) * ((N + 3) / 4);
+    const long long blocks = (groups + RED_GROUPS - 1) / RED_GROUPS;
+    const int ways = splits < RED_WAYS ? splits : RED_WAYS;
+    splitk_reduce_kernel<<<static_cast<unsigned>(blocks), RED_GROUPS * ways, 0, stream>>>(
+        part, splits, part_stride, ldp, M, N, out, ldo, accumulate_f32);
     return cudaGetLastError();
 }
 }  // namespace cola

@@ -92,10 +92,23 @@ GemmParams plan(int64_t M, int64_t N, int64_t K, int bn, int sms, bool split_k)
     const int tiles = p.m_tiles * p.n_tiles;
     int S = 1;
     if (split_k) {
-        S = sms / tiles;
-        const int max_s = p.k_blocks / 4;     // at least 4 k-blocks (256 tokens) per split
-        if (S > max_s) S = max_s;
-        if (S < 1) S = 1;
+        // Token split of a weight gradient: minimise (waves of persistent CTAs)
+        // x (k-blocks per unit + the cost of writing and re-reading its fp32
+        // partial tile, counted in k-blocks of operand bytes: 8 BN / (128 + BN),
+        // plus 2 for the reduction pass), at least 4 k-blocks per split.
+        const int max_s = p.k_blocks / 4 > 1 ? p.k_blocks / 4 : 1;
+        const double c_part = 8.0 * bn / (128.0 + bn) + 2.0;
+        double best = -1.0;
+        for (int s = 1; s <= max_s; ++s) {
+            const long long units = static_cast<long long>(tiles) * s;
+            const long long waves = (units + sms - 1) / sms;
+            const long long kb = (p.k_blocks + s - 1) / s;
+            const double cost = static_cast<double>(waves) * (static_cast<double>(kb) + (s > 1 ? c_part : 0.0));
+            if (best < 0 || cost < best) {
+                best = cost;
+                S = s;
+            }
+        }
     }
     p.kb_per_split = (p.k_blocks + S - 1) / S;
     p.splits = (p.k_blocks + p.kb_per_split - 1) / p.kb_per_split;
@@ -112,10 +125,10 @@ int grid_for(const GemmParams& p, int sms) { return p.units < sms ? p.units : sm
 
 template <bool A_MN, bool B_MN, int EPI>
 cudaError_t dispatch(int bn, const CUtensorMap& ma, const CUtensorMap& mb, const CUtensorMap& md,
-                     const CUtensorMap& md2, const GemmParams& p, int sms, cudaStream_t s)
+                     const CUtensorMap& md2, const CUtensorMap& mz, const GemmParams& p, int sms, cudaStream_t s)
 {
-    if (bn == 256) return launch_gemm<256, A_MN, B_MN, EPI>(ma, mb, md, md2, p, grid_for(p, sms), s);
-    return launch_gemm<128, A_MN, B_MN, EPI>(ma, mb, md, md2, p, grid_for(p, sms), s);
+    if (bn == 256) return launch_gemm<256, A_MN, B_MN, EPI>(ma, mb, md, md2, mz, p, grid_for(p, sms), s);
+    return launch_gemm<128, A_MN, B_MN, EPI>(ma, mb, md, md2, mz, p, grid_for(p, sms), s);
 }
 
 }  // namespace
