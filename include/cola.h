@@ -72,7 +72,7 @@ typedef enum {
 typedef enum {
     COLA_SIGMA_IDENTITY = 0,     /* sigma(z) = z: the plain low-rank product B A x */
     COLA_SIGMA_SILU = 1,         /* Swish / SiLU, z / (1 + e^-z) (LLaMA, Sec. 5) */
-    COLA_SIGMA_GELU = 2          /* GELU, erf form z * Phi(z) (BERT, Sec. 5.3) */
+    COLA_SIGMA_GELU = 2          /* GELU, erf form z * Phi(z) (BERT, Sec. 5.2) */
 } cola_sigma_t;
 
 typedef enum {

@@ -24,7 +24,7 @@
  *
  * Every sum runs in natural index order in fp64.  sigma in {identity, SiLU
  * (Swish, beta = 1), GELU (erf form)}; the paper names GeLU and Swish
- * (Sec. 5.3) without fixing their form.
+ * (Sec. 5.2) without fixing their form.
  *
  * round_store != 0 rounds the stored low-rank tensors Z, H and dZ to the
  * bf16 grid (round to nearest, ties to even) at the point where they are

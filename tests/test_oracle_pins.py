@@ -135,7 +135,7 @@ def test_tau_limit_of_prop_3_1():
 
 @pytest.mark.parametrize("kind", ["silu", "gelu"])
 def test_lemma_rank_one_construction(kind):
-    # Lemma (App. A): every row of A equal to u^T and B = [w, 0, ..., 0]
+    # Lemma (App. H, auxiliary lemmas): every row of A equal to u^T and B = [w, 0, ..., 0]
     # give B sigma(A X) = w sigma(u^T X) exactly.  In the backward only the
     # first column of dH is nonzero, so dA rows 1..r-1 vanish, and all
     # columns of H (hence of dB) coincide.
