@@ -273,6 +273,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem_base = *tmem_slot;
+    // The prologue above overlaps the previous kernel's tail; global memory is
+    // touched only after that kernel has completed.
+    grid_dependency_wait();
+    grid_launch_dependents();
 
     if (warp == 0) {
         // ------------------------------------------------ TMA producer

@@ -5,15 +5,15 @@
 
 namespace cola {
 template cudaError_t launch_gemm<128, false, false, EPI_ZH>(const CUtensorMap&, const CUtensorMap&, const CUtensorMap&,
-                                                            const CUtensorMap&, const CUtensorMap&, const GemmParams&, int,
+                                                            const CUtensorMap&, const CUtensorMap&, const GemmParams&, int, bool,
                                                             cudaStream_t);
 template cudaError_t launch_gemm<256, false, false, EPI_ZH>(const CUtensorMap&, const CUtensorMap&, const CUtensorMap&,
-                                                            const CUtensorMap&, const CUtensorMap&, const GemmParams&, int,
+                                                            const CUtensorMap&, const CUtensorMap&, const GemmParams&, int, bool,
                                                             cudaStream_t);
 template cudaError_t launch_gemm<128, false, false, EPI_STORE>(const CUtensorMap&, const CUtensorMap&, const CUtensorMap&,
-                                                               const CUtensorMap&, const CUtensorMap&, const GemmParams&, int,
+                                                               const CUtensorMap&, const CUtensorMap&, const GemmParams&, int, bool,
                                                             cudaStream_t);
 template cudaError_t launch_gemm<256, false, false, EPI_STORE>(const CUtensorMap&, const CUtensorMap&, const CUtensorMap&,
-                                                               const CUtensorMap&, const CUtensorMap&, const GemmParams&, int,
+                                                               const CUtensorMap&, const CUtensorMap&, const GemmParams&, int, bool,
                                                             cudaStream_t);
 }  // namespace cola

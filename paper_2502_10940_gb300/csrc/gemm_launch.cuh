@@ -11,10 +11,12 @@ namespace cola {
 // map_d / map_d2: bf16 output boxes {32, 32} (64-byte swizzle); map_z: the
 // saved Z that EPI_DSIGMA reads, same box geometry.  Maps an epilogue does
 // not use may be any valid map.
+// pdl: launch with programmatic stream serialization (the prologue overlaps
+// the previous kernel's tail).  Worth it for short launches only.
 template <int BN, bool A_MN, bool B_MN, int EPI>
 cudaError_t launch_gemm(const CUtensorMap& map_a, const CUtensorMap& map_b, const CUtensorMap& map_d,
                         const CUtensorMap& map_d2, const CUtensorMap& map_z, const GemmParams& p, int grid,
-                        cudaStream_t stream);
+                        bool pdl, cudaStream_t stream);
 
 cudaError_t launch_splitk_reduce(const float* part, int splits, long long part_stride, int ldp, int M, int N,
                                  void* out, long long ldo, int accumulate_f32, int grid, cudaStream_t stream);
@@ -23,7 +25,7 @@ cudaError_t launch_splitk_reduce(const float* part, int splits, long long part_s
 template <int BN, bool A_MN, bool B_MN, int EPI>
 cudaError_t launch_gemm(const CUtensorMap& map_a, const CUtensorMap& map_b, const CUtensorMap& map_d,
                         const CUtensorMap& map_d2, const CUtensorMap& map_z, const GemmParams& p, int grid,
-                        cudaStream_t stream)
+                        bool pdl, cudaStream_t stream)
 {
     constexpr int smem = GemmCfg<BN>::SMEM_BYTES;
     auto kern = gemm_kernel<BN, A_MN, B_MN, EPI>;
@@ -37,8 +39,19 @@ cudaError_t launch_gemm(const CUtensorMap& map_a, const CUtensorMap& map_b, cons
         if (e != cudaSuccess) return e;
         if (dev < 64) configured |= 1ull << dev;
     }
-    kern<<<grid, NUM_THREADS, smem, stream>>>(map_a, map_b, map_d, map_d2, map_z, p);
-    return cudaGetLastError();
+    // programmatic stream serialization: this kernel's prologue may overlap
+    // the tail of the previous kernel in the stream (see grid_dependency_wait)
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(grid);
+    cfg.blockDim = dim3(NUM_THREADS);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = pdl ? 1 : 0;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kern, map_a, map_b, map_d, map_d2, map_z, p);
 }
 #endif
 

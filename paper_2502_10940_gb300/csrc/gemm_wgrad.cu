@@ -22,6 +22,8 @@ __global__ void __launch_bounds__(RED_GROUPS * RED_WAYS)
                          void* out, long long ldo, int accumulate_f32)
 {
     __shared__ float4 red[RED_WAYS][RED_GROUPS];
+    grid_dependency_wait();            // the partials come from the GEMM launched just before
+    grid_launch_dependents();
     const int ways = blockDim.x >> 5;
     const int gl = threadIdx.x & 31;
     const int way = threadIdx.x >> 5;
@@ -74,15 +76,15 @@ __global__ void __launch_bounds__(RED_GROUPS * RED_WAYS)
 
 template cudaError_t launch_gemm<128, true, true, EPI_STORE>(const CUtensorMap&, const CUtensorMap&, const CUtensorMap&,
                                                              const CUtensorMap&, const CUtensorMap&, const GemmParams&,
-                                                             int, cudaStream_t);
+                                                             int, bool, cudaStream_t);
 template cudaError_t launch_gemm<256, true, true, EPI_STORE>(const CUtensorMap&, const CUtensorMap&, const CUtensorMap&,
                                                              const CUtensorMap&, const CUtensorMap&, const GemmParams&,
-                                                             int, cudaStream_t);
+                                                             int, bool, cudaStream_t);
 template cudaError_t launch_gemm<128, true, true, EPI_F32>(const CUtensorMap&, const CUtensorMap&, const CUtensorMap&,
-                                                           const CUtensorMap&, const CUtensorMap&, const GemmParams&, int,
+                                                           const CUtensorMap&, const CUtensorMap&, const GemmParams&, int, bool,
                                                             cudaStream_t);
 template cudaError_t launch_gemm<256, true, true, EPI_F32>(const CUtensorMap&, const CUtensorMap&, const CUtensorMap&,
-                                                           const CUtensorMap&, const CUtensorMap&, const GemmParams&, int,
+                                                           const CUtensorMap&, const CUtensorMap&, const GemmParams&, int, bool,
                                                             cudaStream_t);
 
 cudaError_t launch_splitk_reduce(const float* part, int splits, long long part_stride, int ldp, int M, int N,
@@ -92,8 +94,17 @@ cudaError_t launch_splitk_reduce(const float* part, int splits, long long part_s
     const long long groups = static_cast<long long>(M) * ((N + 3) / 4);
     const long long blocks = (groups + RED_GROUPS - 1) / RED_GROUPS;
     const int ways = splits < RED_WAYS ? splits : RED_WAYS;
-    splitk_reduce_kernel<<<static_cast<unsigned>(blocks), RED_GROUPS * ways, 0, stream>>>(
-        part, splits, part_stride, ldp, M, N, out, ldo, accumulate_f32);
-    return cudaGetLastError();
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(static_cast<unsigned>(blocks));
+    cfg.blockDim = dim3(RED_GROUPS * ways);
+    cfg.dynamicSmemBytes = 0;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, splitk_reduce_kernel, part, splits, part_stride, ldp, M, N, out, ldo,
+                              accumulate_f32);
 }
 }  // namespace cola

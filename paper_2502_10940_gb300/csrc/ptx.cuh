@@ -21,6 +21,16 @@ __device__ __forceinline__ uint64_t global_timer_ns()
     return t;
 }
 
+// ------------------------------------------------- programmatic dependent launch
+// Wait until every grid this one depends on (the previous kernel in the
+// stream, when launched with programmatic stream serialization) has completed
+// and its memory is visible; a no-op otherwise.
+__device__ __forceinline__ void grid_dependency_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
+// Allow the next kernel in the stream to start launching (its CTAs still wait
+// in grid_dependency_wait before touching this kernel's results).
+__device__ __forceinline__ void grid_launch_dependents() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
 // ---------------------------------------------------------------- mbarrier
 __device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count)
 {
