@@ -69,11 +69,13 @@ WsLayout ws_layout(const cola_desc_t& d, int fused, int sms)
     if (d.mode == COLA_MODE_COLA_M) off += align_up(static_cast<size_t>(d.n) * R * 2);
     L.part_off = off;
     const int bn_b = choose_bn(d.r);
-    GemmParams pb = plan(d.d_out, d.r, d.n, bn_b, sms, true);
+    const int ms_b = choose_msub(d.d_out, d.r, d.n, bn_b);
+    GemmParams pb = plan(d.d_out, d.r, d.n, bn_b, ms_b, sms, true);
     const int bn_a = choose_bn(d.d_in);
-    GemmParams pa = plan(R, d.d_in, d.n, bn_a, sms, true);
-    const size_t part_b = static_cast<size_t>(pb.splits) * partial_elems(pb, bn_b) * 4;
-    const size_t part_a = static_cast<size_t>(pa.splits) * partial_elems(pa, bn_a) * 4;
+    const int ms_a = choose_msub(R, d.d_in, d.n, bn_a);
+    GemmParams pa = plan(R, d.d_in, d.n, bn_a, ms_a, sms, true);
+    const size_t part_b = static_cast<size_t>(pb.splits) * partial_elems(pb, bn_b, ms_b) * 4;
+    const size_t part_a = static_cast<size_t>(pa.splits) * partial_elems(pa, bn_a, ms_a) * 4;
     off += align_up(part_b > part_a ? part_b : part_a);
     L.total = off;
     return L;
@@ -182,9 +184,10 @@ cola_status_t run_f1(const Shape& s, int sigma, int64_t N, const void* X, const 
                      int64_t ldz, unsigned int* status, int sms, cudaStream_t st)
 {
     const int bn = choose_bn(N);
-    GemmParams p = plan(s.n, N, s.d_in, bn, sms, false);
+    const int ms = choose_msub(s.n, N, s.d_in, bn);
+    GemmParams p = plan(s.n, N, s.d_in, bn, ms, sms, false);
     CUtensorMap ma, mb, md, md2;
-    COLA_MAP(map_kmajor(&ma, X, s.d_in, s.n, s.ld_x, BM));
+    COLA_MAP(map_kmajor(&ma, X, s.d_in, s.n, s.ld_x, BM * ms));
     COLA_MAP(map_kmajor(&mb, A, s.d_in, N, s.ld_a, bn));
     COLA_MAP(map_box32(&md, Z, N, s.n, ldz));
     if (H) COLA_MAP(map_box32(&md2, H, N, s.n, ldz));
@@ -192,7 +195,7 @@ cola_status_t run_f1(const Shape& s, int sigma, int64_t N, const void* X, const 
     p.sigma = sigma;
     p.status = status;
     return launched(traced(COLA_KERNEL_FWD_ZH, s.n, N, s.d_in, 1, H != nullptr, st, [&] {
-        return dispatch<false, false, EPI_ZH>(bn, ma, mb, md, H ? md2 : md, md, p, sms, st);
+        return dispatch<false, false, EPI_ZH>(bn, ms, ma, mb, md, H ? md2 : md, md, p, sms, st);
     }));
 }
 
@@ -201,16 +204,17 @@ cola_status_t run_f2(const Shape& s, const void* H, int64_t ldh, const void* B, 
                      int sms, cudaStream_t st)
 {
     const int bn = choose_bn(s.d_out);
-    GemmParams p = plan(s.n, s.d_out, s.r, bn, sms, false);
+    const int ms = choose_msub(s.n, s.d_out, s.r, bn);
+    GemmParams p = plan(s.n, s.d_out, s.r, bn, ms, sms, false);
     CUtensorMap ma, mb, md;
-    COLA_MAP(map_kmajor(&ma, H, s.r, s.n, ldh, BM));
+    COLA_MAP(map_kmajor(&ma, H, s.r, s.n, ldh, BM * ms));
     COLA_MAP(map_kmajor(&mb, B, s.r, s.d_out, s.r, bn));
     COLA_MAP(map_box32(&md, Y, s.d_out, s.n, s.ld_y));
     p.d_ptr = static_cast<__nv_bfloat16*>(Y);
     p.d_ld = s.ld_y;
     p.status = status;
     return launched(traced(COLA_KERNEL_FWD_Y, s.n, s.d_out, s.r, 1, 0, st, [&] {
-        return dispatch<false, false, EPI_STORE>(bn, ma, mb, md, md, md, p, sms, st);
+        return dispatch<false, false, EPI_STORE>(bn, ms, ma, mb, md, md, md, p, sms, st);
     }));
 }
 
@@ -219,9 +223,10 @@ cola_status_t run_b1(const Shape& s, int sigma, const void* dY, const void* B, c
                      void* dZ, void* Hout, unsigned int* status, int sms, cudaStream_t st)
 {
     const int bn = choose_bn(s.r);
-    GemmParams p = plan(s.n, s.r, s.d_out, bn, sms, false);
+    const int ms = choose_msub(s.n, s.r, s.d_out, bn);
+    GemmParams p = plan(s.n, s.r, s.d_out, bn, ms, sms, false);
     CUtensorMap ma, mb, md, md2, mz;
-    COLA_MAP(map_kmajor(&ma, dY, s.d_out, s.n, s.ld_y, BM));
+    COLA_MAP(map_kmajor(&ma, dY, s.d_out, s.n, s.ld_y, BM * ms));
     COLA_MAP(map_mnmajor(&mb, B, s.r, s.d_out, s.r));
     COLA_MAP(map_box32(&md, dZ, s.r, s.n, ldz));
     COLA_MAP(map_box32(&mz, Z, s.r, s.n, ldz));
@@ -230,7 +235,7 @@ cola_status_t run_b1(const Shape& s, int sigma, const void* dY, const void* B, c
     p.sigma = sigma;
     p.status = status;
     return launched(traced(COLA_KERNEL_BWD_DZ, s.n, s.r, s.d_out, 1, Hout != nullptr, st, [&] {
-        return dispatch<false, true, EPI_DSIGMA>(bn, ma, mb, md, Hout ? md2 : md, mz, p, sms, st);
+        return dispatch<false, true, EPI_DSIGMA>(bn, ms, ma, mb, md, Hout ? md2 : md, mz, p, sms, st);
     }));
 }
 
@@ -241,8 +246,9 @@ cola_status_t run_wgrad(int kind, int64_t ntok, int64_t M, int64_t N, const void
                         unsigned int* status, int sms, cudaStream_t st)
 {
     const int bn = choose_bn(N);
-    GemmParams p = plan(M, N, ntok, bn, sms, true);
-    const int64_t slab = partial_elems(p, bn);
+    const int ms = choose_msub(M, N, ntok, bn);
+    GemmParams p = plan(M, N, ntok, bn, ms, sms, true);
+    const int64_t slab = partial_elems(p, bn, ms);
     if (static_cast<size_t>(p.splits) * slab * 4 > part_bytes) return COLA_ERR_WORKSPACE;
     CUtensorMap ma, mb;
     COLA_MAP(map_mnmajor(&ma, P, M, ntok, ldp));
@@ -255,13 +261,13 @@ cola_status_t run_wgrad(int kind, int64_t ntok, int64_t M, int64_t N, const void
         p.d_ptr = static_cast<__nv_bfloat16*>(out);
         p.d_ld = ldo;
         return launched(traced(kind, M, N, ntok, 1, 0, st,
-                               [&] { return dispatch<true, true, EPI_STORE>(bn, ma, mb, md, md, md, p, sms, st); }));
+                               [&] { return dispatch<true, true, EPI_STORE>(bn, ms, ma, mb, md, md, md, p, sms, st); }));
     }
     p.D = part;
     p.ldd = p.n_tiles * bn;
     p.part_stride = slab;
     COLA_TRY(launched(traced(kind, M, N, ntok, p.splits, 0, st,
-                             [&] { return dispatch<true, true, EPI_F32>(bn, ma, mb, ma, ma, ma, p, sms, st); })));
+                             [&] { return dispatch<true, true, EPI_F32>(bn, ms, ma, mb, ma, ma, ma, p, sms, st); })));
     return launched(traced(COLA_KERNEL_REDUCE, M, N, p.splits, p.splits, 0, st, [&] {
         return launch_splitk_reduce(part, p.splits, slab, p.n_tiles * bn, static_cast<int>(M), static_cast<int>(N),
                                     out, ldo, accumulate_f32, sms * 4, st);
@@ -273,16 +279,17 @@ cola_status_t run_b4(const Shape& s, int64_t K, const void* dZ, int64_t ldz, con
                      unsigned int* status, int sms, cudaStream_t st)
 {
     const int bn = choose_bn(s.d_in);
-    GemmParams p = plan(s.n, s.d_in, K, bn, sms, false);
+    const int ms = choose_msub(s.n, s.d_in, K, bn);
+    GemmParams p = plan(s.n, s.d_in, K, bn, ms, sms, false);
     CUtensorMap ma, mb, md;
-    COLA_MAP(map_kmajor(&ma, dZ, K, s.n, ldz, BM));
+    COLA_MAP(map_kmajor(&ma, dZ, K, s.n, ldz, BM * ms));
     COLA_MAP(map_mnmajor(&mb, A, s.d_in, K, s.ld_a));
     COLA_MAP(map_box32(&md, dX, s.d_in, s.n, s.ld_x));
     p.d_ptr = static_cast<__nv_bfloat16*>(dX);
     p.d_ld = s.ld_x;
     p.status = status;
     return launched(traced(COLA_KERNEL_BWD_DX, s.n, s.d_in, K, 1, 0, st, [&] {
-        return dispatch<false, true, EPI_STORE>(bn, ma, mb, md, md, md, p, sms, st);
+        return dispatch<false, true, EPI_STORE>(bn, ms, ma, mb, md, md, md, p, sms, st);
     }));
 }
 

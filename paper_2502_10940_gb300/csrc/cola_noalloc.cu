@@ -83,8 +83,9 @@ extern "C" cola_status_t cola_wgrad_static_scratch(int64_t n_tokens, int64_t M, 
 
     // ---- plan; shrink the token split until its partials fit the static scratch
     const int bn = choose_bn(N);
-    GemmParams p = plan(M, N, n_tokens, bn, sms, true);
-    const int64_t slab = partial_elems(p, bn);
+    const int ms = choose_msub(M, N, n_tokens, bn);
+    GemmParams p = plan(M, N, n_tokens, bn, ms, sms, true);
+    const int64_t slab = partial_elems(p, bn, ms);
     const size_t slab_bytes = static_cast<size_t>(slab) * 4;
     if (slab_bytes > kStaticScratchBytes) return COLA_ERR_WORKSPACE;   // too large even unsplit
     const int max_splits = static_cast<int>(kStaticScratchBytes / slab_bytes);
@@ -106,7 +107,7 @@ extern "C" cola_status_t cola_wgrad_static_scratch(int64_t n_tokens, int64_t M, 
     p.part_stride = slab;
     p.status = nullptr;   // no workspace to report a device-side timeout through
     cudaStream_t st = static_cast<cudaStream_t>(stream);
-    if (dispatch<true, true, EPI_F32>(bn, ma, mb, ma, ma, ma, p, sms, st) != cudaSuccess) return COLA_ERR_LAUNCH;
+    if (dispatch<true, true, EPI_F32>(bn, ms, ma, mb, ma, ma, ma, p, sms, st) != cudaSuccess) return COLA_ERR_LAUNCH;
     if (launch_splitk_reduce(part, p.splits, slab, p.n_tiles * bn, static_cast<int>(M), static_cast<int>(N), D, ld_d,
                              accumulate_f32, sms * 4, st) != cudaSuccess)
         return COLA_ERR_LAUNCH;

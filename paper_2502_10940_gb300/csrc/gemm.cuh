@@ -88,17 +88,24 @@ constexpr int EPI_OUT_BOXES = 2;
 constexpr int EPI_WARP_BYTES = EPI_OUT_BOXES * EPI_BOX_BYTES;
 constexpr int EPI_SMEM_BYTES = NUM_EPI_WARPS * EPI_WARP_BYTES;
 
-template <int BN>
+// A CTA tile is MSUB x 128 rows by BN columns: MSUB = 2 runs two M = 128
+// MMAs per k-step that share one B tile (halving the B-operand traffic per
+// output row), into two TMEM accumulators of BN columns each.
+template <int BN, int MSUB>
 struct GemmCfg {
     static_assert(BN % 64 == 0 && BN >= 64 && BN <= 256, "BN must be 64..256 in steps of 64");
-    static constexpr int A_BYTES = BM * BK * 2;
+    static_assert(MSUB == 1 || MSUB == 2, "one or two 128-row sub-tiles");
+    static constexpr int TILE_M = BM * MSUB;
+    static constexpr int ACC_COLS = MSUB * BN;   // TMEM columns of one tile's accumulator
+    static_assert(2 * ACC_COLS <= 512, "double-buffered accumulator must fit TMEM");
+    static constexpr int A_BYTES = TILE_M * BK * 2;
     static constexpr int B_BYTES = BN * BK * 2;
     static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
     static constexpr int BAR_BYTES = 256;
     static constexpr int SMEM_LIMIT = 232448;   // opt-in maximum per CTA
     static constexpr int STAGES_FIT = (SMEM_LIMIT - 1024 - BAR_BYTES - EPI_SMEM_BYTES) / STAGE_BYTES;
     static constexpr int STAGES = STAGES_FIT > 8 ? 8 : STAGES_FIT;
-    static constexpr int TMEM_COLS = (2 * BN <= 128) ? 128 : (2 * BN <= 256 ? 256 : 512);
+    static constexpr int TMEM_COLS = (2 * ACC_COLS <= 128) ? 128 : (2 * ACC_COLS <= 256 ? 256 : 512);
     static constexpr int SMEM_BYTES = 1024 + STAGES * STAGE_BYTES + EPI_SMEM_BYTES + BAR_BYTES;
     static_assert(SMEM_BYTES <= SMEM_LIMIT, "shared memory budget");
 };
@@ -220,14 +227,15 @@ __device__ __forceinline__ void stage_row(uint32_t box, int lane, const uint32_t
 }
 
 // ------------------------------------------------------------ the kernel
-template <int BN, bool A_MN, bool B_MN, int EPI>
+template <int BN, int MSUB, bool A_MN, bool B_MN, int EPI>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
     gemm_kernel(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUtensorMap map_b,
                 const __grid_constant__ CUtensorMap map_d, const __grid_constant__ CUtensorMap map_d2,
                 const __grid_constant__ CUtensorMap map_z, const GemmParams p)
 {
-    using C = GemmCfg<BN>;
+    using C = GemmCfg<BN, MSUB>;
     constexpr int STAGES = C::STAGES;
+    constexpr int TILE_M = C::TILE_M;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint8_t* smem_a = smem;                              // STAGES x A_BYTES
@@ -288,7 +296,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             for (int u = blockIdx.x; u < p.units && ok; u += gridDim.x) {
                 int m_blk, n_blk, split, kb0, kb1;
                 decode_unit(p, u, m_blk, n_blk, split, kb0, kb1);
-                const int m0 = m_blk * BM, n0 = n_blk * BN;
+                const int m0 = m_blk * TILE_M, n0 = n_blk * BN;
                 for (int kb = kb0; kb < kb1; ++kb) {
                     if (!wait_bounded(&empty_bar[stage], phase ^ 1u, wc, ST_TIMEOUT_PRODUCER)) {
                         ok = false;
@@ -298,10 +306,11 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                     uint8_t* sb = smem_b + stage * C::B_BYTES;
                     mbar_arrive_expect_tx(&full_bar[stage], C::STAGE_BYTES);
                     const int k0 = kb * BK;
-                    if (A_MN) {
-                        tma_load_2d(&map_a, &full_bar[stage], sa, m0, k0);
-                        tma_load_2d(&map_a, &full_bar[stage], sa + 64 * BK * 2, m0 + 64, k0);
-                    } else {
+                    if (A_MN) {                 // 64-row boxes along M
+#pragma unroll
+                        for (int j = 0; j < TILE_M / 64; ++j)
+                            tma_load_2d(&map_a, &full_bar[stage], sa + j * 64 * BK * 2, m0 + 64 * j, k0);
+                    } else {                    // one box of TILE_M rows
                         tma_load_2d(&map_a, &full_bar[stage], sa, k0, m0);
                     }
                     if (B_MN) {
@@ -366,7 +375,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                     break;
                 }
                 tc_fence_after();
-                const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(buf * BN);
+                const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(buf * C::ACC_COLS);
                 for (int kb = kb0; kb < kb1; ++kb) {
                     if (!wait_bounded(&full_bar[stage], phase, wc, ST_TIMEOUT_MMA)) {
                         ok = false;
@@ -379,11 +388,16 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                     for (int ks = 0; ks < BK / UMMA_K; ++ks) {
                         // K-major: next 16 k = +32 bytes inside the swizzled 128-byte row.
                         // MN-major: next 16 k = +16 rows of 128 bytes.
-                        const uint64_t da = A_MN ? smem_desc_sw128(sa + ks * UMMA_K * 128, 64 * BK * 2, 1024)
-                                                 : smem_desc_sw128(sa + ks * UMMA_K * 2, 16, 1024);
                         const uint64_t db = B_MN ? smem_desc_sw128(sb + ks * UMMA_K * 128, 64 * BK * 2, 1024)
                                                  : smem_desc_sw128(sb + ks * UMMA_K * 2, 16, 1024);
-                        umma_f16(d_tmem, da, db, idesc, (kb > kb0 || ks > 0) ? 1u : 0u);
+#pragma unroll
+                        for (int sub = 0; sub < MSUB; ++sub) {
+                            // sub-tile `sub` = A rows [128 sub, 128 sub + 128): +16 KB either way
+                            const uint32_t sas = sa + sub * BM * BK * 2;
+                            const uint64_t da = A_MN ? smem_desc_sw128(sas + ks * UMMA_K * 128, 64 * BK * 2, 1024)
+                                                     : smem_desc_sw128(sas + ks * UMMA_K * 2, 16, 1024);
+                            umma_f16(d_tmem + sub * BN, da, db, idesc, (kb > kb0 || ks > 0) ? 1u : 0u);
+                        }
                     }
                     issued_any = true;
                     umma_commit(&empty_bar[stage]);   // frees the smem stage once these MMAs are done
@@ -413,8 +427,13 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     } else {
         // ------------------------------------------------ epilogue (warps 2..9)
         const int q = warp & 3;                 // TMEM lane quarter this warp may access
-        const int half = (warp - 2) >> 2;       // the two warps of a quarter take alternate chunks
-        const int row_in_tile = q * 32 + lane;
+        const int half = (warp - 2) >> 2;       // which of the two warps on this quarter
+        // MSUB == 2: each warp of a quarter owns one 128-row sub-tile and all its
+        // chunks; MSUB == 1: the two warps take alternate chunks of the one sub-tile
+        const int sub = (MSUB == 2) ? half : 0;
+        const int c_first = (MSUB == 2) ? 0 : half;
+        constexpr int C_STEP = (MSUB == 2) ? 1 : 2;
+        const int row_in_tile = sub * BM + q * 32 + lane;
         uint8_t* ep_gen = smem_epi + (warp - 2) * EPI_WARP_BYTES;
         const uint32_t ep = smem_u32(ep_gen);
         uint64_t* zbar = zfull_bar + 2 * (warp - 2);
@@ -428,7 +447,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             int m_blk, n_blk, split, kb0, kb1;
             decode_unit(p, u, m_blk, n_blk, split, kb0, kb1);
             if (EPI == EPI_F32) return BN / 32;
-            if (m_blk * BM + q * 32 >= p.M) return 0;   // this warp's 32 rows are all past the end
+            if (m_blk * TILE_M + sub * BM + q * 32 >= p.M) return 0;   // this warp's 32 rows are all past the end
             const int left = p.N - n_blk * BN;
             return left >= BN ? BN / 32 : (left + 31) / 32;
         };
@@ -454,13 +473,13 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         };
 
         // EPI_DSIGMA: Z boxes run one (tile, chunk) item ahead of their use
-        int zu = blockIdx.x, zc = half;         // next item whose Z box is to be loaded
+        int zu = blockIdx.x, zc = c_first;      // next item whose Z box is to be loaded
         uint32_t zphase = 0;                    // bit b: parity of the next wait on zbar[b]
         int zload = 0, zuse = 0;
         auto z_advance = [&]() {                // move (zu, zc) to the next item that has a chunk
             while (zu < p.units && zc >= chunk_count(zu)) {
                 zu += gridDim.x;
-                zc = half;
+                zc = c_first;
             }
         };
         auto z_issue = [&]() {                  // load the Z box of item (zu, zc), then step past it
@@ -471,10 +490,11 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             if (lane == 0) {
                 bulk_wait_group_read<0>();      // the stores that last read box b are done with it
                 mbar_arrive_expect_tx(&zbar[b], EPI_BOX_BYTES);
-                tma_load_2d(&map_z, &zbar[b], ep_gen + b * EPI_BOX_BYTES, n_blk * BN + zc * 32, m_blk * BM + q * 32);
+                tma_load_2d(&map_z, &zbar[b], ep_gen + b * EPI_BOX_BYTES, n_blk * BN + zc * 32,
+                            m_blk * TILE_M + sub * BM + q * 32);
             }
             ++zload;
-            zc += 2;
+            zc += C_STEP;
             z_advance();
         };
         if (EPI == EPI_DSIGMA) {
@@ -485,14 +505,15 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         for (int u = blockIdx.x; u < p.units && ok; u += gridDim.x) {
             int m_blk, n_blk, split, kb0, kb1;
             decode_unit(p, u, m_blk, n_blk, split, kb0, kb1);
-            const int row0 = m_blk * BM + q * 32;
+            const int row0 = m_blk * TILE_M + sub * BM + q * 32;
             const int row = row0 + lane;
             const int nch = chunk_count(u);
             if (!wait_bounded(&tfull_bar[buf], bphase, wc, ST_TIMEOUT_EPILOGUE)) break;
             tc_fence_after();
-            const uint32_t tbase = tmem_base + (static_cast<uint32_t>(q * 32) << 16) + static_cast<uint32_t>(buf * BN);
+            const uint32_t tbase = tmem_base + (static_cast<uint32_t>(q * 32) << 16) +
+                                   static_cast<uint32_t>(buf * C::ACC_COLS + sub * BN);
 #pragma unroll 1
-            for (int c = half; c < nch; c += 2) {
+            for (int c = c_first; c < nch; c += C_STEP) {
                 const int col0 = n_blk * BN + c * 32;
                 if (EPI == EPI_DSIGMA) z_issue();   // the next item's Z box, while this one is processed
                 uint32_t v[32];
@@ -500,7 +521,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                 tmem_ld_wait();
                 if (EPI == EPI_F32) {
                     float* dst = reinterpret_cast<float*>(p.D) + split * p.part_stride +
-                                 static_cast<long long>(m_blk * BM + row_in_tile) * p.ldd + col0;
+                                 static_cast<long long>(m_blk * TILE_M + row_in_tile) * p.ldd + col0;
                     float4* d4 = reinterpret_cast<float4*>(dst);
 #pragma unroll
                     for (int j = 0; j < 8; ++j)

@@ -4,16 +4,16 @@
 #include "gemm_launch.cuh"
 
 namespace cola {
-template cudaError_t launch_gemm<128, false, false, EPI_ZH>(const CUtensorMap&, const CUtensorMap&, const CUtensorMap&,
-                                                            const CUtensorMap&, const CUtensorMap&, const GemmParams&, int, bool,
-                                                            cudaStream_t);
-template cudaError_t launch_gemm<256, false, false, EPI_ZH>(const CUtensorMap&, const CUtensorMap&, const CUtensorMap&,
-                                                            const CUtensorMap&, const CUtensorMap&, const GemmParams&, int, bool,
-                                                            cudaStream_t);
-template cudaError_t launch_gemm<128, false, false, EPI_STORE>(const CUtensorMap&, const CUtensorMap&, const CUtensorMap&,
-                                                               const CUtensorMap&, const CUtensorMap&, const GemmParams&, int, bool,
-                                                            cudaStream_t);
-template cudaError_t launch_gemm<256, false, false, EPI_STORE>(const CUtensorMap&, const CUtensorMap&, const CUtensorMap&,
-                                                               const CUtensorMap&, const CUtensorMap&, const GemmParams&, int, bool,
-                                                            cudaStream_t);
+template cudaError_t launch_gemm<128, 1, false, false, EPI_ZH>(
+    const CUtensorMap&, const CUtensorMap&, const CUtensorMap&, const CUtensorMap&, const CUtensorMap&, const GemmParams&, int, bool, cudaStream_t);
+template cudaError_t launch_gemm<256, 1, false, false, EPI_ZH>(
+    const CUtensorMap&, const CUtensorMap&, const CUtensorMap&, const CUtensorMap&, const CUtensorMap&, const GemmParams&, int, bool, cudaStream_t);
+template cudaError_t launch_gemm<128, 2, false, false, EPI_ZH>(
+    const CUtensorMap&, const CUtensorMap&, const CUtensorMap&, const CUtensorMap&, const CUtensorMap&, const GemmParams&, int, bool, cudaStream_t);
+template cudaError_t launch_gemm<128, 1, false, false, EPI_STORE>(
+    const CUtensorMap&, const CUtensorMap&, const CUtensorMap&, const CUtensorMap&, const CUtensorMap&, const GemmParams&, int, bool, cudaStream_t);
+template cudaError_t launch_gemm<256, 1, false, false, EPI_STORE>(
+    const CUtensorMap&, const CUtensorMap&, const CUtensorMap&, const CUtensorMap&, const CUtensorMap&, const GemmParams&, int, bool, cudaStream_t);
+template cudaError_t launch_gemm<128, 2, false, false, EPI_STORE>(
+    const CUtensorMap&, const CUtensorMap&, const CUtensorMap&, const CUtensorMap&, const CUtensorMap&, const GemmParams&, int, bool, cudaStream_t);
 }  // namespace cola

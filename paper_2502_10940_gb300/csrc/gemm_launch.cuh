@@ -13,7 +13,7 @@ namespace cola {
 // not use may be any valid map.
 // pdl: launch with programmatic stream serialization (the prologue overlaps
 // the previous kernel's tail).  Worth it for short launches only.
-template <int BN, bool A_MN, bool B_MN, int EPI>
+template <int BN, int MSUB, bool A_MN, bool B_MN, int EPI>
 cudaError_t launch_gemm(const CUtensorMap& map_a, const CUtensorMap& map_b, const CUtensorMap& map_d,
                         const CUtensorMap& map_d2, const CUtensorMap& map_z, const GemmParams& p, int grid,
                         bool pdl, cudaStream_t stream);
@@ -22,13 +22,13 @@ cudaError_t launch_splitk_reduce(const float* part, int splits, long long part_s
                                  void* out, long long ldo, int accumulate_f32, int grid, cudaStream_t stream);
 
 #ifdef COLA_DEFINE_LAUNCHERS
-template <int BN, bool A_MN, bool B_MN, int EPI>
+template <int BN, int MSUB, bool A_MN, bool B_MN, int EPI>
 cudaError_t launch_gemm(const CUtensorMap& map_a, const CUtensorMap& map_b, const CUtensorMap& map_d,
                         const CUtensorMap& map_d2, const CUtensorMap& map_z, const GemmParams& p, int grid,
                         bool pdl, cudaStream_t stream)
 {
-    constexpr int smem = GemmCfg<BN>::SMEM_BYTES;
-    auto kern = gemm_kernel<BN, A_MN, B_MN, EPI>;
+    constexpr int smem = GemmCfg<BN, MSUB>::SMEM_BYTES;
+    auto kern = gemm_kernel<BN, MSUB, A_MN, B_MN, EPI>;
     // the opt-in shared-memory size is a per-device function attribute
     static unsigned long long configured = 0;   // bit d: set on device d
     int dev = 0;

@@ -74,18 +74,18 @@ __global__ void __launch_bounds__(RED_GROUPS * RED_WAYS)
     }
 }
 
-template cudaError_t launch_gemm<128, true, true, EPI_STORE>(const CUtensorMap&, const CUtensorMap&, const CUtensorMap&,
-                                                             const CUtensorMap&, const CUtensorMap&, const GemmParams&,
-                                                             int, bool, cudaStream_t);
-template cudaError_t launch_gemm<256, true, true, EPI_STORE>(const CUtensorMap&, const CUtensorMap&, const CUtensorMap&,
-                                                             const CUtensorMap&, const CUtensorMap&, const GemmParams&,
-                                                             int, bool, cudaStream_t);
-template cudaError_t launch_gemm<128, true, true, EPI_F32>(const CUtensorMap&, const CUtensorMap&, const CUtensorMap&,
-                                                           const CUtensorMap&, const CUtensorMap&, const GemmParams&, int, bool,
-                                                            cudaStream_t);
-template cudaError_t launch_gemm<256, true, true, EPI_F32>(const CUtensorMap&, const CUtensorMap&, const CUtensorMap&,
-                                                           const CUtensorMap&, const CUtensorMap&, const GemmParams&, int, bool,
-                                                            cudaStream_t);
+template cudaError_t launch_gemm<128, 1, true, true, EPI_STORE>(
+    const CUtensorMap&, const CUtensorMap&, const CUtensorMap&, const CUtensorMap&, const CUtensorMap&, const GemmParams&, int, bool, cudaStream_t);
+template cudaError_t launch_gemm<256, 1, true, true, EPI_STORE>(
+    const CUtensorMap&, const CUtensorMap&, const CUtensorMap&, const CUtensorMap&, const CUtensorMap&, const GemmParams&, int, bool, cudaStream_t);
+template cudaError_t launch_gemm<128, 2, true, true, EPI_STORE>(
+    const CUtensorMap&, const CUtensorMap&, const CUtensorMap&, const CUtensorMap&, const CUtensorMap&, const GemmParams&, int, bool, cudaStream_t);
+template cudaError_t launch_gemm<128, 1, true, true, EPI_F32>(
+    const CUtensorMap&, const CUtensorMap&, const CUtensorMap&, const CUtensorMap&, const CUtensorMap&, const GemmParams&, int, bool, cudaStream_t);
+template cudaError_t launch_gemm<256, 1, true, true, EPI_F32>(
+    const CUtensorMap&, const CUtensorMap&, const CUtensorMap&, const CUtensorMap&, const CUtensorMap&, const GemmParams&, int, bool, cudaStream_t);
+template cudaError_t launch_gemm<128, 2, true, true, EPI_F32>(
+    const CUtensorMap&, const CUtensorMap&, const CUtensorMap&, const CUtensorMap&, const CUtensorMap&, const GemmParams&, int, bool, cudaStream_t);
 
 cudaError_t launch_splitk_reduce(const float* part, int splits, long long part_stride, int ldp, int M, int N,
                                  void* out, long long ldo, int accumulate_f32, int grid, cudaStream_t stream)

@@ -80,14 +80,25 @@ int choose_bn(int64_t N)
     return pad256 <= pad128 ? 256 : 128;
 }
 
-GemmParams plan(int64_t M, int64_t N, int64_t K, int bn, int sms, bool split_k)
+// Rows per CTA tile: two 128-row sub-tiles sharing each B tile when the
+// accumulator fits TMEM twice over (BN = 128), M spans more than one and the
+// launch is compute-heavy (>= 64 GFLOP).  Measured: it lifts the tensor-bound
+// 1B/7B blocks by 4-6 % but slows the HBM-bound 60M block, whose short GEMMs
+// are limited by the epilogue, which a taller tile makes longer.
+int choose_msub(int64_t M, int64_t N, int64_t K, int bn)
+{
+    const double flops = 2.0 * static_cast<double>(M) * static_cast<double>(N) * static_cast<double>(K);
+    return (bn == 128 && M > BM && flops >= 64e9) ? 2 : 1;
+}
+
+GemmParams plan(int64_t M, int64_t N, int64_t K, int bn, int msub, int sms, bool split_k)
 {
     GemmParams p;
     std::memset(&p, 0, sizeof p);
     p.M = static_cast<int>(M);
     p.N = static_cast<int>(N);
     p.k_blocks = static_cast<int>((K + BK - 1) / BK);
-    p.m_tiles = static_cast<int>((M + BM - 1) / BM);
+    p.m_tiles = static_cast<int>((M + BM * msub - 1) / (BM * msub));
     p.n_tiles = static_cast<int>((N + bn - 1) / bn);
     const int tiles = p.m_tiles * p.n_tiles;
     int S = 1;
@@ -97,7 +108,7 @@ GemmParams plan(int64_t M, int64_t N, int64_t K, int bn, int sms, bool split_k)
         // partial tile, counted in k-blocks of operand bytes: 8 BN / (128 + BN),
         // plus 2 for the reduction pass), at least 4 k-blocks per split.
         const int max_s = p.k_blocks / 4 > 1 ? p.k_blocks / 4 : 1;
-        const double c_part = 8.0 * bn / (128.0 + bn) + 2.0;
+        const double c_part = 8.0 * bn * msub / (128.0 * msub + bn) + 2.0;
         double best = -1.0;
         for (int s = 1; s <= max_s; ++s) {
             const long long units = static_cast<long long>(tiles) * s;
@@ -116,15 +127,15 @@ GemmParams plan(int64_t M, int64_t N, int64_t K, int bn, int sms, bool split_k)
     return p;
 }
 
-int64_t partial_elems(const GemmParams& p, int bn)
+int64_t partial_elems(const GemmParams& p, int bn, int msub)
 {
-    return static_cast<int64_t>(p.m_tiles) * BM * p.n_tiles * bn;
+    return static_cast<int64_t>(p.m_tiles) * BM * msub * p.n_tiles * bn;
 }
 
 int grid_for(const GemmParams& p, int sms) { return p.units < sms ? p.units : sms; }
 
 template <bool A_MN, bool B_MN, int EPI>
-cudaError_t dispatch(int bn, const CUtensorMap& ma, const CUtensorMap& mb, const CUtensorMap& md,
+cudaError_t dispatch(int bn, int msub, const CUtensorMap& ma, const CUtensorMap& mb, const CUtensorMap& md,
                      const CUtensorMap& md2, const CUtensorMap& mz, const GemmParams& p, int sms, cudaStream_t s)
 {
     // Programmatic dependent launch hides launch latency and the prologue of
@@ -132,8 +143,9 @@ cudaError_t dispatch(int bn, const CUtensorMap& ma, const CUtensorMap& mb, const
     // costs ~1 % on long ones, so it is used below 64 GFLOP per launch.
     const double flops = 2.0 * p.M * p.N * (static_cast<double>(p.k_blocks) * BK);
     const bool pdl = flops < 64e9;
-    if (bn == 256) return launch_gemm<256, A_MN, B_MN, EPI>(ma, mb, md, md2, mz, p, grid_for(p, sms), pdl, s);
-    return launch_gemm<128, A_MN, B_MN, EPI>(ma, mb, md, md2, mz, p, grid_for(p, sms), pdl, s);
+    if (bn == 256) return launch_gemm<256, 1, A_MN, B_MN, EPI>(ma, mb, md, md2, mz, p, grid_for(p, sms), pdl, s);
+    if (msub == 2) return launch_gemm<128, 2, A_MN, B_MN, EPI>(ma, mb, md, md2, mz, p, grid_for(p, sms), pdl, s);
+    return launch_gemm<128, 1, A_MN, B_MN, EPI>(ma, mb, md, md2, mz, p, grid_for(p, sms), pdl, s);
 }
 
 }  // namespace

@@ -1,0 +1,74 @@
+"""GPU parity at full workload sizes, in the launch configuration bench.py
+times (one layer through cola_fwd / cola_bwd), against the fp64 oracle on
+sampled outputs the oracle computes one by one: random token rows of Z, H,
+Y and dX (row-local), random entries of dA and dB (each a full reduction
+over all n tokens).
+
+The shapes exercise the tile configurations the production workloads select
+and the small parity cases do not reach: the two-sub-tile (256-row) CTA tiles
+of compute-heavy launches in every epilogue, 256-column tiles, ragged widths
+with padded pitches (5461 -> 5464), and multi-wave token splits.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from cola_helpers import assert_close, gpu_layer, to64
+from paper_2502_10940_gb300 import inputs as I
+
+pytestmark = pytest.mark.gpu
+
+SHAPES = [
+    (65536, 2048, 5461, 512),    # LLaMA-1B gate/up: Y with 5461 columns on 256-row tiles
+    (65536, 5461, 2048, 512),    # LLaMA-1B down: K = 5461 forward, dA / dX with 5461 columns
+    (32768, 8192, 8192, 128),    # r = 128 at 68.7 GFLOP per GEMM: 256-row tiles for Z/H, dZ and dB
+]
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _cuda():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2502_10940_gb300 import build
+    build.build()
+
+
+def _full_bits(t):
+    """bf16 bits of the whole padded row-major buffer behind a view."""
+    full = torch.as_strided(t, (t.shape[0], t.stride(0)), (t.stride(0), 1))
+    return I.bf16_bits(full)
+
+
+@pytest.mark.parametrize("shape", SHAPES, ids=lambda s: "x".join(map(str, s)))
+def test_full_size_layer_sampled(shape):
+    n, d_in, d_out, r = shape
+    inp = I.layer_inputs(n, d_in, d_out, r, seed=7, device="cuda")
+    g = gpu_layer(inp, "silu", "cola")
+    torch.cuda.synchronize()
+
+    Xb, dYb = _full_bits(inp["X"]), _full_bits(inp["dY"])
+    Ab, Bb = I.bf16_bits(inp["A"]), I.bf16_bits(inp["B"])
+    rng = np.random.default_rng(1234)
+    rows = np.sort(rng.choice(n, 48, replace=False))
+    rows[-1] = n - 1                                    # the last (possibly ragged) tile
+    Z, H, Y, dZ, dX = oracle.rows_bf16(Xb, Ab, Bb, rows, dYb, "silu", d_in=d_in, d_out=d_out)
+    ridx = torch.from_numpy(rows).cuda()
+    assert_close("Z rows", to64(g["Z"][ridx]), Z)
+    assert_close("H rows", to64(g["H"][ridx]), H)
+    assert_close("Y rows", to64(g["Y"][ridx]), Y)
+    assert_close("dX rows", to64(g["dX"][ridx]), dX)
+
+    ii = rng.integers(0, r, 32)
+    kk = rng.integers(0, d_in, 32)
+    kk[-1] = d_in - 1
+    dA_o = oracle.dA_entries_bf16(Xb, Ab, Bb, dYb, ii, kk, "silu", d_out=d_out)
+    dA_g = to64(g["dA"])[ii, kk]
+    assert_close("dA entries", dA_g, dA_o)
+
+    oo = rng.integers(0, d_out, 32)
+    oo[-1] = d_out - 1
+    jj = rng.integers(0, r, 32)
+    dB_o = oracle.dB_entries_bf16(Xb, Ab, dYb, oo, jj, "silu")
+    dB_g = to64(g["dB"])[oo, jj]
+    assert_close("dB entries", dB_g, dB_o)
