@@ -165,30 +165,37 @@ class Block:
 
 
 # ---------------------------------------------------------------- per-launch accounting
-def launch_cost(kind, m, n, k, splits, flags):
-    """(algorithmic bytes, flops) of one library launch: each operand read once,
-    each result written once, bf16 (2 B); the fp32 token-split partials of the
-    weight gradients are implementation traffic and are not counted."""
+def launch_cost(kind, shapes, splits, flags):
+    """(algorithmic bytes, flops) of one library launch, summed over the GEMMs
+    it runs: each operand read once, each result written once, bf16 (2 B);
+    the fp32 token-split partials of the weight gradients are implementation
+    traffic and are not counted."""
     e = 2
-    if kind == "fwd_zh":
-        return e * (m * k + n * k + m * n * (2 if flags & 1 else 1)), 2.0 * m * n * k
-    if kind == "fwd_y":
-        return e * (m * k + n * k + m * n), 2.0 * m * n * k
-    if kind == "bwd_dz":
-        return e * (m * k + n * k + m * n * (3 if flags & 1 else 2)), 2.0 * m * n * k
-    if kind in ("wgrad_db", "wgrad_da"):
-        return e * (k * m + k * n + m * n), 2.0 * m * n * k
-    if kind == "bwd_dx":
-        return e * (m * k + n * k + m * n), 2.0 * m * n * k
-    if kind == "reduce":
-        return e * m * n, 0.0
-    return 0, 0.0
+    tb, tf = 0.0, 0.0
+    for (m, n, k) in shapes:
+        if kind == "fwd_zh":
+            b = e * (m * k + n * k + m * n * (2 if flags & 1 else 1))
+        elif kind == "fwd_y":
+            b = e * (m * k + n * k + m * n)
+        elif kind == "bwd_dz":
+            b = e * (m * k + n * k + m * n * (3 if flags & 1 else 2))
+        elif kind == "wgrad":
+            b = e * (k * m + k * n + m * n)
+        elif kind == "bwd_dx":
+            b = e * (m * k + n * k + m * n)
+        elif kind == "reduce":
+            b = e * m * n
+        else:
+            b = 0
+        tb += b
+        tf += 0.0 if kind == "reduce" else 2.0 * m * n * k
+    return tb, tf
 
 
 def summarize_trace(records, peaks, ridge):
     kinds = {}
-    for kind, m, n, k, splits, flags, ms in records:
-        b, f = launch_cost(kind, m, n, k, splits, flags)
+    for kind, shapes, splits, flags, ms in records:
+        b, f = launch_cost(kind, shapes, splits, flags)
         d = kinds.setdefault(kind, {"launches": 0, "ms": 0.0, "bytes": 0.0, "flops": 0.0})
         d["launches"] += 1
         d["ms"] += ms

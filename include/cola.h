@@ -193,27 +193,29 @@ cola_status_t cola_wgrad_static_scratch(int64_t n_tokens, int64_t M, int64_t N, 
 /* ---- launch tracing (optional; for measurement) ----
  * While a slot array is attached, every kernel the library launches is
  * bracketed by two CUDA events recorded on the launch stream: slot
- * (*count) receives the events' use, the kernel kind and the GEMM extents,
- * and *count is incremented (host side) until it reaches `capacity`.
+ * (*count) receives the events' use, the kernel kind and the extents of the
+ * GEMMs (one launch may run up to four of one kind: the q/k/v outputs, the
+ * weight gradients of a layer), and *count is incremented (host side) until
+ * it reaches `capacity`.
  * `start` / `stop` are cudaEvent_t handles the caller created with timing
  * enabled, one distinct pair per slot; the library only records them.
  * The attachment is process-wide and not thread-safe: attach, launch and
  * detach from one host thread. */
 typedef enum {
-    COLA_KERNEL_FWD_ZH = 0,      /* Z = X A^T, H = sigma(Z)              (M=n, N=r or 3r, K=d_in) */
-    COLA_KERNEL_FWD_Y = 1,       /* Y = H B^T                            (M=n, N=d_out, K=r) */
-    COLA_KERNEL_BWD_DZ = 2,      /* dZ = (dY B) * sigma'(Z)              (M=n, N=r, K=d_out) */
-    COLA_KERNEL_WGRAD_DB = 3,    /* dB partials = dY^T H, token split    (M=d_out, N=r, K=n) */
-    COLA_KERNEL_WGRAD_DA = 4,    /* dA partials = dZ^T X, token split    (M=r or 3r, N=d_in, K=n) */
-    COLA_KERNEL_REDUCE = 5,      /* fixed-order sum of the partials      (M, N of the gradient, K=splits) */
-    COLA_KERNEL_BWD_DX = 6       /* dX = dZ A                            (M=n, N=d_in, K=r or 3r) */
+    COLA_KERNEL_FWD_ZH = 0,      /* Z = X A^T, H = sigma(Z)               (M=n, N=r or 3r, K=d_in) */
+    COLA_KERNEL_FWD_Y = 1,       /* Y = H B^T                             (M=n, N=d_out, K=r) */
+    COLA_KERNEL_BWD_DZ = 2,      /* dZ = (dY B) * sigma'(Z)               (M=n, N=r, K=d_out) */
+    COLA_KERNEL_WGRAD = 3,       /* dB = dY^T H and dA = dZ^T X, token split (M=d_out | r, N=r | d_in, K=n) */
+    COLA_KERNEL_REDUCE = 4,      /* fixed-order sum of the partials       (M, N of the gradient, K=splits) */
+    COLA_KERNEL_BWD_DX = 5       /* dX = dZ A                             (M=n, N=d_in, K=r or 3r) */
 } cola_kernel_t;
 
 typedef struct {
     void* start;        /* cudaEvent_t, recorded just before the launch */
     void* stop;         /* cudaEvent_t, recorded just after the launch */
     int32_t kernel;     /* cola_kernel_t */
-    int32_t m, n, k;    /* GEMM extents of the launch */
+    int32_t count;      /* GEMMs (or reductions) this one launch runs, 1..4 */
+    int32_t mnk[4][3];  /* M, N, K of each (reductions: M, N, splits) */
     int32_t splits;     /* token splits (weight gradients), else 1 */
     int32_t flags;      /* bit 0: the epilogue also wrote H (CoLA forward or CoLA-M backward) */
 } cola_trace_slot_t;

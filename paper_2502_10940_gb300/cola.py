@@ -26,7 +26,7 @@ SYMBOLS = ("cola_workspace_size", "cola_workspace_init", "cola_fwd", "cola_bwd",
            "cola_bwd_qkv_fused", "cola_check_status", "cola_wgrad_static_scratch", "cola_trace_attach",
            "cola_trace_detach", "cola_status_string")
 STATIC_SCRATCH_BYTES = 64 * 1024 * 1024
-KERNELS = {0: "fwd_zh", 1: "fwd_y", 2: "bwd_dz", 3: "wgrad_db", 4: "wgrad_da", 5: "reduce", 6: "bwd_dx"}
+KERNELS = {0: "fwd_zh", 1: "fwd_y", 2: "bwd_dz", 3: "wgrad", 4: "reduce", 5: "bwd_dx"}
 
 
 class ColaError(RuntimeError):
@@ -44,7 +44,7 @@ class cola_desc_t(ctypes.Structure):
 
 class cola_trace_slot_t(ctypes.Structure):
     _fields_ = [("start", ctypes.c_void_p), ("stop", ctypes.c_void_p), ("kernel", ctypes.c_int32),
-                ("m", ctypes.c_int32), ("n", ctypes.c_int32), ("k", ctypes.c_int32), ("splits", ctypes.c_int32),
+                ("count", ctypes.c_int32), ("mnk", (ctypes.c_int32 * 3) * 4), ("splits", ctypes.c_int32),
                 ("flags", ctypes.c_int32)]
 
 
@@ -221,14 +221,14 @@ class Trace:
         return False
 
     def records(self):
-        """[(kernel name, m, n, k, splits, flags, ms)] of the recorded launches."""
+        """[(kernel name, [(M, N, K) of each GEMM of the launch], splits, flags, ms)]."""
         torch.cuda.synchronize()
         out = []
         for i in range(self.count.value):
             s_ = self.slots[i]
             a, b = self.events[i]
-            out.append((KERNELS.get(s_.kernel, str(s_.kernel)), s_.m, s_.n, s_.k, s_.splits, s_.flags,
-                        a.elapsed_time(b)))
+            shapes = [tuple(int(v) for v in s_.mnk[g]) for g in range(s_.count)]
+            out.append((KERNELS.get(s_.kernel, str(s_.kernel)), shapes, s_.splits, s_.flags, a.elapsed_time(b)))
         return out
 
 

@@ -46,41 +46,6 @@ cola_status_t device_info(int* sms)
     return COLA_OK;
 }
 
-// ------------------------------------------------------------ workspace
-constexpr size_t WS_HEADER = 256;
-constexpr size_t WS_ALIGN = 256;
-
-size_t align_up(size_t v) { return (v + WS_ALIGN - 1) / WS_ALIGN * WS_ALIGN; }
-
-struct WsLayout {
-    size_t dz_off, h_off, part_off, total;
-};
-
-// dZ [n x R] bf16, H [n x R] bf16 (CoLA-M only), fp32 split-K partial slabs
-// sized for the larger of the two weight-gradient GEMMs.
-WsLayout ws_layout(const cola_desc_t& d, int fused, int sms)
-{
-    const int64_t R = fused ? 3 * d.r : d.r;
-    WsLayout L;
-    size_t off = WS_HEADER;
-    L.dz_off = off;
-    off += align_up(static_cast<size_t>(d.n) * R * 2);
-    L.h_off = off;
-    if (d.mode == COLA_MODE_COLA_M) off += align_up(static_cast<size_t>(d.n) * R * 2);
-    L.part_off = off;
-    const int bn_b = choose_bn(d.r);
-    const int ms_b = choose_msub(d.d_out, d.r, d.n, bn_b);
-    GemmParams pb = plan(d.d_out, d.r, d.n, bn_b, ms_b, sms, true);
-    const int bn_a = choose_bn(d.d_in);
-    const int ms_a = choose_msub(R, d.d_in, d.n, bn_a);
-    GemmParams pa = plan(R, d.d_in, d.n, bn_a, ms_a, sms, true);
-    const size_t part_b = static_cast<size_t>(pb.splits) * partial_elems(pb, bn_b, ms_b) * 4;
-    const size_t part_a = static_cast<size_t>(pa.splits) * partial_elems(pa, bn_a, ms_a) * 4;
-    off += align_up(part_b > part_a ? part_b : part_a);
-    L.total = off;
-    return L;
-}
-
 // ------------------------------------------------------------ validation
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
@@ -122,6 +87,50 @@ cola_status_t check_ptrs(std::initializer_list<const void*> required)
     return COLA_OK;
 }
 
+// ------------------------------------------------------------ workspace
+constexpr size_t WS_HEADER = 256;
+constexpr size_t WS_ALIGN = 256;
+
+size_t align_up(size_t v) { return (v + WS_ALIGN - 1) / WS_ALIGN * WS_ALIGN; }
+
+struct WsLayout {
+    size_t dz_off, h_off, part_off, total;
+};
+
+// The weight-gradient group of one backward call: dB (per projection) and dA,
+// all reduced over the same n tokens in one launch.
+WgradPlan wgrad_plan(const cola_desc_t& d, int fused, int sms)
+{
+    const int64_t R = fused ? 3 * d.r : d.r;
+    int64_t M[MAX_GROUP], N[MAX_GROUP];
+    const int nb = fused ? 3 : 1;
+    for (int j = 0; j < nb; ++j) {
+        M[j] = d.d_out;
+        N[j] = d.r;
+    }
+    M[nb] = R;
+    N[nb] = d.d_in;
+    return plan_wgrad(M, N, nb + 1, d.n, sms);
+}
+
+// dZ [n x R] bf16, H [n x R] bf16 (CoLA-M only), the fp32 split partials of
+// the weight-gradient group.
+WsLayout ws_layout(const cola_desc_t& d, int fused, int sms)
+{
+    const int64_t R = fused ? 3 * d.r : d.r;
+    WsLayout L;
+    size_t off = WS_HEADER;
+    L.dz_off = off;
+    off += align_up(static_cast<size_t>(d.n) * R * 2);
+    L.h_off = off;
+    if (d.mode == COLA_MODE_COLA_M) off += align_up(static_cast<size_t>(d.n) * R * 2);
+    L.part_off = off;
+    const WgradPlan w = wgrad_plan(d, fused, sms);
+    if (w.splits > 1 || d.wgrad_fp32) off += align_up(static_cast<size_t>(w.part_elems) * 4);
+    L.total = off;
+    return L;
+}
+
 cola_status_t check_ws(const cola_desc_t& d, int fused, int sms, void* ws, size_t ws_bytes, WsLayout* L)
 {
     if (!ws) return COLA_ERR_INVALID;
@@ -132,37 +141,6 @@ cola_status_t check_ws(const cola_desc_t& d, int fused, int sms, void* ws, size_
 }
 
 inline cola_status_t launched(cudaError_t e) { return e == cudaSuccess ? COLA_OK : COLA_ERR_LAUNCH; }
-
-// ------------------------------------------------------------ launch tracing
-struct TraceState {
-    cola_trace_slot_t* slots = nullptr;
-    int32_t capacity = 0;
-    int32_t* count = nullptr;
-};
-TraceState g_trace;
-
-// Launch through `fn`, bracketed by the next free trace slot's events.
-template <class Fn>
-cudaError_t traced(int kind, int64_t m, int64_t n, int64_t k, int splits, int flags, cudaStream_t st, Fn&& fn)
-{
-    cola_trace_slot_t* slot = nullptr;
-    if (g_trace.slots && g_trace.count && *g_trace.count >= 0 && *g_trace.count < g_trace.capacity)
-        slot = &g_trace.slots[*g_trace.count];
-    cudaError_t e;
-    if (slot && (e = cudaEventRecord(static_cast<cudaEvent_t>(slot->start), st)) != cudaSuccess) return e;
-    if ((e = fn()) != cudaSuccess) return e;
-    if (slot) {
-        if ((e = cudaEventRecord(static_cast<cudaEvent_t>(slot->stop), st)) != cudaSuccess) return e;
-        slot->kernel = kind;
-        slot->m = static_cast<int32_t>(m);
-        slot->n = static_cast<int32_t>(n);
-        slot->k = static_cast<int32_t>(k);
-        slot->splits = splits;
-        slot->flags = flags;
-        ++*g_trace.count;
-    }
-    return cudaSuccess;
-}
 
 #define COLA_TRY(expr)                          \
     do {                                        \
@@ -178,100 +156,198 @@ cudaError_t traced(int kind, int64_t m, int64_t n, int64_t k, int splits, int fl
 uint8_t* wsb(void* ws) { return static_cast<uint8_t*>(ws); }
 unsigned int* ws_status(void* ws) { return static_cast<unsigned int*>(ws); }
 
+// ------------------------------------------------------------ launch tracing
+struct TraceState {
+    cola_trace_slot_t* slots = nullptr;
+    int32_t capacity = 0;
+    int32_t* count = nullptr;
+};
+TraceState g_trace;
+
+// Launch through `fn`, bracketed by the next free trace slot's events.
+template <class Fn>
+cudaError_t traced(int kind, int count, const int64_t (*mnk)[3], int splits, int flags, cudaStream_t st, Fn&& fn)
+{
+    cola_trace_slot_t* slot = nullptr;
+    if (g_trace.slots && g_trace.count && *g_trace.count >= 0 && *g_trace.count < g_trace.capacity)
+        slot = &g_trace.slots[*g_trace.count];
+    cudaError_t e;
+    if (slot && (e = cudaEventRecord(static_cast<cudaEvent_t>(slot->start), st)) != cudaSuccess) return e;
+    if ((e = fn()) != cudaSuccess) return e;
+    if (slot) {
+        if ((e = cudaEventRecord(static_cast<cudaEvent_t>(slot->stop), st)) != cudaSuccess) return e;
+        slot->kernel = kind;
+        slot->count = count;
+        for (int g = 0; g < MAX_GROUP; ++g)
+            for (int j = 0; j < 3; ++j) slot->mnk[g][j] = g < count ? static_cast<int32_t>(mnk[g][j]) : 0;
+        slot->splits = splits;
+        slot->flags = flags;
+        ++*g_trace.count;
+    }
+    return cudaSuccess;
+}
+
+// Launch a batch of `count` problems of one configuration, traced as one launch.
+template <bool A_MN, bool B_MN, int EPI>
+cola_status_t run_batch(int kind, int bn, int msub, const GemmProblem* probs, const int64_t (*mnk)[3], int count,
+                        int flags, int sms, cudaStream_t st)
+{
+    GemmBatch b;
+    std::memset(&b, 0, sizeof b);
+    b.count = count;
+    for (int g = 0; g < count; ++g) b.prob[g] = probs[g];
+    return launched(traced(kind, count, mnk, probs[0].p.splits, flags, st,
+                           [&] { return dispatch<A_MN, B_MN, EPI>(bn, msub, b, sms, st); }));
+}
+
 // ------------------------------------------------------------ passes
-// F1: Z = X A^T, H = sigma(Z)  (Z pitch / H pitch ldz; N = the r columns of A given)
+// F1: Z = X A^T, H = sigma(Z)  (N = r, or 3r for the fused q/k/v factors;
+// Z / H pitch ldz)
 cola_status_t run_f1(const Shape& s, int sigma, int64_t N, const void* X, const void* A, void* Z, void* H,
                      int64_t ldz, unsigned int* status, int sms, cudaStream_t st)
 {
     const int bn = choose_bn(N);
     const int ms = choose_msub(s.n, N, s.d_in, bn);
-    GemmParams p = plan(s.n, N, s.d_in, bn, ms, sms, false);
-    CUtensorMap ma, mb, md, md2;
-    COLA_MAP(map_kmajor(&ma, X, s.d_in, s.n, s.ld_x, BM * ms));
-    COLA_MAP(map_kmajor(&mb, A, s.d_in, N, s.ld_a, bn));
-    COLA_MAP(map_box32(&md, Z, N, s.n, ldz));
-    if (H) COLA_MAP(map_box32(&md2, H, N, s.n, ldz));
-    p.has_d2 = H != nullptr;
-    p.sigma = sigma;
-    p.status = status;
-    return launched(traced(COLA_KERNEL_FWD_ZH, s.n, N, s.d_in, 1, H != nullptr, st, [&] {
-        return dispatch<false, false, EPI_ZH>(bn, ms, ma, mb, md, H ? md2 : md, md, p, sms, st);
-    }));
+    GemmProblem pr;
+    std::memset(&pr, 0, sizeof pr);
+    pr.p = base_params(s.n, N, s.d_in, bn, ms);
+    COLA_MAP(map_kmajor(&pr.map_a, X, s.d_in, s.n, s.ld_x, BM * ms));
+    COLA_MAP(map_kmajor(&pr.map_b, A, s.d_in, N, s.ld_a, bn));
+    COLA_MAP(map_box32(&pr.map_d, Z, N, s.n, ldz));
+    pr.map_d2 = pr.map_d;
+    if (H) COLA_MAP(map_box32(&pr.map_d2, H, N, s.n, ldz));
+    pr.map_z = pr.map_d;
+    pr.p.has_d2 = H != nullptr;
+    pr.p.sigma = sigma;
+    pr.p.status = status;
+    const int64_t mnk[1][3] = {{s.n, N, s.d_in}};
+    return run_batch<false, false, EPI_ZH>(COLA_KERNEL_FWD_ZH, bn, ms, &pr, mnk, 1, H != nullptr, sms, st);
 }
 
-// F2: Y = H B^T  (H [n x r] with pitch ldh)
-cola_status_t run_f2(const Shape& s, const void* H, int64_t ldh, const void* B, void* Y, unsigned int* status,
-                     int sms, cudaStream_t st)
+// F2: Y_j = H_j B_j^T for `count` projections of one shape (H_j [n x r] with
+// pitch ldh; Y_j pitch ld_y), one launch
+cola_status_t run_f2(const Shape& s, int count, const void* const* H, int64_t ldh, const void* const* B,
+                     void* const* Y, unsigned int* status, int sms, cudaStream_t st)
 {
     const int bn = choose_bn(s.d_out);
     const int ms = choose_msub(s.n, s.d_out, s.r, bn);
-    GemmParams p = plan(s.n, s.d_out, s.r, bn, ms, sms, false);
-    CUtensorMap ma, mb, md;
-    COLA_MAP(map_kmajor(&ma, H, s.r, s.n, ldh, BM * ms));
-    COLA_MAP(map_kmajor(&mb, B, s.r, s.d_out, s.r, bn));
-    COLA_MAP(map_box32(&md, Y, s.d_out, s.n, s.ld_y));
-    p.d_ptr = static_cast<__nv_bfloat16*>(Y);
-    p.d_ld = s.ld_y;
-    p.status = status;
-    return launched(traced(COLA_KERNEL_FWD_Y, s.n, s.d_out, s.r, 1, 0, st, [&] {
-        return dispatch<false, false, EPI_STORE>(bn, ms, ma, mb, md, md, md, p, sms, st);
-    }));
+    GemmProblem pr[MAX_GROUP];
+    int64_t mnk[MAX_GROUP][3];
+    std::memset(pr, 0, sizeof pr);
+    for (int j = 0; j < count; ++j) {
+        pr[j].p = base_params(s.n, s.d_out, s.r, bn, ms);
+        COLA_MAP(map_kmajor(&pr[j].map_a, H[j], s.r, s.n, ldh, BM * ms));
+        COLA_MAP(map_kmajor(&pr[j].map_b, B[j], s.r, s.d_out, s.r, bn));
+        COLA_MAP(map_box32(&pr[j].map_d, Y[j], s.d_out, s.n, s.ld_y));
+        pr[j].map_d2 = pr[j].map_z = pr[j].map_d;
+        pr[j].p.d_ptr = static_cast<__nv_bfloat16*>(Y[j]);
+        pr[j].p.d_ld = s.ld_y;
+        pr[j].p.status = status;
+        mnk[j][0] = s.n;
+        mnk[j][1] = s.d_out;
+        mnk[j][2] = s.r;
+    }
+    return run_batch<false, false, EPI_STORE>(COLA_KERNEL_FWD_Y, bn, ms, pr, mnk, count, 0, sms, st);
 }
 
-// B1: dZ = (dY B) * sigma'(Z), and H = sigma(Z) when Hout != null (CoLA-M)
-cola_status_t run_b1(const Shape& s, int sigma, const void* dY, const void* B, const void* Z, int64_t ldz,
-                     void* dZ, void* Hout, unsigned int* status, int sms, cudaStream_t st)
+// B1: dZ_j = (dY_j B_j) * sigma'(Z_j) for `count` projections (Z_j, dZ_j, H_j
+// column blocks of pitch ldz); H_j = sigma(Z_j) too when Hout != null (CoLA-M)
+cola_status_t run_b1(const Shape& s, int sigma, int count, const void* const* dY, const void* const* B,
+                     const void* const* Z, int64_t ldz, void* const* dZ, void* const* Hout, unsigned int* status,
+                     int sms, cudaStream_t st)
 {
     const int bn = choose_bn(s.r);
     const int ms = choose_msub(s.n, s.r, s.d_out, bn);
-    GemmParams p = plan(s.n, s.r, s.d_out, bn, ms, sms, false);
-    CUtensorMap ma, mb, md, md2, mz;
-    COLA_MAP(map_kmajor(&ma, dY, s.d_out, s.n, s.ld_y, BM * ms));
-    COLA_MAP(map_mnmajor(&mb, B, s.r, s.d_out, s.r));
-    COLA_MAP(map_box32(&md, dZ, s.r, s.n, ldz));
-    COLA_MAP(map_box32(&mz, Z, s.r, s.n, ldz));
-    if (Hout) COLA_MAP(map_box32(&md2, Hout, s.r, s.n, ldz));
-    p.has_d2 = Hout != nullptr;
-    p.sigma = sigma;
-    p.status = status;
-    return launched(traced(COLA_KERNEL_BWD_DZ, s.n, s.r, s.d_out, 1, Hout != nullptr, st, [&] {
-        return dispatch<false, true, EPI_DSIGMA>(bn, ms, ma, mb, md, Hout ? md2 : md, mz, p, sms, st);
-    }));
+    GemmProblem pr[MAX_GROUP];
+    int64_t mnk[MAX_GROUP][3];
+    std::memset(pr, 0, sizeof pr);
+    for (int j = 0; j < count; ++j) {
+        pr[j].p = base_params(s.n, s.r, s.d_out, bn, ms);
+        COLA_MAP(map_kmajor(&pr[j].map_a, dY[j], s.d_out, s.n, s.ld_y, BM * ms));
+        COLA_MAP(map_mnmajor(&pr[j].map_b, B[j], s.r, s.d_out, s.r));
+        COLA_MAP(map_box32(&pr[j].map_d, dZ[j], s.r, s.n, ldz));
+        COLA_MAP(map_box32(&pr[j].map_z, Z[j], s.r, s.n, ldz));
+        pr[j].map_d2 = pr[j].map_d;
+        if (Hout) COLA_MAP(map_box32(&pr[j].map_d2, Hout[j], s.r, s.n, ldz));
+        pr[j].p.has_d2 = Hout != nullptr;
+        pr[j].p.sigma = sigma;
+        pr[j].p.status = status;
+        mnk[j][0] = s.n;
+        mnk[j][1] = s.r;
+        mnk[j][2] = s.d_out;
+    }
+    return run_batch<false, true, EPI_DSIGMA>(COLA_KERNEL_BWD_DZ, bn, ms, pr, mnk, count, Hout != nullptr, sms, st);
 }
 
-// Weight gradient D[M x N] = sum_t P[t, m] Q[t, n] over the n tokens, both
-// operands token-major (MN-major): split over tokens, fixed-order reduce.
-cola_status_t run_wgrad(int kind, int64_t ntok, int64_t M, int64_t N, const void* P, int64_t ldp, const void* Q,
-                        int64_t ldq, void* out, int64_t ldo, int accumulate_f32, float* part, size_t part_bytes,
-                        unsigned int* status, int sms, cudaStream_t st)
+// Weight gradients of one backward call, in one launch: D_j[M_j x N_j] =
+// sum_t P_j[t, m] Q_j[t, n] over the n tokens, both operands token-major
+// (MN-major).  Split over tokens into fp32 partial slabs (laid out one
+// gradient after another) reduced in a fixed order, or, unsplit, stored
+// directly as bf16.
+struct WgradJob {
+    const void* P;
+    int64_t ldp;
+    const void* Q;
+    int64_t ldq;
+    void* out;
+    int64_t ldo;
+};
+
+cola_status_t run_wgrad(const WgradPlan& w, int64_t ntok, const WgradJob* jobs, int accumulate_f32, float* part,
+                        size_t part_bytes, unsigned int* status, int sms, cudaStream_t st)
 {
-    const int bn = choose_bn(N);
-    const int ms = choose_msub(M, N, ntok, bn);
-    GemmParams p = plan(M, N, ntok, bn, ms, sms, true);
-    const int64_t slab = partial_elems(p, bn, ms);
-    if (static_cast<size_t>(p.splits) * slab * 4 > part_bytes) return COLA_ERR_WORKSPACE;
-    CUtensorMap ma, mb;
-    COLA_MAP(map_mnmajor(&ma, P, M, ntok, ldp));
-    COLA_MAP(map_mnmajor(&mb, Q, N, ntok, ldq));
-    p.status = status;
-    if (p.splits == 1 && !accumulate_f32) {
-        // no token split: the epilogue writes the bf16 gradient directly
-        CUtensorMap md;
-        COLA_MAP(map_box32(&md, out, N, M, ldo));
-        p.d_ptr = static_cast<__nv_bfloat16*>(out);
-        p.d_ld = ldo;
-        return launched(traced(kind, M, N, ntok, 1, 0, st,
-                               [&] { return dispatch<true, true, EPI_STORE>(bn, ms, ma, mb, md, md, md, p, sms, st); }));
+    const bool direct = w.splits == 1 && !accumulate_f32;
+    if (!direct && static_cast<size_t>(w.part_elems) * 4 > part_bytes) return COLA_ERR_WORKSPACE;
+    GemmProblem pr[MAX_GROUP];
+    int64_t mnk[MAX_GROUP][3];
+    std::memset(pr, 0, sizeof pr);
+    ReduceBatch rb;
+    std::memset(&rb, 0, sizeof rb);
+    float* slab_base = part;
+    for (int j = 0; j < w.count; ++j) {
+        const GemmParams& pj = w.p[j];
+        pr[j].p = pj;
+        COLA_MAP(map_mnmajor(&pr[j].map_a, jobs[j].P, pj.M, ntok, jobs[j].ldp));
+        COLA_MAP(map_mnmajor(&pr[j].map_b, jobs[j].Q, pj.N, ntok, jobs[j].ldq));
+        pr[j].p.status = status;
+        if (direct) {
+            COLA_MAP(map_box32(&pr[j].map_d, jobs[j].out, pj.N, pj.M, jobs[j].ldo));
+            pr[j].p.d_ptr = static_cast<__nv_bfloat16*>(jobs[j].out);
+            pr[j].p.d_ld = jobs[j].ldo;
+        } else {
+            pr[j].map_d = pr[j].map_a;
+            pr[j].p.D = slab_base;
+            pr[j].p.ldd = static_cast<long long>(pj.n_tiles) * w.bn;
+            pr[j].p.part_stride = w.slab[j];
+            ReduceJob& rj = rb.job[j];
+            rj.part = slab_base;
+            rj.part_stride = w.slab[j];
+            rj.ldp = pj.n_tiles * w.bn;
+            rj.M = pj.M;
+            rj.N = pj.N;
+            rj.out = jobs[j].out;
+            rj.ldo = jobs[j].ldo;
+            slab_base += static_cast<int64_t>(pj.splits) * w.slab[j];
+        }
+        pr[j].map_d2 = pr[j].map_z = pr[j].map_d;
+        mnk[j][0] = pj.M;
+        mnk[j][1] = pj.N;
+        mnk[j][2] = ntok;
     }
-    p.D = part;
-    p.ldd = p.n_tiles * bn;
-    p.part_stride = slab;
-    COLA_TRY(launched(traced(kind, M, N, ntok, p.splits, 0, st,
-                             [&] { return dispatch<true, true, EPI_F32>(bn, ms, ma, mb, ma, ma, ma, p, sms, st); })));
-    return launched(traced(COLA_KERNEL_REDUCE, M, N, p.splits, p.splits, 0, st, [&] {
-        return launch_splitk_reduce(part, p.splits, slab, p.n_tiles * bn, static_cast<int>(M), static_cast<int>(N),
-                                    out, ldo, accumulate_f32, sms * 4, st);
-    }));
+    if (direct)
+        return run_batch<true, true, EPI_STORE>(COLA_KERNEL_WGRAD, w.bn, w.msub, pr, mnk, w.count, 0, sms, st);
+    COLA_TRY((run_batch<true, true, EPI_F32>(COLA_KERNEL_WGRAD, w.bn, w.msub, pr, mnk, w.count, 0, sms, st)));
+    rb.count = w.count;
+    rb.splits = w.splits;
+    rb.accumulate_f32 = accumulate_f32;
+    int64_t rmnk[MAX_GROUP][3];
+    for (int j = 0; j < w.count; ++j) {
+        rmnk[j][0] = w.p[j].M;
+        rmnk[j][1] = w.p[j].N;
+        rmnk[j][2] = w.splits;
+    }
+    return launched(traced(COLA_KERNEL_REDUCE, w.count, rmnk, w.splits, 0, st,
+                           [&] { return launch_splitk_reduce(rb, st); }));
 }
 
 // B4: dX = dZ A  (dZ [n x K] pitch ldz, A [K x d_in] pitch ld_a; K = r or 3r)
@@ -280,17 +356,18 @@ cola_status_t run_b4(const Shape& s, int64_t K, const void* dZ, int64_t ldz, con
 {
     const int bn = choose_bn(s.d_in);
     const int ms = choose_msub(s.n, s.d_in, K, bn);
-    GemmParams p = plan(s.n, s.d_in, K, bn, ms, sms, false);
-    CUtensorMap ma, mb, md;
-    COLA_MAP(map_kmajor(&ma, dZ, K, s.n, ldz, BM * ms));
-    COLA_MAP(map_mnmajor(&mb, A, s.d_in, K, s.ld_a));
-    COLA_MAP(map_box32(&md, dX, s.d_in, s.n, s.ld_x));
-    p.d_ptr = static_cast<__nv_bfloat16*>(dX);
-    p.d_ld = s.ld_x;
-    p.status = status;
-    return launched(traced(COLA_KERNEL_BWD_DX, s.n, s.d_in, K, 1, 0, st, [&] {
-        return dispatch<false, true, EPI_STORE>(bn, ms, ma, mb, md, md, md, p, sms, st);
-    }));
+    GemmProblem pr;
+    std::memset(&pr, 0, sizeof pr);
+    pr.p = base_params(s.n, s.d_in, K, bn, ms);
+    COLA_MAP(map_kmajor(&pr.map_a, dZ, K, s.n, ldz, BM * ms));
+    COLA_MAP(map_mnmajor(&pr.map_b, A, s.d_in, K, s.ld_a));
+    COLA_MAP(map_box32(&pr.map_d, dX, s.d_in, s.n, s.ld_x));
+    pr.map_d2 = pr.map_z = pr.map_d;
+    pr.p.d_ptr = static_cast<__nv_bfloat16*>(dX);
+    pr.p.d_ld = s.ld_x;
+    pr.p.status = status;
+    const int64_t mnk[1][3] = {{s.n, s.d_in, K}};
+    return run_batch<false, true, EPI_STORE>(COLA_KERNEL_BWD_DX, bn, ms, &pr, mnk, 1, 0, sms, st);
 }
 
 }  // namespace
@@ -335,7 +412,10 @@ cola_status_t cola_fwd(const cola_desc_t* desc, const void* X, const void* A, co
     unsigned int* status = ws_status(ws);
     void* H = cola_m ? static_cast<void*>(wsb(ws) + L.h_off) : H_save;
     COLA_TRY(run_f1(s, desc->sigma, s.r, X, A, Z_save, H, s.r, status, sms, st));
-    return run_f2(s, H, s.r, B, Y, status, sms, st);
+    const void* Hs[1] = {H};
+    const void* Bs[1] = {B};
+    void* Ys[1] = {Y};
+    return run_f2(s, 1, Hs, s.r, Bs, Ys, status, sms, st);
 }
 
 cola_status_t cola_bwd(const cola_desc_t* desc, const void* X, const void* A, const void* B, const void* dY,
@@ -358,12 +438,17 @@ cola_status_t cola_bwd(const cola_desc_t* desc, const void* X, const void* A, co
     void* Hrec = cola_m ? static_cast<void*>(wsb(ws) + L.h_off) : nullptr;
     float* part = reinterpret_cast<float*>(wsb(ws) + L.part_off);
     const size_t part_bytes = L.total - L.part_off;
-    const int acc = desc->wgrad_fp32;
 
-    COLA_TRY(run_b1(s, desc->sigma, dY, B, Z_save, s.r, dZ, Hrec, status, sms, st));
+    const void* dYs[1] = {dY};
+    const void* Bs[1] = {B};
+    const void* Zs[1] = {Z_save};
+    void* dZs[1] = {dZ};
+    void* Hs[1] = {Hrec};
+    COLA_TRY(run_b1(s, desc->sigma, 1, dYs, Bs, Zs, s.r, dZs, cola_m ? Hs : nullptr, status, sms, st));
     const void* Hsrc = cola_m ? Hrec : H_save;
-    COLA_TRY(run_wgrad(COLA_KERNEL_WGRAD_DB, s.n, s.d_out, s.r, dY, s.ld_y, Hsrc, s.r, dB, s.r, acc, part, part_bytes, status, sms, st));
-    COLA_TRY(run_wgrad(COLA_KERNEL_WGRAD_DA, s.n, s.r, s.d_in, dZ, s.r, X, s.ld_x, dA, s.ld_a, acc, part, part_bytes, status, sms, st));
+    const WgradPlan w = wgrad_plan(*desc, 0, sms);
+    const WgradJob jobs[2] = {{dY, s.ld_y, Hsrc, s.r, dB, s.r}, {dZ, s.r, X, s.ld_x, dA, s.ld_a}};
+    COLA_TRY(run_wgrad(w, s.n, jobs, desc->wgrad_fp32, part, part_bytes, status, sms, st));
     return run_b4(s, s.r, dZ, s.r, A, dX, status, sms, st);
 }
 
@@ -384,13 +469,13 @@ cola_status_t cola_fwd_qkv_fused(const cola_desc_t* desc, const void* X, const v
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     unsigned int* status = ws_status(ws);
     const int64_t R = 3 * s.r;
+    const size_t slice = static_cast<size_t>(s.r) * 2;   // bytes between the q, k, v column blocks
     uint8_t* H = cola_m ? wsb(ws) + L.h_off : static_cast<uint8_t*>(H_qkv);
     COLA_TRY(run_f1(s, desc->sigma, R, X, A_qkv, Z_qkv, H, R, status, sms, st));
+    const void* Hs[3] = {H, H + slice, H + 2 * slice};
     const void* Bs[3] = {B_q, B_k, B_v};
     void* Ys[3] = {Y_q, Y_k, Y_v};
-    for (int j = 0; j < 3; ++j)
-        COLA_TRY(run_f2(s, H + static_cast<size_t>(j) * s.r * 2, R, Bs[j], Ys[j], status, sms, st));
-    return COLA_OK;
+    return run_f2(s, 3, Hs, R, Bs, Ys, status, sms, st);
 }
 
 cola_status_t cola_bwd_qkv_fused(const cola_desc_t* desc, const void* X, const void* A_qkv, const void* B_q,
@@ -416,19 +501,21 @@ cola_status_t cola_bwd_qkv_fused(const cola_desc_t* desc, const void* X, const v
     uint8_t* Hrec = cola_m ? wsb(ws) + L.h_off : nullptr;
     float* part = reinterpret_cast<float*>(wsb(ws) + L.part_off);
     const size_t part_bytes = L.total - L.part_off;
-    const int acc = desc->wgrad_fp32;
-    const void* Bs[3] = {B_q, B_k, B_v};
-    const void* dYs[3] = {dY_q, dY_k, dY_v};
-    void* dBs[3] = {dB_q, dB_k, dB_v};
     const uint8_t* Zb = static_cast<const uint8_t*>(Z_qkv);
     const uint8_t* Hsrc = cola_m ? Hrec : static_cast<const uint8_t*>(H_qkv);
-    for (int j = 0; j < 3; ++j) {
-        COLA_TRY(run_b1(s, desc->sigma, dYs[j], Bs[j], Zb + j * slice, R, dZ + j * slice,
-                        Hrec ? Hrec + j * slice : nullptr, status, sms, st));
-        COLA_TRY(run_wgrad(COLA_KERNEL_WGRAD_DB, s.n, s.d_out, s.r, dYs[j], s.ld_y, Hsrc + j * slice, R, dBs[j], s.r, acc, part,
-                           part_bytes, status, sms, st));
-    }
-    COLA_TRY(run_wgrad(COLA_KERNEL_WGRAD_DA, s.n, R, s.d_in, dZ, R, X, s.ld_x, dA_qkv, s.ld_a, acc, part, part_bytes, status, sms, st));
+
+    const void* dYs[3] = {dY_q, dY_k, dY_v};
+    const void* Bs[3] = {B_q, B_k, B_v};
+    const void* Zs[3] = {Zb, Zb + slice, Zb + 2 * slice};
+    void* dZs[3] = {dZ, dZ + slice, dZ + 2 * slice};
+    void* Hr[3] = {Hrec, Hrec + slice, Hrec + 2 * slice};
+    COLA_TRY(run_b1(s, desc->sigma, 3, dYs, Bs, Zs, R, dZs, cola_m ? Hr : nullptr, status, sms, st));
+    const WgradPlan w = wgrad_plan(*desc, 1, sms);
+    const WgradJob jobs[4] = {{dY_q, s.ld_y, Hsrc, R, dB_q, s.r},
+                              {dY_k, s.ld_y, Hsrc + slice, R, dB_k, s.r},
+                              {dY_v, s.ld_y, Hsrc + 2 * slice, R, dB_v, s.r},
+                              {dZ, R, X, s.ld_x, dA_qkv, s.ld_a}};
+    COLA_TRY(run_wgrad(w, s.n, jobs, desc->wgrad_fp32, part, part_bytes, status, sms, st));
     return run_b4(s, R, dZ, R, A_qkv, dX, status, sms, st);
 }
 

@@ -16,6 +16,7 @@
 #include <cuda_runtime.h>
 
 #include <cstdint>
+#include <cstring>
 #include <mutex>
 
 #include "cola.h"
@@ -82,34 +83,44 @@ extern "C" cola_status_t cola_wgrad_static_scratch(int64_t n_tokens, int64_t M, 
     if (major != 10 || minor != 3) return COLA_ERR_UNSUPPORTED;
 
     // ---- plan; shrink the token split until its partials fit the static scratch
-    const int bn = choose_bn(N);
-    const int ms = choose_msub(M, N, n_tokens, bn);
-    GemmParams p = plan(M, N, n_tokens, bn, ms, sms, true);
-    const int64_t slab = partial_elems(p, bn, ms);
-    const size_t slab_bytes = static_cast<size_t>(slab) * 4;
+    const int64_t Ms[1] = {M}, Ns[1] = {N};
+    WgradPlan w = plan_wgrad(Ms, Ns, 1, n_tokens, sms);
+    const size_t slab_bytes = static_cast<size_t>(w.slab[0]) * 4;
     if (slab_bytes > kStaticScratchBytes) return COLA_ERR_WORKSPACE;   // too large even unsplit
     const int max_splits = static_cast<int>(kStaticScratchBytes / slab_bytes);
-    if (p.splits > max_splits) {
-        p.kb_per_split = (p.k_blocks + max_splits - 1) / max_splits;
-        p.splits = (p.k_blocks + p.kb_per_split - 1) / p.kb_per_split;
-        p.units = p.m_tiles * p.n_tiles * p.splits;
-    }
+    if (w.p[0].splits > max_splits) set_splits(w.p[0], max_splits);
 
     // ---- set-up: the scratch's device address on this device (first call only)
     void* scratch = nullptr;
     if (scratch_address(dev, &scratch) != cudaSuccess || scratch == nullptr) return COLA_ERR_LAUNCH;
 
-    CUtensorMap ma, mb;
-    if (!map_mnmajor(&ma, P, M, n_tokens, ld_p) || !map_mnmajor(&mb, Q, N, n_tokens, ld_q)) return COLA_ERR_LAUNCH;
-    float* part = static_cast<float*>(scratch);
-    p.D = part;
-    p.ldd = p.n_tiles * bn;
-    p.part_stride = slab;
-    p.status = nullptr;   // no workspace to report a device-side timeout through
-    cudaStream_t st = static_cast<cudaStream_t>(stream);
-    if (dispatch<true, true, EPI_F32>(bn, ms, ma, mb, ma, ma, ma, p, sms, st) != cudaSuccess) return COLA_ERR_LAUNCH;
-    if (launch_splitk_reduce(part, p.splits, slab, p.n_tiles * bn, static_cast<int>(M), static_cast<int>(N), D, ld_d,
-                             accumulate_f32, sms * 4, st) != cudaSuccess)
+    GemmBatch b;
+    std::memset(&b, 0, sizeof b);
+    b.count = 1;
+    GemmProblem& pr = b.prob[0];
+    pr.p = w.p[0];
+    if (!map_mnmajor(&pr.map_a, P, M, n_tokens, ld_p) || !map_mnmajor(&pr.map_b, Q, N, n_tokens, ld_q))
         return COLA_ERR_LAUNCH;
+    pr.map_d = pr.map_d2 = pr.map_z = pr.map_a;
+    float* part = static_cast<float*>(scratch);
+    pr.p.D = part;
+    pr.p.ldd = static_cast<long long>(pr.p.n_tiles) * w.bn;
+    pr.p.part_stride = w.slab[0];
+    pr.p.status = nullptr;   // no workspace to report a device-side timeout through
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    if (dispatch<true, true, EPI_F32>(w.bn, w.msub, b, sms, st) != cudaSuccess) return COLA_ERR_LAUNCH;
+    ReduceBatch rb;
+    std::memset(&rb, 0, sizeof rb);
+    rb.count = 1;
+    rb.splits = pr.p.splits;
+    rb.accumulate_f32 = accumulate_f32;
+    rb.job[0].part = part;
+    rb.job[0].part_stride = w.slab[0];
+    rb.job[0].ldp = pr.p.n_tiles * w.bn;
+    rb.job[0].M = static_cast<int>(M);
+    rb.job[0].N = static_cast<int>(N);
+    rb.job[0].out = D;
+    rb.job[0].ldo = ld_d;
+    if (launch_splitk_reduce(rb, st) != cudaSuccess) return COLA_ERR_LAUNCH;
     return COLA_OK;
 }

@@ -193,6 +193,40 @@ __device__ __forceinline__ void decode_unit(const GemmParams& p, int u, int& m_b
     kb1 = min(kb0 + p.kb_per_split, p.k_blocks);
 }
 
+constexpr int MAX_GROUP = 4;
+
+// One GEMM of a batch: its operand / output tensor maps and parameters.
+struct GemmProblem {
+    CUtensorMap map_a, map_b, map_d, map_d2, map_z;
+    GemmParams p;
+    int unit_begin;   // first batch-wide unit index of this problem
+};
+
+// Up to MAX_GROUP independent GEMMs of one configuration (tile shape,
+// operand majors, epilogue) run by a single persistent launch; their work
+// units are numbered consecutively, problem after problem.
+struct GemmBatch {
+    GemmProblem prob[MAX_GROUP];
+    int count;
+    int units;
+};
+
+struct Unit {
+    int g, m_blk, n_blk, split, kb0, kb1;
+};
+
+__device__ __forceinline__ Unit decode(const GemmBatch& b, int u)
+{
+    int g = 0;
+#pragma unroll
+    for (int j = 1; j < MAX_GROUP; ++j)
+        if (j < b.count && u >= b.prob[j].unit_begin) g = j;
+    Unit x;
+    x.g = g;
+    decode_unit(b.prob[g].p, u - b.prob[g].unit_begin, x.m_blk, x.n_blk, x.split, x.kb0, x.kb1);
+    return x;
+}
+
 __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi)
 {
     __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
@@ -229,9 +263,7 @@ __device__ __forceinline__ void stage_row(uint32_t box, int lane, const uint32_t
 // ------------------------------------------------------------ the kernel
 template <int BN, int MSUB, bool A_MN, bool B_MN, int EPI>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
-    gemm_kernel(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUtensorMap map_b,
-                const __grid_constant__ CUtensorMap map_d, const __grid_constant__ CUtensorMap map_d2,
-                const __grid_constant__ CUtensorMap map_z, const GemmParams p)
+    gemm_kernel(const __grid_constant__ GemmBatch batch)
 {
     using C = GemmCfg<BN, MSUB>;
     constexpr int STAGES = C::STAGES;
@@ -253,7 +285,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
-    const WaitCtx wc{abort_flag, p.status};
+    unsigned int* const status = batch.prob[0].p.status;
+    const WaitCtx wc{abort_flag, status};
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < STAGES; ++s) {
@@ -268,10 +301,12 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         for (int j = 0; j < 2 * NUM_EPI_WARPS; ++j) mbar_init(&zfull_bar[j], 1);
         *abort_flag = 0;
         fence_mbar_init();
-        tma_prefetch_desc(&map_a);
-        tma_prefetch_desc(&map_b);
-        if (EPI != EPI_F32) tma_prefetch_desc(&map_d);
-        if (EPI == EPI_DSIGMA) tma_prefetch_desc(&map_z);
+        for (int g = 0; g < batch.count; ++g) {
+            tma_prefetch_desc(&batch.prob[g].map_a);
+            tma_prefetch_desc(&batch.prob[g].map_b);
+            if (EPI != EPI_F32) tma_prefetch_desc(&batch.prob[g].map_d);
+            if (EPI == EPI_DSIGMA) tma_prefetch_desc(&batch.prob[g].map_z);
+        }
     }
     if (warp == 1) {
         tmem_alloc(tmem_slot, C::TMEM_COLS);
@@ -293,11 +328,12 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             uint32_t phase = 0;
             long long issued = 0;
             bool ok = true;
-            for (int u = blockIdx.x; u < p.units && ok; u += gridDim.x) {
-                int m_blk, n_blk, split, kb0, kb1;
-                decode_unit(p, u, m_blk, n_blk, split, kb0, kb1);
-                const int m0 = m_blk * TILE_M, n0 = n_blk * BN;
-                for (int kb = kb0; kb < kb1; ++kb) {
+            for (int u = blockIdx.x; u < batch.units && ok; u += gridDim.x) {
+                const Unit x = decode(batch, u);
+                const CUtensorMap* map_a = &batch.prob[x.g].map_a;
+                const CUtensorMap* map_b = &batch.prob[x.g].map_b;
+                const int m0 = x.m_blk * TILE_M, n0 = x.n_blk * BN;
+                for (int kb = x.kb0; kb < x.kb1; ++kb) {
                     if (!wait_bounded(&empty_bar[stage], phase ^ 1u, wc, ST_TIMEOUT_PRODUCER)) {
                         ok = false;
                         break;
@@ -309,16 +345,16 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                     if (A_MN) {                 // 64-row boxes along M
 #pragma unroll
                         for (int j = 0; j < TILE_M / 64; ++j)
-                            tma_load_2d(&map_a, &full_bar[stage], sa + j * 64 * BK * 2, m0 + 64 * j, k0);
+                            tma_load_2d(map_a, &full_bar[stage], sa + j * 64 * BK * 2, m0 + 64 * j, k0);
                     } else {                    // one box of TILE_M rows
-                        tma_load_2d(&map_a, &full_bar[stage], sa, k0, m0);
+                        tma_load_2d(map_a, &full_bar[stage], sa, k0, m0);
                     }
                     if (B_MN) {
 #pragma unroll
                         for (int j = 0; j < BN / 64; ++j)
-                            tma_load_2d(&map_b, &full_bar[stage], sb + j * 64 * BK * 2, n0 + 64 * j, k0);
+                            tma_load_2d(map_b, &full_bar[stage], sb + j * 64 * BK * 2, n0 + 64 * j, k0);
                     } else {
-                        tma_load_2d(&map_b, &full_bar[stage], sb, k0, n0);
+                        tma_load_2d(map_b, &full_bar[stage], sb, k0, n0);
                     }
                     ++issued;
                     if (++stage == STAGES) {
@@ -350,7 +386,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                     const uint64_t t0 = global_timer_ns();
                     while (!mbar_try_wait(&full_bar[s], ph)) {
                         if (global_timer_ns() - t0 > WAIT_LIMIT_NS) {
-                            if (p.status) atomicOr(p.status, ST_TIMEOUT_DRAIN);
+                            if (status) atomicOr(status, ST_TIMEOUT_DRAIN);
                             break;
                         }
                     }
@@ -367,9 +403,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             uint32_t bphase = 0;
             bool ok = true;
             bool issued_any = false;
-            for (int u = blockIdx.x; u < p.units && ok; u += gridDim.x) {
-                int m_blk, n_blk, split, kb0, kb1;
-                decode_unit(p, u, m_blk, n_blk, split, kb0, kb1);
+            for (int u = blockIdx.x; u < batch.units && ok; u += gridDim.x) {
+                const Unit x = decode(batch, u);
+                const int kb0 = x.kb0, kb1 = x.kb1;
                 if (!wait_bounded(&tempty_bar[buf], bphase ^ 1u, wc, ST_TIMEOUT_MMA)) {
                     ok = false;
                     break;
@@ -418,7 +454,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                 const uint64_t t0 = global_timer_ns();
                 while (!mbar_try_wait(drain_bar, 0)) {
                     if (global_timer_ns() - t0 > WAIT_LIMIT_NS) {
-                        if (p.status) atomicOr(p.status, ST_TIMEOUT_DRAIN);
+                        if (status) atomicOr(status, ST_TIMEOUT_DRAIN);
                         break;
                     }
                 }
@@ -442,15 +478,16 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         uint32_t bphase = 0;
         bool ok = true;
 
-        // 32-column chunks of tile u that hold output rows of this warp
+        // 32-column chunks of unit u that hold output rows of this warp
         auto chunk_count = [&](int u) {
-            int m_blk, n_blk, split, kb0, kb1;
-            decode_unit(p, u, m_blk, n_blk, split, kb0, kb1);
+            const Unit x = decode(batch, u);
+            const GemmParams& pu = batch.prob[x.g].p;
             if (EPI == EPI_F32) return BN / 32;
-            if (m_blk * TILE_M + sub * BM + q * 32 >= p.M) return 0;   // this warp's 32 rows are all past the end
-            const int left = p.N - n_blk * BN;
+            if (x.m_blk * TILE_M + sub * BM + q * 32 >= pu.M) return 0;   // this warp's 32 rows are all past the end
+            const int left = pu.N - x.n_blk * BN;
             return left >= BN ? BN / 32 : (left + 31) / 32;
         };
+        int cur_M = 0;                          // output rows of the tile in hand
 
         // hand box `box` (already staged, fenced) to the TMA engine
         auto store_box = [&](const CUtensorMap* map, uint32_t box, int x, int y) {
@@ -462,7 +499,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         };
         // stage one output box (this thread's row) from the ring and store it
         auto emit = [&](const CUtensorMap* map, const uint32_t (&w)[16], int x, int y) {
-            if (y >= p.M) return;               // whole box below the last row: nothing to store
+            if (y >= cur_M) return;             // whole box below the last row: nothing to store
             const uint32_t box = ep + out_slot * EPI_BOX_BYTES;
             if (lane == 0) bulk_wait_group_read<EPI_OUT_BOXES - 1>();   // its previous store has read it
             __syncwarp();
@@ -477,21 +514,20 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         uint32_t zphase = 0;                    // bit b: parity of the next wait on zbar[b]
         int zload = 0, zuse = 0;
         auto z_advance = [&]() {                // move (zu, zc) to the next item that has a chunk
-            while (zu < p.units && zc >= chunk_count(zu)) {
+            while (zu < batch.units && zc >= chunk_count(zu)) {
                 zu += gridDim.x;
                 zc = c_first;
             }
         };
         auto z_issue = [&]() {                  // load the Z box of item (zu, zc), then step past it
-            if (zu >= p.units) return;
-            int m_blk, n_blk, split, kb0, kb1;
-            decode_unit(p, zu, m_blk, n_blk, split, kb0, kb1);
+            if (zu >= batch.units) return;
+            const Unit x = decode(batch, zu);
             const int b = zload & 1;
             if (lane == 0) {
                 bulk_wait_group_read<0>();      // the stores that last read box b are done with it
                 mbar_arrive_expect_tx(&zbar[b], EPI_BOX_BYTES);
-                tma_load_2d(&map_z, &zbar[b], ep_gen + b * EPI_BOX_BYTES, n_blk * BN + zc * 32,
-                            m_blk * TILE_M + sub * BM + q * 32);
+                tma_load_2d(&batch.prob[x.g].map_z, &zbar[b], ep_gen + b * EPI_BOX_BYTES, x.n_blk * BN + zc * 32,
+                            x.m_blk * TILE_M + sub * BM + q * 32);
             }
             ++zload;
             zc += C_STEP;
@@ -502,9 +538,13 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             z_issue();
         }
 
-        for (int u = blockIdx.x; u < p.units && ok; u += gridDim.x) {
-            int m_blk, n_blk, split, kb0, kb1;
-            decode_unit(p, u, m_blk, n_blk, split, kb0, kb1);
+        for (int u = blockIdx.x; u < batch.units && ok; u += gridDim.x) {
+            const Unit x = decode(batch, u);
+            const GemmParams& p = batch.prob[x.g].p;
+            const CUtensorMap* map_d = &batch.prob[x.g].map_d;
+            const CUtensorMap* map_d2 = &batch.prob[x.g].map_d2;
+            const int m_blk = x.m_blk, n_blk = x.n_blk, split = x.split;
+            cur_M = p.M;
             const int row0 = m_blk * TILE_M + sub * BM + q * 32;
             const int row = row0 + lane;
             const int nch = chunk_count(u);
@@ -546,12 +586,12 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                         }
                         continue;
                     }
-                    emit(&map_d, w, col0, row0);
+                    emit(map_d, w, col0, row0);
                 } else if (EPI == EPI_ZH) {
 #pragma unroll
                     for (int j = 0; j < 16; ++j)
                         w[j] = pack_bf16x2(__uint_as_float(v[2 * j]), __uint_as_float(v[2 * j + 1]));
-                    emit(&map_d, w, col0, row0);
+                    emit(map_d, w, col0, row0);
                     if (p.has_d2) {
                         with_sigma(p.sigma, [&](auto tag) {
                             constexpr int S = decltype(tag)::value;
@@ -559,7 +599,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                             for (int j = 0; j < 16; ++j)
                                 w[j] = pack_bf16x2(act_sigma<S>(bf16_lo(w[j])), act_sigma<S>(bf16_hi(w[j])));
                         });
-                        emit(&map_d2, w, col0, row0);
+                        emit(map_d2, w, col0, row0);
                     }
                 } else if (EPI == EPI_DSIGMA) {
                     const int b = zuse & 1;
@@ -589,7 +629,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                     });
                     stage_row(box, lane, w);        // dZ in place of this row's Z
                     fence_proxy_async_smem();
-                    store_box(&map_d, box, col0, row0);
+                    store_box(map_d, box, col0, row0);
                     if (p.has_d2) {                 // CoLA-M: H = sigma(Z) through the same box
                         with_sigma(p.sigma, [&](auto tag) {
                             constexpr int S = decltype(tag)::value;
@@ -601,7 +641,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                         __syncwarp();
                         stage_row(box, lane, w);
                         fence_proxy_async_smem();
-                        store_box(&map_d2, box, col0, row0);
+                        store_box(map_d2, box, col0, row0);
                     }
                 }
             }
@@ -618,7 +658,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             const uint64_t t0 = global_timer_ns();
             while (!mbar_try_wait(&zbar[b], (zphase >> b) & 1u)) {
                 if (global_timer_ns() - t0 > WAIT_LIMIT_NS) {
-                    if (p.status) atomicOr(p.status, ST_TIMEOUT_DRAIN);
+                    if (status) atomicOr(status, ST_TIMEOUT_DRAIN);
                     break;
                 }
             }

@@ -5,16 +5,10 @@
 #include "gemm_launch.cuh"
 
 namespace cola {
-template cudaError_t launch_gemm<128, 1, false, true, EPI_DSIGMA>(
-    const CUtensorMap&, const CUtensorMap&, const CUtensorMap&, const CUtensorMap&, const CUtensorMap&, const GemmParams&, int, bool, cudaStream_t);
-template cudaError_t launch_gemm<256, 1, false, true, EPI_DSIGMA>(
-    const CUtensorMap&, const CUtensorMap&, const CUtensorMap&, const CUtensorMap&, const CUtensorMap&, const GemmParams&, int, bool, cudaStream_t);
-template cudaError_t launch_gemm<128, 2, false, true, EPI_DSIGMA>(
-    const CUtensorMap&, const CUtensorMap&, const CUtensorMap&, const CUtensorMap&, const CUtensorMap&, const GemmParams&, int, bool, cudaStream_t);
-template cudaError_t launch_gemm<128, 1, false, true, EPI_STORE>(
-    const CUtensorMap&, const CUtensorMap&, const CUtensorMap&, const CUtensorMap&, const CUtensorMap&, const GemmParams&, int, bool, cudaStream_t);
-template cudaError_t launch_gemm<256, 1, false, true, EPI_STORE>(
-    const CUtensorMap&, const CUtensorMap&, const CUtensorMap&, const CUtensorMap&, const CUtensorMap&, const GemmParams&, int, bool, cudaStream_t);
-template cudaError_t launch_gemm<128, 2, false, true, EPI_STORE>(
-    const CUtensorMap&, const CUtensorMap&, const CUtensorMap&, const CUtensorMap&, const CUtensorMap&, const GemmParams&, int, bool, cudaStream_t);
+template cudaError_t launch_gemm<128, 1, false, true, EPI_DSIGMA>(const GemmBatch&, int, bool, cudaStream_t);
+template cudaError_t launch_gemm<256, 1, false, true, EPI_DSIGMA>(const GemmBatch&, int, bool, cudaStream_t);
+template cudaError_t launch_gemm<128, 2, false, true, EPI_DSIGMA>(const GemmBatch&, int, bool, cudaStream_t);
+template cudaError_t launch_gemm<128, 1, false, true, EPI_STORE>(const GemmBatch&, int, bool, cudaStream_t);
+template cudaError_t launch_gemm<256, 1, false, true, EPI_STORE>(const GemmBatch&, int, bool, cudaStream_t);
+template cudaError_t launch_gemm<128, 2, false, true, EPI_STORE>(const GemmBatch&, int, bool, cudaStream_t);
 }  // namespace cola

@@ -4,16 +4,10 @@
 #include "gemm_launch.cuh"
 
 namespace cola {
-template cudaError_t launch_gemm<128, 1, false, false, EPI_ZH>(
-    const CUtensorMap&, const CUtensorMap&, const CUtensorMap&, const CUtensorMap&, const CUtensorMap&, const GemmParams&, int, bool, cudaStream_t);
-template cudaError_t launch_gemm<256, 1, false, false, EPI_ZH>(
-    const CUtensorMap&, const CUtensorMap&, const CUtensorMap&, const CUtensorMap&, const CUtensorMap&, const GemmParams&, int, bool, cudaStream_t);
-template cudaError_t launch_gemm<128, 2, false, false, EPI_ZH>(
-    const CUtensorMap&, const CUtensorMap&, const CUtensorMap&, const CUtensorMap&, const CUtensorMap&, const GemmParams&, int, bool, cudaStream_t);
-template cudaError_t launch_gemm<128, 1, false, false, EPI_STORE>(
-    const CUtensorMap&, const CUtensorMap&, const CUtensorMap&, const CUtensorMap&, const CUtensorMap&, const GemmParams&, int, bool, cudaStream_t);
-template cudaError_t launch_gemm<256, 1, false, false, EPI_STORE>(
-    const CUtensorMap&, const CUtensorMap&, const CUtensorMap&, const CUtensorMap&, const CUtensorMap&, const GemmParams&, int, bool, cudaStream_t);
-template cudaError_t launch_gemm<128, 2, false, false, EPI_STORE>(
-    const CUtensorMap&, const CUtensorMap&, const CUtensorMap&, const CUtensorMap&, const CUtensorMap&, const GemmParams&, int, bool, cudaStream_t);
+template cudaError_t launch_gemm<128, 1, false, false, EPI_ZH>(const GemmBatch&, int, bool, cudaStream_t);
+template cudaError_t launch_gemm<256, 1, false, false, EPI_ZH>(const GemmBatch&, int, bool, cudaStream_t);
+template cudaError_t launch_gemm<128, 2, false, false, EPI_ZH>(const GemmBatch&, int, bool, cudaStream_t);
+template cudaError_t launch_gemm<128, 1, false, false, EPI_STORE>(const GemmBatch&, int, bool, cudaStream_t);
+template cudaError_t launch_gemm<256, 1, false, false, EPI_STORE>(const GemmBatch&, int, bool, cudaStream_t);
+template cudaError_t launch_gemm<128, 2, false, false, EPI_STORE>(const GemmBatch&, int, bool, cudaStream_t);
 }  // namespace cola

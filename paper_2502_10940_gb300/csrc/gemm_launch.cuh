@@ -8,24 +8,35 @@
 
 namespace cola {
 
-// map_d / map_d2: bf16 output boxes {32, 32} (64-byte swizzle); map_z: the
-// saved Z that EPI_DSIGMA reads, same box geometry.  Maps an epilogue does
-// not use may be any valid map.
-// pdl: launch with programmatic stream serialization (the prologue overlaps
-// the previous kernel's tail).  Worth it for short launches only.
+// Launch the GEMM kernel over a batch of problems (see GemmBatch).  pdl:
+// launch with programmatic stream serialization (the prologue overlaps the
+// previous kernel's tail).
 template <int BN, int MSUB, bool A_MN, bool B_MN, int EPI>
-cudaError_t launch_gemm(const CUtensorMap& map_a, const CUtensorMap& map_b, const CUtensorMap& map_d,
-                        const CUtensorMap& map_d2, const CUtensorMap& map_z, const GemmParams& p, int grid,
-                        bool pdl, cudaStream_t stream);
+cudaError_t launch_gemm(const GemmBatch& batch, int grid, bool pdl, cudaStream_t stream);
 
-cudaError_t launch_splitk_reduce(const float* part, int splits, long long part_stride, int ldp, int M, int N,
-                                 void* out, long long ldo, int accumulate_f32, int grid, cudaStream_t stream);
+// One fixed-order reduction of fp32 split partials into a gradient.
+struct ReduceJob {
+    const float* part;          // splits slabs of part_stride elements
+    long long part_stride;
+    int ldp;                    // row pitch of a slab
+    int M, N;
+    void* out;                  // bf16 (or fp32 when accumulating)
+    long long ldo;
+    long long block_begin;      // first block of this job in the launch
+};
+
+struct ReduceBatch {
+    ReduceJob job[MAX_GROUP];
+    int count;
+    int splits;
+    int accumulate_f32;
+};
+
+cudaError_t launch_splitk_reduce(ReduceBatch& batch, cudaStream_t stream);
 
 #ifdef COLA_DEFINE_LAUNCHERS
 template <int BN, int MSUB, bool A_MN, bool B_MN, int EPI>
-cudaError_t launch_gemm(const CUtensorMap& map_a, const CUtensorMap& map_b, const CUtensorMap& map_d,
-                        const CUtensorMap& map_d2, const CUtensorMap& map_z, const GemmParams& p, int grid,
-                        bool pdl, cudaStream_t stream)
+cudaError_t launch_gemm(const GemmBatch& batch, int grid, bool pdl, cudaStream_t stream)
 {
     constexpr int smem = GemmCfg<BN, MSUB>::SMEM_BYTES;
     auto kern = gemm_kernel<BN, MSUB, A_MN, B_MN, EPI>;
@@ -39,8 +50,6 @@ cudaError_t launch_gemm(const CUtensorMap& map_a, const CUtensorMap& map_b, cons
         if (e != cudaSuccess) return e;
         if (dev < 64) configured |= 1ull << dev;
     }
-    // programmatic stream serialization: this kernel's prologue may overlap
-    // the tail of the previous kernel in the stream (see grid_dependency_wait)
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(grid);
     cfg.blockDim = dim3(NUM_THREADS);
@@ -51,7 +60,7 @@ cudaError_t launch_gemm(const CUtensorMap& map_a, const CUtensorMap& map_b, cons
     attr[0].val.programmaticStreamSerializationAllowed = pdl ? 1 : 0;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, kern, map_a, map_b, map_d, map_d2, map_z, p);
+    return cudaLaunchKernelEx(&cfg, kern, batch);
 }
 #endif
 

@@ -91,7 +91,8 @@ int choose_msub(int64_t M, int64_t N, int64_t K, int bn)
     return (bn == 128 && M > BM && flops >= 64e9) ? 2 : 1;
 }
 
-GemmParams plan(int64_t M, int64_t N, int64_t K, int bn, int msub, int sms, bool split_k)
+// Tile grid of one GEMM, without a token split.
+GemmParams base_params(int64_t M, int64_t N, int64_t K, int bn, int msub)
 {
     GemmParams p;
     std::memset(&p, 0, sizeof p);
@@ -100,31 +101,41 @@ GemmParams plan(int64_t M, int64_t N, int64_t K, int bn, int msub, int sms, bool
     p.k_blocks = static_cast<int>((K + BK - 1) / BK);
     p.m_tiles = static_cast<int>((M + BM * msub - 1) / (BM * msub));
     p.n_tiles = static_cast<int>((N + bn - 1) / bn);
-    const int tiles = p.m_tiles * p.n_tiles;
+    p.kb_per_split = p.k_blocks;
+    p.splits = 1;
+    p.units = p.m_tiles * p.n_tiles;
+    return p;
+}
+
+// Token split of weight-gradient GEMMs sharing one launch (same K): minimise
+// (waves of persistent CTAs) x (k-blocks per unit + the cost of writing and
+// re-reading its fp32 partial tile, counted in k-blocks of operand bytes:
+// 8 BN msub / (128 msub + BN), plus 2 for the reduction pass), with at least
+// 4 k-blocks per split.
+int choose_splits(int tiles, int k_blocks, int bn, int msub, int sms)
+{
+    const int max_s = k_blocks / 4 > 1 ? k_blocks / 4 : 1;
+    const double c_part = 8.0 * bn * msub / (128.0 * msub + bn) + 2.0;
+    double best = -1.0;
     int S = 1;
-    if (split_k) {
-        // Token split of a weight gradient: minimise (waves of persistent CTAs)
-        // x (k-blocks per unit + the cost of writing and re-reading its fp32
-        // partial tile, counted in k-blocks of operand bytes: 8 BN / (128 + BN),
-        // plus 2 for the reduction pass), at least 4 k-blocks per split.
-        const int max_s = p.k_blocks / 4 > 1 ? p.k_blocks / 4 : 1;
-        const double c_part = 8.0 * bn * msub / (128.0 * msub + bn) + 2.0;
-        double best = -1.0;
-        for (int s = 1; s <= max_s; ++s) {
-            const long long units = static_cast<long long>(tiles) * s;
-            const long long waves = (units + sms - 1) / sms;
-            const long long kb = (p.k_blocks + s - 1) / s;
-            const double cost = static_cast<double>(waves) * (static_cast<double>(kb) + (s > 1 ? c_part : 0.0));
-            if (best < 0 || cost < best) {
-                best = cost;
-                S = s;
-            }
+    for (int s = 1; s <= max_s; ++s) {
+        const long long units = static_cast<long long>(tiles) * s;
+        const long long waves = (units + sms - 1) / sms;
+        const long long kb = (k_blocks + s - 1) / s;
+        const double cost = static_cast<double>(waves) * (static_cast<double>(kb) + (s > 1 ? c_part : 0.0));
+        if (best < 0 || cost < best) {
+            best = cost;
+            S = s;
         }
     }
+    return S;
+}
+
+void set_splits(GemmParams& p, int S)
+{
     p.kb_per_split = (p.k_blocks + S - 1) / S;
     p.splits = (p.k_blocks + p.kb_per_split - 1) / p.kb_per_split;
-    p.units = tiles * p.splits;
-    return p;
+    p.units = p.m_tiles * p.n_tiles * p.splits;
 }
 
 int64_t partial_elems(const GemmParams& p, int bn, int msub)
@@ -132,20 +143,63 @@ int64_t partial_elems(const GemmParams& p, int bn, int msub)
     return static_cast<int64_t>(p.m_tiles) * BM * msub * p.n_tiles * bn;
 }
 
-int grid_for(const GemmParams& p, int sms) { return p.units < sms ? p.units : sms; }
+// Weight-gradient group plan: count GEMMs D_i[M_i x N_i] = sum over the same
+// ntok tokens, run by one launch with one tile configuration and one split.
+struct WgradPlan {
+    int bn, msub, splits, count;
+    GemmParams p[MAX_GROUP];
+    int64_t slab[MAX_GROUP];       // fp32 elements per split slab of each GEMM
+    int64_t part_elems;            // all slabs of all splits
+};
 
-template <bool A_MN, bool B_MN, int EPI>
-cudaError_t dispatch(int bn, int msub, const CUtensorMap& ma, const CUtensorMap& mb, const CUtensorMap& md,
-                     const CUtensorMap& md2, const CUtensorMap& mz, const GemmParams& p, int sms, cudaStream_t s)
+WgradPlan plan_wgrad(const int64_t* M, const int64_t* N, int count, int64_t ntok, int sms)
 {
-    // Programmatic dependent launch hides launch latency and the prologue of
-    // short GEMMs (measured: -8 % step time on the HBM-bound 60M block) but
-    // costs ~1 % on long ones, so it is used below 64 GFLOP per launch.
-    const double flops = 2.0 * p.M * p.N * (static_cast<double>(p.k_blocks) * BK);
+    WgradPlan w;
+    std::memset(&w, 0, sizeof w);
+    w.count = count;
+    w.bn = 256;
+    for (int i = 0; i < count; ++i) w.bn = choose_bn(N[i]) < w.bn ? choose_bn(N[i]) : w.bn;
+    w.msub = 2;
+    for (int i = 0; i < count; ++i) {
+        const int ms = choose_msub(M[i], N[i], ntok, w.bn);
+        w.msub = ms < w.msub ? ms : w.msub;
+    }
+    int tiles = 0;
+    for (int i = 0; i < count; ++i) {
+        w.p[i] = base_params(M[i], N[i], ntok, w.bn, w.msub);
+        tiles += w.p[i].m_tiles * w.p[i].n_tiles;
+    }
+    const int S = choose_splits(tiles, w.p[0].k_blocks, w.bn, w.msub, sms);
+    w.part_elems = 0;
+    for (int i = 0; i < count; ++i) {
+        set_splits(w.p[i], S);
+        w.slab[i] = partial_elems(w.p[i], w.bn, w.msub);
+        w.part_elems += static_cast<int64_t>(w.p[i].splits) * w.slab[i];
+    }
+    w.splits = w.p[0].splits;
+    return w;
+}
+
+// Launch one batch (all problems of one configuration).  Programmatic
+// dependent launch hides launch latency and the prologue of short GEMMs
+// (measured: -8 % step time on the HBM-bound 60M block) but costs ~1 % on
+// long ones, so it is used below 64 GFLOP per launch.
+template <bool A_MN, bool B_MN, int EPI>
+cudaError_t dispatch(int bn, int msub, GemmBatch& b, int sms, cudaStream_t s)
+{
+    double flops = 0.0;
+    int units = 0;
+    for (int g = 0; g < b.count; ++g) {
+        b.prob[g].unit_begin = units;
+        units += b.prob[g].p.units;
+        flops += 2.0 * b.prob[g].p.M * b.prob[g].p.N * (static_cast<double>(b.prob[g].p.k_blocks) * BK);
+    }
+    b.units = units;
+    const int grid = units < sms ? units : sms;
     const bool pdl = flops < 64e9;
-    if (bn == 256) return launch_gemm<256, 1, A_MN, B_MN, EPI>(ma, mb, md, md2, mz, p, grid_for(p, sms), pdl, s);
-    if (msub == 2) return launch_gemm<128, 2, A_MN, B_MN, EPI>(ma, mb, md, md2, mz, p, grid_for(p, sms), pdl, s);
-    return launch_gemm<128, 1, A_MN, B_MN, EPI>(ma, mb, md, md2, mz, p, grid_for(p, sms), pdl, s);
+    if (bn == 256) return launch_gemm<256, 1, A_MN, B_MN, EPI>(b, grid, pdl, s);
+    if (msub == 2) return launch_gemm<128, 2, A_MN, B_MN, EPI>(b, grid, pdl, s);
+    return launch_gemm<128, 1, A_MN, B_MN, EPI>(b, grid, pdl, s);
 }
 
 }  // namespace
