@@ -67,8 +67,11 @@ class Block:
         for li, L in enumerate(wl.layers):
             if L.x not in self.X:
                 self.X[L.x] = I.activation(n, L.d_in, seed, device, layer=100 + len(self.X))
-        names = [L.name for L in wl.layers]
-        self.qkv = wl.fused_qkv and all(k in names for k in ("q", "k", "v"))
+        # projections that read one X with equal shapes (q/k/v, gate/up) run
+        # through the shared-input entry points: one A-GEMM with N = count*r
+        groups = {}
+        for li, L in enumerate(wl.layers):
+            groups.setdefault(L.x, []).append(li)
         self.layers = []
         for li, L in enumerate(wl.layers):
             t = I.layer_inputs(n, L.d_in, L.d_out, L.r, seed=seed, device=device, layer=li, with_x=False)
@@ -78,35 +81,32 @@ class Block:
             st["Y"] = torch.empty((n, ldy), dtype=bf, device=device)[:, :L.d_out]
             st["desc"] = cola.desc(n, L.d_in, L.d_out, L.r, ld_x=cola.ld_of(X), ld_y=ldy, ld_a=cola.ld_of(t["A"]),
                                    sigma=sigma, mode=mode)
+            st["dB"] = torch.empty((L.d_out, L.r), dtype=bf, device=device)
             self.layers.append(st)
+        self.groups = []
         self.ws_bytes = 0
-        self.plain = [s for s in self.layers if not (self.qkv and s["L"].name in ("q", "k", "v"))]
-        for s in self.plain:
-            L = s["L"]
-            s["Z"] = torch.empty((n, L.r), dtype=bf, device=device)
-            s["H"] = torch.empty((n, L.r), dtype=bf, device=device) if mode == "cola" else None
-            ldx = cola.ld_of(s["X"])
-            s["dX"] = torch.empty((n, ldx), dtype=bf, device=device)[:, :L.d_in]
-            s["dA"] = torch.empty((L.r, ldx), dtype=bf, device=device)[:, :L.d_in]
-            s["dB"] = torch.empty((L.d_out, L.r), dtype=bf, device=device)
-            self.ws_bytes = max(self.ws_bytes, cola.cola_workspace_size(s["desc"], 0))
-        if self.qkv:
-            q = [s for s in self.layers if s["L"].name in ("q", "k", "v")]
-            self.q3 = q
-            L = q[0]["L"]
-            r3 = 3 * L.r
-            ldx = cola.ld_of(q[0]["X"])
-            A3 = torch.empty((r3, ldx), dtype=bf, device=device)[:, :L.d_in]
-            for j, s in enumerate(q):
-                A3[j * L.r:(j + 1) * L.r].copy_(s["A"])
-            self.A_qkv = A3
-            self.Z_qkv = torch.empty((n, r3), dtype=bf, device=device)
-            self.H_qkv = torch.empty((n, r3), dtype=bf, device=device) if mode == "cola" else None
-            self.dX_qkv = torch.empty((n, ldx), dtype=bf, device=device)[:, :L.d_in]
-            self.dA_qkv = torch.empty((r3, ldx), dtype=bf, device=device)[:, :L.d_in]
-            for s in q:
-                s["dB"] = torch.empty((L.d_out, L.r), dtype=bf, device=device)
-            self.ws_bytes = max(self.ws_bytes, cola.cola_workspace_size(q[0]["desc"], 1))
+        for key, idx in groups.items():
+            mem = [self.layers[i] for i in idx]
+            L = mem[0]["L"]
+            fuse = (wl.fused_qkv and 2 <= len(mem) <= 3
+                    and all((m["L"].d_out, m["L"].r) == (L.d_out, L.r) for m in mem))
+            parts = [mem] if fuse else [[m] for m in mem]
+            for part in parts:
+                c = len(part)
+                ldx = cola.ld_of(part[0]["X"])
+                g = dict(members=part, desc=part[0]["desc"], X=part[0]["X"])
+                if c == 1:
+                    g["A"] = part[0]["A"]
+                else:
+                    g["A"] = torch.empty((c * L.r, ldx), dtype=bf, device=device)[:, :L.d_in]
+                    for j, m in enumerate(part):
+                        g["A"][j * L.r:(j + 1) * L.r].copy_(m["A"])
+                g["Z"] = torch.empty((n, c * L.r), dtype=bf, device=device)
+                g["H"] = torch.empty((n, c * L.r), dtype=bf, device=device) if mode == "cola" else None
+                g["dX"] = torch.empty((n, ldx), dtype=bf, device=device)[:, :L.d_in]
+                g["dA"] = torch.empty((c * L.r, ldx), dtype=bf, device=device)[:, :L.d_in]
+                self.ws_bytes = max(self.ws_bytes, cola.cola_workspace_size(g["desc"], c))
+                self.groups.append(g)
         self.ws = torch.empty(self.ws_bytes, dtype=torch.uint8, device=device)
         cola.cola_workspace_init(self.ws)
         self.launches_per_step = None
@@ -116,30 +116,30 @@ class Block:
         return list(self.X.values()) + [s["dY"] for s in self.layers]
 
     def step_results(self):
-        out = [s["dA"] for s in self.plain] + [s["dB"] for s in self.layers]
-        if self.qkv:
-            out.append(self.dA_qkv)
-        return out
+        return [g["dA"] for g in self.groups] + [s["dB"] for s in self.layers]
 
     def forward(self):
         c = self.cola
-        if self.qkv:
-            q, k, v = self.q3
-            c.cola_fwd_qkv_fused(q["desc"], q["X"], self.A_qkv, q["B"], k["B"], v["B"], q["Y"], k["Y"], v["Y"],
-                                 self.Z_qkv, self.H_qkv, self.ws)
-        for s in self.plain:
-            c.cola_fwd(s["desc"], s["X"], s["A"], s["B"], s["Y"], s["Z"], s["H"], self.ws)
+        for g in self.groups:
+            m = g["members"]
+            if len(m) == 1:
+                s = m[0]
+                c.cola_fwd(g["desc"], g["X"], g["A"], s["B"], s["Y"], g["Z"], g["H"], self.ws)
+            else:
+                c.cola_fwd_shared_x(g["desc"], g["X"], g["A"], [s["B"] for s in m], [s["Y"] for s in m], g["Z"],
+                                    g["H"], self.ws)
 
     def backward(self):
         c = self.cola
-        for s in reversed(self.plain):
-            c.cola_bwd(s["desc"], s["X"], s["A"], s["B"], s["dY"], s["Z"], s["H"], s["dX"], s["dA"], s["dB"],
-                       self.ws)
-        if self.qkv:
-            q, k, v = self.q3
-            c.cola_bwd_qkv_fused(q["desc"], q["X"], self.A_qkv, q["B"], k["B"], v["B"], q["dY"], k["dY"], v["dY"],
-                                 self.Z_qkv, self.H_qkv, self.dX_qkv, self.dA_qkv, q["dB"], k["dB"], v["dB"],
-                                 self.ws)
+        for g in reversed(self.groups):
+            m = g["members"]
+            if len(m) == 1:
+                s = m[0]
+                c.cola_bwd(g["desc"], g["X"], g["A"], s["B"], s["dY"], g["Z"], g["H"], g["dX"], g["dA"], s["dB"],
+                           self.ws)
+            else:
+                c.cola_bwd_shared_x(g["desc"], g["X"], g["A"], [s["B"] for s in m], [s["dY"] for s in m], g["Z"],
+                                    g["H"], g["dX"], g["dA"], [s["dB"] for s in m], self.ws)
 
     def step(self):
         self.forward()
@@ -227,9 +227,10 @@ def summarize_trace(records, peaks, ridge):
                       "tflops": round(v["flops"] / (v["ms"] / 1e3) / 1e12, 1)} for k, v in kinds.items()}
 
 
-def traffic_from_profile(kernel_key, workload):
+def traffic_from_profile(kernel_key, workload, algorithmic_bytes):
     """dram bytes per launch from a committed ncu summary, valid only while the
-    kernel sources are unchanged (hash match); else None."""
+    kernel sources are unchanged (hash match) and the launches it averaged
+    carry the same algorithmic bytes as the ones timed now; else None."""
     import hashlib
 
     path = os.path.join(ROOT, "profiles", "ncu_traffic.json")
@@ -243,7 +244,8 @@ def traffic_from_profile(kernel_key, workload):
             with open(os.path.join(ROOT, "paper_2502_10940_gb300", "csrc", name), "rb") as g:
                 h.update(g.read())
         entry = rec.get(workload, {}).get(kernel_key)
-        if entry and entry.get("src_sha256") == h.hexdigest():
+        if (entry and entry.get("src_sha256") == h.hexdigest()
+                and entry.get("algorithmic_bytes_per_launch") == algorithmic_bytes):
             return entry["dram_bytes_per_launch"]
     except Exception:  # noqa: BLE001 -- a missing or stale summary means "no traffic figure"
         return None
@@ -452,7 +454,8 @@ def time_steps(fn, steps, stream, dist=None):
 
 def full_rank_baseline(wl, device, steps, warmup, seed=0):
     """Same-shape full-rank layers (fwd Y = X W^T, bwd dX = dY W, dW = dY^T X)
-    with torch.matmul (cuBLAS), q/k/v fused as one N = 3d GEMM."""
+    with torch.matmul (cuBLAS); layers reading one input (q/k/v, gate/up) are
+    fused into one GEMM with their output widths concatenated."""
     import torch
 
     n = wl.n
@@ -460,7 +463,7 @@ def full_rank_baseline(wl, device, steps, warmup, seed=0):
     g = torch.Generator(device=device).manual_seed(seed + 77)
     groups = {}
     for L in wl.layers:
-        key = "qkv" if (wl.fused_qkv and L.name in ("q", "k", "v")) else L.name
+        key = L.x if wl.fused_qkv else L.name
         groups.setdefault(key, []).append(L)
     bufs = []
     flops = 0.0
@@ -535,7 +538,8 @@ def run_cola(args, wl):
         time_steps(blk.step, args.steps, stream)
     records = tr.records()
     roofline, kinds = summarize_trace(records, peaks, ridge)
-    roofline["traffic"] = traffic_from_profile(roofline["kernel"], wl.name)
+    roofline["traffic"] = traffic_from_profile(roofline["kernel"], wl.name,
+                                               roofline["algorithmic_bytes_per_launch"])
 
     flops = wl.flops
     value = flops * world / (ms / 1e3) / 1e12
@@ -544,7 +548,7 @@ def run_cola(args, wl):
             "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
             "config": {"workload": wl.desc, "n_tokens": wl.n, "mode": mode, "sigma": "silu",
                        "layers": [f"{L.name}:{L.d_in}->{L.d_out},r={L.r}" for L in wl.layers],
-                       "fused_qkv": blk.qkv, "parallelism": "replicas" if world > 1 else "single-gpu",
+                       "shared_x_groups": ["+".join(m["L"].name for m in g["members"]) for g in blk.groups], "parallelism": "replicas" if world > 1 else "single-gpu",
                        "l2": f"no flush: working set {blk.working_set_bytes() / 1e9:.2f} GB > 129 MB L2"},
             "tokens_per_s": round(wl.n * world / (ms / 1e3), 1),
             "pct_dense_bf16_peak": round(100.0 * value / world / peaks["bf16_tflops"], 2),

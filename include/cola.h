@@ -97,11 +97,13 @@ typedef struct {
     int32_t reserved;   /* must be 0 */
 } cola_desc_t;
 
-/* Bytes of workspace that cola_fwd / cola_bwd (fused_qkv = 0) or the fused
- * q/k/v entry points (fused_qkv = 1) need for `desc` on the current device.
- * The value depends on n, r, d_in, d_out, the mode and the device's SM count
- * (it sizes the weight-gradient split over tokens). */
-cola_status_t cola_workspace_size(const cola_desc_t* desc, int fused_qkv, size_t* bytes);
+/* Bytes of workspace the calls on `nproj` projections of shape `desc` that
+ * share one input need on the current device: nproj = 1 for cola_fwd /
+ * cola_bwd, 2 or 3 for cola_fwd_shared_x / cola_bwd_shared_x with that count
+ * (3 for the q/k/v entry points).  The value depends on n, r, d_in, d_out,
+ * the mode, wgrad_fp32 and the device's SM count (it sizes the
+ * weight-gradient split over tokens). */
+cola_status_t cola_workspace_size(const cola_desc_t* desc, int32_t nproj, size_t* bytes);
 
 /* Zero the workspace status word (first 256 bytes of ws), asynchronously. */
 cola_status_t cola_workspace_init(void* ws, void* stream);
@@ -129,7 +131,29 @@ cola_status_t cola_bwd(const cola_desc_t* desc, const void* X, const void* A, co
                        const void* Z_save, const void* H_save, void* dX, void* dA, void* dB, void* ws,
                        size_t ws_bytes, void* stream);
 
-/* Fused q/k/v forward (Fig. 4: the q, k and v auto-encoders read the same x).
+/* Projections that read the same input (Fig. 4: q, k and v read the
+ * attention input; gate and up read the MLP input): `count` = 2 or 3 CoLA
+ * layers of one shape (desc: d_in, d_out, r per projection) on one X.
+ *   A_cat [count r x d_in] (ld_a): the A_j stacked by rows.  One GEMM with
+ *     N = count r reads X once and writes Z_cat [n x count r] = [Z_1 .. Z_c]
+ *     and, under COLA, H_cat [n x count r] (NULL under COLA_M).
+ *   B[j] [d_out x r], Y[j] [n x d_out] (ld_y): host arrays of `count` device
+ *     pointers; the count output GEMMs Y_j = H_j B_j^T run as one launch. */
+cola_status_t cola_fwd_shared_x(const cola_desc_t* desc, int32_t count, const void* X, const void* A_cat,
+                                const void* const* B, void* const* Y, void* Z_cat, void* H_cat, void* ws,
+                                size_t ws_bytes, void* stream);
+
+/* Backward of cola_fwd_shared_x: dZ_j = (dY_j B_j) * sigma'(Z_j) for all j in
+ * one launch; dB_j = dY_j^T H_j and dA_cat = dZ_cat^T X (M = count r) in one
+ * launch; dX = dZ_cat A_cat (K = count r), i.e. the sum of the count input
+ * gradients, as one GEMM.  dY[j], dB[j]: host arrays of device pointers;
+ * dA_cat [count r x d_in] (ld_a); H_cat NULL under COLA_M. */
+cola_status_t cola_bwd_shared_x(const cola_desc_t* desc, int32_t count, const void* X, const void* A_cat,
+                                const void* const* B, const void* const* dY, const void* Z_cat, const void* H_cat,
+                                void* dX, void* dA_cat, void* const* dB, void* ws, size_t ws_bytes, void* stream);
+
+/* Fused q/k/v forward (Fig. 4: the q, k and v auto-encoders read the same x);
+ * cola_fwd_shared_x with count = 3.
  * desc->d_out is the width of each projection; desc->r the rank of each.
  *   A_qkv [3r x d_in] (ld_a) = [A_q; A_k; A_v] stacked by rows: one GEMM with
  *   N = 3r reads X once and writes Z_qkv [n x 3r] = [Z_q Z_k Z_v] and (COLA)
@@ -139,7 +163,8 @@ cola_status_t cola_fwd_qkv_fused(const cola_desc_t* desc, const void* X, const v
                                  const void* B_k, const void* B_v, void* Y_q, void* Y_k, void* Y_v,
                                  void* Z_qkv, void* H_qkv, void* ws, size_t ws_bytes, void* stream);
 
-/* Fused q/k/v backward: three dZ_j = (dY_j B_j) * sigma'(Z_j) into one
+/* Fused q/k/v backward (cola_bwd_shared_x with count = 3): three
+ * dZ_j = (dY_j B_j) * sigma'(Z_j) into one
  * [n x 3r] buffer, then one GEMM with M = 3r gives dA_qkv [3r x d_in] (ld_a),
  * one GEMM with K = 3r gives dX = sum_j dZ_j A_j (ld_x), and dB_j = dY_j^T H_j.
  * H_qkv must be NULL under COLA_M. */

@@ -22,9 +22,9 @@ STATUS = {0: "COLA_OK", 1: "COLA_ERR_INVALID", 2: "COLA_ERR_ALIGN", 3: "COLA_ERR
           4: "COLA_ERR_WORKSPACE", 5: "COLA_ERR_LAUNCH", 6: "COLA_ERR_DEVICE_TIMEOUT"}
 
 # the entry points include/cola.h declares
-SYMBOLS = ("cola_workspace_size", "cola_workspace_init", "cola_fwd", "cola_bwd", "cola_fwd_qkv_fused",
-           "cola_bwd_qkv_fused", "cola_check_status", "cola_wgrad_static_scratch", "cola_trace_attach",
-           "cola_trace_detach", "cola_status_string")
+SYMBOLS = ("cola_workspace_size", "cola_workspace_init", "cola_fwd", "cola_bwd", "cola_fwd_shared_x",
+           "cola_bwd_shared_x", "cola_fwd_qkv_fused", "cola_bwd_qkv_fused", "cola_check_status",
+           "cola_wgrad_static_scratch", "cola_trace_attach", "cola_trace_detach", "cola_status_string")
 STATIC_SCRATCH_BYTES = 64 * 1024 * 1024
 KERNELS = {0: "fwd_zh", 1: "fwd_y", 2: "bwd_dz", 3: "wgrad", 4: "reduce", 5: "bwd_dx"}
 
@@ -61,7 +61,7 @@ def lib():
         l = ctypes.CDLL(LIB_PATH)
         D = ctypes.POINTER(cola_desc_t)
         st = ctypes.c_int
-        l.cola_workspace_size.argtypes = [D, ctypes.c_int, ctypes.POINTER(ctypes.c_size_t)]
+        l.cola_workspace_size.argtypes = [D, ctypes.c_int32, ctypes.POINTER(ctypes.c_size_t)]
         l.cola_workspace_size.restype = st
         l.cola_workspace_init.argtypes = [_vp, _vp]
         l.cola_workspace_init.restype = st
@@ -69,6 +69,12 @@ def lib():
         l.cola_fwd.restype = st
         l.cola_bwd.argtypes = [D] + [_vp] * 10 + [ctypes.c_size_t, _vp]
         l.cola_bwd.restype = st
+        PP = ctypes.POINTER(ctypes.c_void_p)
+        l.cola_fwd_shared_x.argtypes = [D, ctypes.c_int32, _vp, _vp, PP, PP, _vp, _vp, _vp, ctypes.c_size_t, _vp]
+        l.cola_fwd_shared_x.restype = st
+        l.cola_bwd_shared_x.argtypes = [D, ctypes.c_int32, _vp, _vp, PP, PP, _vp, _vp, _vp, _vp, PP, _vp,
+                                        ctypes.c_size_t, _vp]
+        l.cola_bwd_shared_x.restype = st
         l.cola_fwd_qkv_fused.argtypes = [D] + [_vp] * 11 + [ctypes.c_size_t, _vp]
         l.cola_fwd_qkv_fused.restype = st
         l.cola_bwd_qkv_fused.argtypes = [D] + [_vp] * 16 + [ctypes.c_size_t, _vp]
@@ -132,9 +138,11 @@ def _nbytes(ws):
     return ws.numel() * ws.element_size()
 
 
-def cola_workspace_size(d: cola_desc_t, fused_qkv: int = 0) -> int:
+def cola_workspace_size(d: cola_desc_t, nproj: int = 1) -> int:
+    """Workspace bytes for calls on `nproj` projections sharing one input
+    (1: cola_fwd / cola_bwd; 2, 3: the shared-input entry points)."""
     out = ctypes.c_size_t(0)
-    _check(lib().cola_workspace_size(ctypes.byref(d), int(fused_qkv), ctypes.byref(out)), "cola_workspace_size")
+    _check(lib().cola_workspace_size(ctypes.byref(d), int(nproj), ctypes.byref(out)), "cola_workspace_size")
     return int(out.value)
 
 
@@ -150,6 +158,25 @@ def cola_fwd(d, X, A, B, Y, Z_save, H_save, ws, stream=None):
 def cola_bwd(d, X, A, B, dY, Z_save, H_save, dX, dA, dB, ws, stream=None):
     _check(lib().cola_bwd(ctypes.byref(d), _ptr(X), _ptr(A), _ptr(B), _ptr(dY), _ptr(Z_save), _ptr(H_save),
                           _ptr(dX), _ptr(dA), _ptr(dB), _ptr(ws), _nbytes(ws), _stream(stream)), "cola_bwd")
+
+
+def _ptr_array(ts):
+    arr = (ctypes.c_void_p * len(ts))()
+    for i, t in enumerate(ts):
+        arr[i] = _ptr(t)
+    return arr
+
+
+def cola_fwd_shared_x(d, X, A_cat, Bs, Ys, Z_cat, H_cat, ws, stream=None):
+    _check(lib().cola_fwd_shared_x(ctypes.byref(d), len(Bs), _ptr(X), _ptr(A_cat), _ptr_array(Bs), _ptr_array(Ys),
+                                   _ptr(Z_cat), _ptr(H_cat), _ptr(ws), _nbytes(ws), _stream(stream)),
+           "cola_fwd_shared_x")
+
+
+def cola_bwd_shared_x(d, X, A_cat, Bs, dYs, Z_cat, H_cat, dX, dA_cat, dBs, ws, stream=None):
+    _check(lib().cola_bwd_shared_x(ctypes.byref(d), len(Bs), _ptr(X), _ptr(A_cat), _ptr_array(Bs), _ptr_array(dYs),
+                                   _ptr(Z_cat), _ptr(H_cat), _ptr(dX), _ptr(dA_cat), _ptr_array(dBs), _ptr(ws),
+                                   _nbytes(ws), _stream(stream)), "cola_bwd_shared_x")
 
 
 def cola_fwd_qkv_fused(d, X, A_qkv, B_q, B_k, B_v, Y_q, Y_k, Y_v, Z_qkv, H_qkv, ws, stream=None):
@@ -239,9 +266,9 @@ def ld_of(t) -> int:
     return int(t.stride(0))
 
 
-def workspace(d: cola_desc_t, fused_qkv: int = 0, device="cuda"):
+def workspace(d: cola_desc_t, nproj: int = 1, device="cuda"):
     """A zero-initialised workspace tensor for `d` (allocated by torch)."""
-    nbytes = cola_workspace_size(d, fused_qkv)
+    nbytes = cola_workspace_size(d, nproj)
     ws = torch.empty(nbytes + 256, dtype=torch.uint8, device=device)
     off = (-ws.data_ptr()) % 256
     ws = ws[off:off + nbytes]

@@ -99,11 +99,11 @@ struct WsLayout {
 
 // The weight-gradient group of one backward call: dB (per projection) and dA,
 // all reduced over the same n tokens in one launch.
-WgradPlan wgrad_plan(const cola_desc_t& d, int fused, int sms)
+WgradPlan wgrad_plan(const cola_desc_t& d, int nproj, int sms)
 {
-    const int64_t R = fused ? 3 * d.r : d.r;
+    const int64_t R = nproj * d.r;
     int64_t M[MAX_GROUP], N[MAX_GROUP];
-    const int nb = fused ? 3 : 1;
+    const int nb = nproj;
     for (int j = 0; j < nb; ++j) {
         M[j] = d.d_out;
         N[j] = d.r;
@@ -115,9 +115,9 @@ WgradPlan wgrad_plan(const cola_desc_t& d, int fused, int sms)
 
 // dZ [n x R] bf16, H [n x R] bf16 (CoLA-M only), the fp32 split partials of
 // the weight-gradient group.
-WsLayout ws_layout(const cola_desc_t& d, int fused, int sms)
+WsLayout ws_layout(const cola_desc_t& d, int nproj, int sms)
 {
-    const int64_t R = fused ? 3 * d.r : d.r;
+    const int64_t R = nproj * d.r;
     WsLayout L;
     size_t off = WS_HEADER;
     L.dz_off = off;
@@ -125,17 +125,17 @@ WsLayout ws_layout(const cola_desc_t& d, int fused, int sms)
     L.h_off = off;
     if (d.mode == COLA_MODE_COLA_M) off += align_up(static_cast<size_t>(d.n) * R * 2);
     L.part_off = off;
-    const WgradPlan w = wgrad_plan(d, fused, sms);
+    const WgradPlan w = wgrad_plan(d, nproj, sms);
     if (w.splits > 1 || d.wgrad_fp32) off += align_up(static_cast<size_t>(w.part_elems) * 4);
     L.total = off;
     return L;
 }
 
-cola_status_t check_ws(const cola_desc_t& d, int fused, int sms, void* ws, size_t ws_bytes, WsLayout* L)
+cola_status_t check_ws(const cola_desc_t& d, int nproj, int sms, void* ws, size_t ws_bytes, WsLayout* L)
 {
     if (!ws) return COLA_ERR_INVALID;
     if (reinterpret_cast<uintptr_t>(ws) & (WS_ALIGN - 1)) return COLA_ERR_ALIGN;
-    *L = ws_layout(d, fused, sms);
+    *L = ws_layout(d, nproj, sms);
     if (ws_bytes < L->total) return COLA_ERR_WORKSPACE;
     return COLA_OK;
 }
@@ -377,14 +377,14 @@ using namespace cola;
 
 extern "C" {
 
-cola_status_t cola_workspace_size(const cola_desc_t* desc, int fused_qkv, size_t* bytes)
+cola_status_t cola_workspace_size(const cola_desc_t* desc, int32_t nproj, size_t* bytes)
 {
     Shape s;
     COLA_TRY(check_desc(desc, &s));
-    if (!bytes || (fused_qkv != 0 && fused_qkv != 1)) return COLA_ERR_INVALID;
+    if (!bytes || nproj < 1 || nproj > 3) return COLA_ERR_INVALID;
     int sms = 0;
     COLA_TRY(device_info(&sms));
-    *bytes = ws_layout(*desc, fused_qkv, sms).total;
+    *bytes = ws_layout(*desc, nproj, sms).total;
     return COLA_OK;
 }
 
@@ -407,7 +407,7 @@ cola_status_t cola_fwd(const cola_desc_t* desc, const void* X, const void* A, co
     int sms = 0;
     COLA_TRY(device_info(&sms));
     WsLayout L;
-    COLA_TRY(check_ws(*desc, 0, sms, ws, ws_bytes, &L));
+    COLA_TRY(check_ws(*desc, 1, sms, ws, ws_bytes, &L));
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     unsigned int* status = ws_status(ws);
     void* H = cola_m ? static_cast<void*>(wsb(ws) + L.h_off) : H_save;
@@ -431,7 +431,7 @@ cola_status_t cola_bwd(const cola_desc_t* desc, const void* X, const void* A, co
     int sms = 0;
     COLA_TRY(device_info(&sms));
     WsLayout L;
-    COLA_TRY(check_ws(*desc, 0, sms, ws, ws_bytes, &L));
+    COLA_TRY(check_ws(*desc, 1, sms, ws, ws_bytes, &L));
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     unsigned int* status = ws_status(ws);
     void* dZ = wsb(ws) + L.dz_off;
@@ -446,36 +446,89 @@ cola_status_t cola_bwd(const cola_desc_t* desc, const void* X, const void* A, co
     void* Hs[1] = {Hrec};
     COLA_TRY(run_b1(s, desc->sigma, 1, dYs, Bs, Zs, s.r, dZs, cola_m ? Hs : nullptr, status, sms, st));
     const void* Hsrc = cola_m ? Hrec : H_save;
-    const WgradPlan w = wgrad_plan(*desc, 0, sms);
+    const WgradPlan w = wgrad_plan(*desc, 1, sms);
     const WgradJob jobs[2] = {{dY, s.ld_y, Hsrc, s.r, dB, s.r}, {dZ, s.r, X, s.ld_x, dA, s.ld_a}};
     COLA_TRY(run_wgrad(w, s.n, jobs, desc->wgrad_fp32, part, part_bytes, status, sms, st));
     return run_b4(s, s.r, dZ, s.r, A, dX, status, sms, st);
+}
+
+cola_status_t cola_fwd_shared_x(const cola_desc_t* desc, int32_t count, const void* X, const void* A_cat,
+                                const void* const* B, void* const* Y, void* Z_cat, void* H_cat, void* ws,
+                                size_t ws_bytes, void* stream)
+{
+    Shape s;
+    COLA_TRY(check_desc(desc, &s));
+    if (count < 2 || count > 3 || !B || !Y) return COLA_ERR_INVALID;
+    COLA_TRY(check_ptrs({X, A_cat, Z_cat}));
+    for (int j = 0; j < count; ++j) COLA_TRY(check_ptrs({B[j], Y[j]}));
+    const bool cola_m = desc->mode == COLA_MODE_COLA_M;
+    if (cola_m ? H_cat != nullptr : H_cat == nullptr) return COLA_ERR_INVALID;
+    if (H_cat && !aligned16(H_cat)) return COLA_ERR_ALIGN;
+    int sms = 0;
+    COLA_TRY(device_info(&sms));
+    WsLayout L;
+    COLA_TRY(check_ws(*desc, count, sms, ws, ws_bytes, &L));
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    unsigned int* status = ws_status(ws);
+    const int64_t R = count * s.r;
+    const size_t slice = static_cast<size_t>(s.r) * 2;   // bytes between the projections' column blocks
+    uint8_t* H = cola_m ? wsb(ws) + L.h_off : static_cast<uint8_t*>(H_cat);
+    COLA_TRY(run_f1(s, desc->sigma, R, X, A_cat, Z_cat, H, R, status, sms, st));
+    const void* Hs[3] = {H, H + slice, H + 2 * slice};
+    return run_f2(s, count, Hs, R, B, Y, status, sms, st);
+}
+
+cola_status_t cola_bwd_shared_x(const cola_desc_t* desc, int32_t count, const void* X, const void* A_cat,
+                                const void* const* B, const void* const* dY, const void* Z_cat, const void* H_cat,
+                                void* dX, void* dA_cat, void* const* dB, void* ws, size_t ws_bytes, void* stream)
+{
+    Shape s;
+    COLA_TRY(check_desc(desc, &s));
+    if (count < 2 || count > 3 || !B || !dY || !dB) return COLA_ERR_INVALID;
+    COLA_TRY(check_ptrs({X, A_cat, Z_cat, dX, dA_cat}));
+    for (int j = 0; j < count; ++j) COLA_TRY(check_ptrs({B[j], dY[j], dB[j]}));
+    const bool cola_m = desc->mode == COLA_MODE_COLA_M;
+    if (cola_m ? H_cat != nullptr : H_cat == nullptr) return COLA_ERR_INVALID;
+    if (H_cat && !aligned16(H_cat)) return COLA_ERR_ALIGN;
+    int sms = 0;
+    COLA_TRY(device_info(&sms));
+    WsLayout L;
+    COLA_TRY(check_ws(*desc, count, sms, ws, ws_bytes, &L));
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    unsigned int* status = ws_status(ws);
+    const int64_t R = count * s.r;
+    const size_t slice = static_cast<size_t>(s.r) * 2;   // bytes between the projections' column blocks
+    uint8_t* dZ = wsb(ws) + L.dz_off;
+    uint8_t* Hrec = cola_m ? wsb(ws) + L.h_off : nullptr;
+    float* part = reinterpret_cast<float*>(wsb(ws) + L.part_off);
+    const size_t part_bytes = L.total - L.part_off;
+    const uint8_t* Zb = static_cast<const uint8_t*>(Z_cat);
+    const uint8_t* Hsrc = cola_m ? Hrec : static_cast<const uint8_t*>(H_cat);
+
+    const void* Zs[3];
+    void* dZs[3];
+    void* Hr[3];
+    WgradJob jobs[MAX_GROUP];
+    for (int j = 0; j < count; ++j) {
+        Zs[j] = Zb + j * slice;
+        dZs[j] = dZ + j * slice;
+        Hr[j] = Hrec ? Hrec + j * slice : nullptr;
+        jobs[j] = {dY[j], s.ld_y, Hsrc + j * slice, R, dB[j], s.r};
+    }
+    jobs[count] = {dZ, R, X, s.ld_x, dA_cat, s.ld_a};
+    COLA_TRY(run_b1(s, desc->sigma, count, dY, B, Zs, R, dZs, cola_m ? Hr : nullptr, status, sms, st));
+    const WgradPlan w = wgrad_plan(*desc, count, sms);
+    COLA_TRY(run_wgrad(w, s.n, jobs, desc->wgrad_fp32, part, part_bytes, status, sms, st));
+    return run_b4(s, R, dZ, R, A_cat, dX, status, sms, st);
 }
 
 cola_status_t cola_fwd_qkv_fused(const cola_desc_t* desc, const void* X, const void* A_qkv, const void* B_q,
                                  const void* B_k, const void* B_v, void* Y_q, void* Y_k, void* Y_v, void* Z_qkv,
                                  void* H_qkv, void* ws, size_t ws_bytes, void* stream)
 {
-    Shape s;
-    COLA_TRY(check_desc(desc, &s));
-    COLA_TRY(check_ptrs({X, A_qkv, B_q, B_k, B_v, Y_q, Y_k, Y_v, Z_qkv}));
-    const bool cola_m = desc->mode == COLA_MODE_COLA_M;
-    if (cola_m ? H_qkv != nullptr : H_qkv == nullptr) return COLA_ERR_INVALID;
-    if (H_qkv && !aligned16(H_qkv)) return COLA_ERR_ALIGN;
-    int sms = 0;
-    COLA_TRY(device_info(&sms));
-    WsLayout L;
-    COLA_TRY(check_ws(*desc, 1, sms, ws, ws_bytes, &L));
-    cudaStream_t st = static_cast<cudaStream_t>(stream);
-    unsigned int* status = ws_status(ws);
-    const int64_t R = 3 * s.r;
-    const size_t slice = static_cast<size_t>(s.r) * 2;   // bytes between the q, k, v column blocks
-    uint8_t* H = cola_m ? wsb(ws) + L.h_off : static_cast<uint8_t*>(H_qkv);
-    COLA_TRY(run_f1(s, desc->sigma, R, X, A_qkv, Z_qkv, H, R, status, sms, st));
-    const void* Hs[3] = {H, H + slice, H + 2 * slice};
-    const void* Bs[3] = {B_q, B_k, B_v};
-    void* Ys[3] = {Y_q, Y_k, Y_v};
-    return run_f2(s, 3, Hs, R, Bs, Ys, status, sms, st);
+    const void* B[3] = {B_q, B_k, B_v};
+    void* Y[3] = {Y_q, Y_k, Y_v};
+    return cola_fwd_shared_x(desc, 3, X, A_qkv, B, Y, Z_qkv, H_qkv, ws, ws_bytes, stream);
 }
 
 cola_status_t cola_bwd_qkv_fused(const cola_desc_t* desc, const void* X, const void* A_qkv, const void* B_q,
@@ -483,40 +536,10 @@ cola_status_t cola_bwd_qkv_fused(const cola_desc_t* desc, const void* X, const v
                                  const void* dY_v, const void* Z_qkv, const void* H_qkv, void* dX, void* dA_qkv,
                                  void* dB_q, void* dB_k, void* dB_v, void* ws, size_t ws_bytes, void* stream)
 {
-    Shape s;
-    COLA_TRY(check_desc(desc, &s));
-    COLA_TRY(check_ptrs({X, A_qkv, B_q, B_k, B_v, dY_q, dY_k, dY_v, Z_qkv, dX, dA_qkv, dB_q, dB_k, dB_v}));
-    const bool cola_m = desc->mode == COLA_MODE_COLA_M;
-    if (cola_m ? H_qkv != nullptr : H_qkv == nullptr) return COLA_ERR_INVALID;
-    if (H_qkv && !aligned16(H_qkv)) return COLA_ERR_ALIGN;
-    int sms = 0;
-    COLA_TRY(device_info(&sms));
-    WsLayout L;
-    COLA_TRY(check_ws(*desc, 1, sms, ws, ws_bytes, &L));
-    cudaStream_t st = static_cast<cudaStream_t>(stream);
-    unsigned int* status = ws_status(ws);
-    const int64_t R = 3 * s.r;
-    const size_t slice = static_cast<size_t>(s.r) * 2;   // bytes between the q, k, v column blocks
-    uint8_t* dZ = wsb(ws) + L.dz_off;
-    uint8_t* Hrec = cola_m ? wsb(ws) + L.h_off : nullptr;
-    float* part = reinterpret_cast<float*>(wsb(ws) + L.part_off);
-    const size_t part_bytes = L.total - L.part_off;
-    const uint8_t* Zb = static_cast<const uint8_t*>(Z_qkv);
-    const uint8_t* Hsrc = cola_m ? Hrec : static_cast<const uint8_t*>(H_qkv);
-
-    const void* dYs[3] = {dY_q, dY_k, dY_v};
-    const void* Bs[3] = {B_q, B_k, B_v};
-    const void* Zs[3] = {Zb, Zb + slice, Zb + 2 * slice};
-    void* dZs[3] = {dZ, dZ + slice, dZ + 2 * slice};
-    void* Hr[3] = {Hrec, Hrec + slice, Hrec + 2 * slice};
-    COLA_TRY(run_b1(s, desc->sigma, 3, dYs, Bs, Zs, R, dZs, cola_m ? Hr : nullptr, status, sms, st));
-    const WgradPlan w = wgrad_plan(*desc, 1, sms);
-    const WgradJob jobs[4] = {{dY_q, s.ld_y, Hsrc, R, dB_q, s.r},
-                              {dY_k, s.ld_y, Hsrc + slice, R, dB_k, s.r},
-                              {dY_v, s.ld_y, Hsrc + 2 * slice, R, dB_v, s.r},
-                              {dZ, R, X, s.ld_x, dA_qkv, s.ld_a}};
-    COLA_TRY(run_wgrad(w, s.n, jobs, desc->wgrad_fp32, part, part_bytes, status, sms, st));
-    return run_b4(s, R, dZ, R, A_qkv, dX, status, sms, st);
+    const void* B[3] = {B_q, B_k, B_v};
+    const void* dY[3] = {dY_q, dY_k, dY_v};
+    void* dB[3] = {dB_q, dB_k, dB_v};
+    return cola_bwd_shared_x(desc, 3, X, A_qkv, B, dY, Z_qkv, H_qkv, dX, dA_qkv, dB, ws, ws_bytes, stream);
 }
 
 cola_status_t cola_check_status(void* ws, void* stream, uint32_t* code_out)

@@ -50,9 +50,9 @@ def test_desc_layout_matches_header(L):
     assert ctypes.sizeof(L.cola_desc_t) == 7 * 8 + 4 * 4
 
 
-def _ws_size(L, d, fused=0):
+def _ws_size(L, d, nproj=1):
     out = ctypes.c_size_t(0)
-    return L.lib().cola_workspace_size(ctypes.byref(d), fused, ctypes.byref(out))
+    return L.lib().cola_workspace_size(ctypes.byref(d), nproj, ctypes.byref(out))
 
 
 @pytest.mark.parametrize("kw,code", [
@@ -73,12 +73,13 @@ def test_workspace_size_rejects_bad_desc(L, kw, code):
     assert _ws_size(L, d) == code
 
 
-def test_workspace_size_rejects_null_out_and_bad_flag(L):
+def test_workspace_size_rejects_null_out_and_bad_nproj(L):
     d = L.desc(256, 128, 128, 64)
-    assert L.lib().cola_workspace_size(ctypes.byref(d), 0, None) == 1
+    assert L.lib().cola_workspace_size(ctypes.byref(d), 1, None) == 1
     out = ctypes.c_size_t(0)
-    assert L.lib().cola_workspace_size(ctypes.byref(d), 2, ctypes.byref(out)) == 1
-    assert L.lib().cola_workspace_size(None, 0, ctypes.byref(out)) == 1
+    assert L.lib().cola_workspace_size(ctypes.byref(d), 0, ctypes.byref(out)) == 1
+    assert L.lib().cola_workspace_size(ctypes.byref(d), 4, ctypes.byref(out)) == 1
+    assert L.lib().cola_workspace_size(None, 1, ctypes.byref(out)) == 1
 
 
 FAKE = 0x100000  # 16-byte aligned, never dereferenced
@@ -128,6 +129,23 @@ def test_qkv_argument_errors(L):
     args = [FAKE] * 16
     args[13] = FAKE + 4  # misaligned dB_k
     assert g(ctypes.byref(d), *args, 1 << 20, None) == 2
+
+
+def test_shared_x_argument_errors(L):
+    d = L.desc(256, 128, 128, 64, mode="cola")
+    f = L.lib().cola_fwd_shared_x
+    ok2 = (ctypes.c_void_p * 2)(FAKE, FAKE)
+    bad = (ctypes.c_void_p * 2)(FAKE, FAKE + 4)
+    nul = (ctypes.c_void_p * 2)(FAKE, None)
+    assert f(ctypes.byref(d), 1, FAKE, FAKE, ok2, ok2, FAKE, FAKE, FAKE, 1 << 20, None) == 1   # count < 2
+    assert f(ctypes.byref(d), 4, FAKE, FAKE, ok2, ok2, FAKE, FAKE, FAKE, 1 << 20, None) == 1   # count > 3
+    assert f(ctypes.byref(d), 2, FAKE, FAKE, nul, ok2, FAKE, FAKE, FAKE, 1 << 20, None) == 1   # null B[1]
+    assert f(ctypes.byref(d), 2, FAKE, FAKE, ok2, bad, FAKE, FAKE, FAKE, 1 << 20, None) == 2   # misaligned Y[1]
+    assert f(ctypes.byref(d), 2, FAKE, FAKE, None, ok2, FAKE, FAKE, FAKE, 1 << 20, None) == 1  # no B array
+    g = L.lib().cola_bwd_shared_x
+    dm = L.desc(256, 128, 128, 64, mode="cola_m")
+    assert g(ctypes.byref(dm), 2, FAKE, FAKE, ok2, ok2, FAKE, FAKE, FAKE, FAKE, ok2, FAKE, 1 << 20, None) == 1  # H under CoLA-M
+    assert g(ctypes.byref(dm), 2, FAKE, FAKE, ok2, ok2, FAKE, None, FAKE, FAKE, bad, FAKE, 1 << 20, None) == 2
 
 
 def test_workspace_init_and_check_reject_null(L):

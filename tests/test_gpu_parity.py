@@ -120,7 +120,7 @@ def test_qkv_fused_matches_oracle(shape, mode):
     dYs = [p["dY"] for p in parts]
     ldy = cola.ld_of(dYs[0])
     desc = cola.desc(n, d, d, r, ld_x=ldx, ld_y=ldy, ld_a=ldx, sigma="silu", mode=mode)
-    ws = cola.workspace(desc, fused_qkv=1)
+    ws = cola.workspace(desc, nproj=3)
     Ys = [padded_empty(n, d, ldy) for _ in range(3)]
     Z = torch.empty((n, 3 * r), dtype=torch.bfloat16, device="cuda")
     H = torch.empty((n, 3 * r), dtype=torch.bfloat16, device="cuda") if mode == "cola" else None
@@ -144,3 +144,45 @@ def test_qkv_fused_matches_oracle(shape, mode):
         assert_close(f"dB{j}", to64(dBs[j]), dBo[j])
         assert_close(f"dA{j}", to64(dA[j * r:(j + 1) * r]), dAo[j])
     assert_close("dX", to64(dX), dXo)
+
+
+@pytest.mark.parametrize("mode", ["cola", "cola_m"])
+@pytest.mark.parametrize("shape", [(300, 200, 328, 128), (2048, 512, 1376, 128)], ids=str)
+def test_shared_x_pair_matches_oracle(shape, mode):
+    # gate / up: two projections of one shape reading one X (Fig. 4); dX is
+    # the sum of both input gradients, dA_cat one GEMM with M = 2r
+    import oracle
+    from paper_2502_10940_gb300 import cola
+    n, d_in, d_out, r = shape
+    X = make_inputs(n, d_in, d_out, r, seed=30)["X"]
+    parts = [make_inputs(n, d_in, d_out, r, seed=31 + j) for j in range(2)]
+    ldx = cola.ld_of(X)
+    A_cat = padded_empty(2 * r, d_in, ldx)
+    A_cat.copy_(torch.cat([p["A"] for p in parts], 0))
+    Bs = [p["B"] for p in parts]
+    dYs = [p["dY"] for p in parts]
+    ldy = cola.ld_of(dYs[0])
+    desc = cola.desc(n, d_in, d_out, r, ld_x=ldx, ld_y=ldy, ld_a=ldx, sigma="silu", mode=mode)
+    ws = cola.workspace(desc, nproj=2)
+    Ys = [padded_empty(n, d_out, ldy) for _ in range(2)]
+    Z = torch.empty((n, 2 * r), dtype=torch.bfloat16, device="cuda")
+    H = torch.empty((n, 2 * r), dtype=torch.bfloat16, device="cuda") if mode == "cola" else None
+    cola.cola_fwd_shared_x(desc, X, A_cat, Bs, Ys, Z, H, ws)
+    dX = padded_empty(n, d_in, ldx)
+    dA = padded_empty(2 * r, d_in, ldx)
+    dBs = [torch.empty((d_out, r), dtype=torch.bfloat16, device="cuda") for _ in range(2)]
+    cola.cola_bwd_shared_x(desc, X, A_cat, Bs, dYs, Z, H, dX, dA, dBs, ws)
+    assert cola.cola_check_status(ws)[0] == 0
+
+    X64 = to64(X)
+    As = [to64(p["A"]) for p in parts]
+    Bo = [to64(b) for b in Bs]
+    Zs, Hs, Yo = oracle.fwd_qkv(X64, As, Bo, "silu")
+    dXo, dAo, dBo, _ = oracle.bwd_qkv(X64, As, Bo, [to64(t) for t in dYs], Zs, Hs, "silu", "cola")
+    for j in range(2):
+        assert_close(f"Y{j}", to64(Ys[j]), Yo[j])
+        assert_close(f"Z{j}", to64(Z[:, j * r:(j + 1) * r]), Zs[j])
+        assert_close(f"dB{j}", to64(dBs[j]), dBo[j])
+        assert_close(f"dA{j}", to64(dA[j * r:(j + 1) * r]), dAo[j])
+    assert_close("dX", to64(dX), dXo)
+    assert padding_intact(dX, d_in) and padding_intact(Ys[0], d_out)
