@@ -7,7 +7,7 @@ h = B sigma(A x) each, Sec. 3.2 / Fig. 4) followed by their backward
 (Sec. 3.4), every GEMM on the library's tcgen05 kernels through the C ABI.
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--workload 60m|350m|1b|7b|60m-q]
-                    [--mode cola|cola_m] [--impl cola|reference]
+                    [--mode cola|cola_m|infer] [--impl cola|reference] [--graph auto|on|off]
 
 Prints ONE JSON line (rank 0).  `value` is whole-job TFLOP/s (algorithmic
 6 n r (d_in + d_out) per layer), device-timed with CUDA events, inputs
@@ -35,6 +35,8 @@ if ROOT not in sys.path:
     sys.path.insert(0, ROOT)
 
 METRIC = "CoLA layer fwd+bwd TFLOP/s and % of GB300 dense-BF16 peak; tokens/s per block"
+METRIC_INFER = "CoLA block forward (inference) TFLOP/s and % of GB300 dense-BF16 peak; tokens/s"
+L2_BYTES = 129 << 20
 
 
 def _peaks():
@@ -73,15 +75,18 @@ class Block:
         for li, L in enumerate(wl.layers):
             groups.setdefault(L.x, []).append(li)
         self.layers = []
+        self.train = mode != "infer"
         for li, L in enumerate(wl.layers):
-            t = I.layer_inputs(n, L.d_in, L.d_out, L.r, seed=seed, device=device, layer=li, with_x=False)
+            t = I.layer_inputs(n, L.d_in, L.d_out, L.r, seed=seed, device=device, layer=li, with_x=False,
+                               with_dy=self.train)
             X = self.X[L.x]
-            st = dict(L=L, X=X, A=t["A"], B=t["B"], dY=t["dY"])
-            ldy = cola.ld_of(t["dY"])
+            st = dict(L=L, X=X, A=t["A"], B=t["B"], dY=t.get("dY"))
+            ldy = I.padded_ld(L.d_out)
             st["Y"] = torch.empty((n, ldy), dtype=bf, device=device)[:, :L.d_out]
             st["desc"] = cola.desc(n, L.d_in, L.d_out, L.r, ld_x=cola.ld_of(X), ld_y=ldy, ld_a=cola.ld_of(t["A"]),
                                    sigma=sigma, mode=mode)
-            st["dB"] = torch.empty((L.d_out, L.r), dtype=bf, device=device)
+            if self.train:
+                st["dB"] = torch.empty((L.d_out, L.r), dtype=bf, device=device)
             self.layers.append(st)
         self.groups = []
         self.ws_bytes = 0
@@ -101,21 +106,26 @@ class Block:
                     g["A"] = torch.empty((c * L.r, ldx), dtype=bf, device=device)[:, :L.d_in]
                     for j, m in enumerate(part):
                         g["A"][j * L.r:(j + 1) * L.r].copy_(m["A"])
-                g["Z"] = torch.empty((n, c * L.r), dtype=bf, device=device)
+                g["Z"] = torch.empty((n, c * L.r), dtype=bf, device=device) if self.train else None
                 g["H"] = torch.empty((n, c * L.r), dtype=bf, device=device) if mode == "cola" else None
-                g["dX"] = torch.empty((n, ldx), dtype=bf, device=device)[:, :L.d_in]
-                g["dA"] = torch.empty((c * L.r, ldx), dtype=bf, device=device)[:, :L.d_in]
+                if self.train:
+                    g["dX"] = torch.empty((n, ldx), dtype=bf, device=device)[:, :L.d_in]
+                    g["dA"] = torch.empty((c * L.r, ldx), dtype=bf, device=device)[:, :L.d_in]
                 self.ws_bytes = max(self.ws_bytes, cola.cola_workspace_size(g["desc"], c))
                 self.groups.append(g)
         self.ws = torch.empty(self.ws_bytes, dtype=torch.uint8, device=device)
         cola.cola_workspace_init(self.ws)
         self.launches_per_step = None
 
-    # inputs a step consumes from outside (activations + upstream gradients)
+    # inputs a step consumes from outside (activations, and upstream gradients
+    # when training)
     def step_inputs(self):
-        return list(self.X.values()) + [s["dY"] for s in self.layers]
+        return list(self.X.values()) + ([s["dY"] for s in self.layers] if self.train else [])
 
+    # what a step hands back: the weight gradients (training) or the outputs
     def step_results(self):
+        if not self.train:
+            return [s["Y"] for s in self.layers]
         return [g["dA"] for g in self.groups] + [s["dB"] for s in self.layers]
 
     def forward(self):
@@ -143,7 +153,8 @@ class Block:
 
     def step(self):
         self.forward()
-        self.backward()
+        if self.train:
+            self.backward()
 
     def check(self):
         st, code = self.cola.cola_check_status(self.ws)
@@ -360,23 +371,31 @@ def oracle_block_sample(wl, n_s, seed=0):
     tokens of the same synthetic distribution.  Returns (seconds, flops)."""
     import oracle
     from paper_2502_10940_gb300 import inputs as I
-    from paper_2502_10940_gb300.workloads import layer_flops
+    from paper_2502_10940_gb300.workloads import fwd_flops, layer_flops
 
+    train = wl.phase != "infer"
     xs = {}
     for L in wl.layers:
         if L.x not in xs:
             xs[L.x] = I.activation(n_s, L.d_in, seed, "cpu", layer=100 + len(xs)).float().double().numpy()
     prepared = []
     for li, L in enumerate(wl.layers):
-        t = I.layer_inputs(n_s, L.d_in, L.d_out, L.r, seed=seed, device="cpu", layer=li, with_x=False)
+        t = I.layer_inputs(n_s, L.d_in, L.d_out, L.r, seed=seed, device="cpu", layer=li, with_x=False,
+                           with_dy=train)
         prepared.append((xs[L.x], t["A"].float().double().numpy(), t["B"].float().double().numpy(),
-                         t["dY"].float().double().numpy()))
+                         t["dY"].float().double().numpy() if train else None))
     t0 = time.perf_counter()
     for X, A, B, dY in prepared:
         Z, H, Y = oracle.fwd(X, A, B, "silu")
-        oracle.bwd(X, A, B, dY, Z, H, "silu", "cola")
+        if train:
+            oracle.bwd(X, A, B, dY, Z, H, "silu", "cola")
     dt = time.perf_counter() - t0
-    return dt, float(sum(layer_flops(n_s, L.d_in, L.d_out, L.r) for L in wl.layers))
+    f = layer_flops if train else fwd_flops
+    return dt, float(sum(f(n_s, L.d_in, L.d_out, L.r) for L in wl.layers))
+
+
+def phase_words(wl):
+    return "fwd+bwd" if wl.phase != "infer" else "fwd only"
 
 
 def calibrate_tokens(wl, target_s):
@@ -395,7 +414,7 @@ def cpu_baseline(wl, target_s=10.0):
     n_s = calibrate_tokens(wl, target_s)
     dt, fl = oracle_block_sample(wl, n_s)
     return {"value": round(fl / dt / 1e12, 6), "unit": "TFLOP/s", "cores": oracle.num_threads(), "kind": "oracle",
-            "sample": f"{wl.name} block, all {len(wl.layers)} layers fwd+bwd on {n_s} of {wl.n} tokens "
+            "sample": f"{wl.name} block, all {len(wl.layers)} layers {phase_words(wl)} on {n_s} of {wl.n} tokens "
                       f"({dt:.1f} s, fp64 loops, OpenMP)"}
 
 
@@ -417,11 +436,12 @@ def run_reference(args, wl):
         tot_t += dt
         tot_f += fl
     value = tot_f / tot_t / 1e12
-    sample = f"{wl.name} block, all {len(wl.layers)} layers fwd+bwd on {n_s} of {wl.n} tokens per step"
-    line = {"impl": "reference", "metric": METRIC, "value": round(value, 6), "unit": "TFLOP/s", "n_gpus": args.gpus,
+    sample = f"{wl.name} block, all {len(wl.layers)} layers {phase_words(wl)} on {n_s} of {wl.n} tokens per step"
+    line = {"impl": "reference", "metric": METRIC if wl.phase != "infer" else METRIC_INFER, "value": round(value, 6), "unit": "TFLOP/s", "n_gpus": args.gpus,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(tot_t / args.steps * 1e3, 3),
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
-            "data": "synthetic", "config": {"workload": wl.desc, "n_tokens_sampled": n_s, "mode": "cola"},
+            "data": "synthetic", "config": {"workload": wl.desc, "n_tokens_sampled": n_s,
+                                            "mode": "cola" if wl.phase != "infer" else "infer"},
             "cpu_baseline": {"value": round(value, 6), "unit": "TFLOP/s", "cores": oracle.num_threads(),
                              "kind": "oracle", "sample": sample},
             "e2e": {"value": round(value, 6), "unit": "TFLOP/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
@@ -429,22 +449,36 @@ def run_reference(args, wl):
     return 0
 
 
-def time_steps(fn, steps, stream, dist=None):
+def time_steps(fn, steps, stream, dist=None, flush=None):
+    """Mean device time of one fn() over `steps` back-to-back calls.  With
+    `flush` (a buffer larger than L2), each call is timed alone and the
+    buffer is rewritten between calls, outside the timed intervals."""
     import torch
 
     if dist:
         dist.barrier()
     torch.cuda.synchronize()
-    e0 = torch.cuda.Event(enable_timing=True)
-    e1 = torch.cuda.Event(enable_timing=True)
-    e0.record(stream)
-    for _ in range(steps):
-        fn()
-    e1.record(stream)
-    torch.cuda.synchronize()
+    if flush is None:
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(steps):
+            fn()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        total = e0.elapsed_time(e1)
+    else:
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(steps)]
+        for a, b in ev:
+            flush.fill_(1)
+            a.record(stream)
+            fn()
+            b.record(stream)
+        torch.cuda.synchronize()
+        total = sum(a.elapsed_time(b) for a, b in ev)
     if dist:
         dist.barrier()
-    ms = e0.elapsed_time(e1) / steps
+    ms = total / steps
     if dist:
         t = torch.tensor([ms], device="cuda")
         dist.all_reduce(t, op=dist.ReduceOp.MAX)
@@ -452,14 +486,16 @@ def time_steps(fn, steps, stream, dist=None):
     return ms
 
 
-def full_rank_baseline(wl, device, steps, warmup, seed=0):
-    """Same-shape full-rank layers (fwd Y = X W^T, bwd dX = dY W, dW = dY^T X)
-    with torch.matmul (cuBLAS); layers reading one input (q/k/v, gate/up) are
-    fused into one GEMM with their output widths concatenated."""
+def full_rank_baseline(wl, device, steps, warmup, seed=0, flush=None):
+    """Same-shape full-rank layers (fwd Y = X W^T, bwd dX = dY W, dW = dY^T X;
+    forward only for an inference workload) with torch.matmul (cuBLAS);
+    layers reading one input (q/k/v, gate/up) are fused into one GEMM with
+    their output widths concatenated."""
     import torch
 
     n = wl.n
     bf = torch.bfloat16
+    train = wl.phase != "infer"
     g = torch.Generator(device=device).manual_seed(seed + 77)
     groups = {}
     for L in wl.layers:
@@ -470,24 +506,32 @@ def full_rank_baseline(wl, device, steps, warmup, seed=0):
     for key, Ls in groups.items():
         d_in = Ls[0].d_in
         d_out = sum(L.d_out for L in Ls)
+        # flops count the logical widths; the GEMMs run on widths rounded up
+        # to a multiple of 8 so that cuBLAS gets 16-byte aligned rows (as the
+        # CoLA path gets through its padded pitches)
+        flops += (6.0 if train else 2.0) * n * d_in * d_out
+        d_in, d_out = -(-d_in // 8) * 8, -(-d_out // 8) * 8
         X = torch.randn((n, d_in), generator=g, device=device, dtype=torch.float32).to(bf)
         W = (torch.randn((d_out, d_in), generator=g, device=device, dtype=torch.float32) * d_in ** -0.5).to(bf)
-        dY = torch.randn((n, d_out), generator=g, device=device, dtype=torch.float32).to(bf)
-        bufs.append(dict(X=X, W=W, dY=dY, Y=torch.empty((n, d_out), dtype=bf, device=device),
-                         dX=torch.empty((n, d_in), dtype=bf, device=device),
-                         dW=torch.empty((d_out, d_in), dtype=bf, device=device)))
-        flops += 6.0 * n * d_in * d_out
+        b = dict(X=X, W=W, Y=torch.empty((n, d_out), dtype=bf, device=device))
+        if train:
+            b["dY"] = torch.randn((n, d_out), generator=g, device=device, dtype=torch.float32).to(bf)
+            b["dX"] = torch.empty((n, d_in), dtype=bf, device=device)
+            b["dW"] = torch.empty((d_out, d_in), dtype=bf, device=device)
+        bufs.append(b)
 
     def step():
         for b in bufs:
             torch.matmul(b["X"], b["W"].t(), out=b["Y"])
+        if not train:
+            return
         for b in reversed(bufs):
             torch.matmul(b["dY"], b["W"], out=b["dX"])
             torch.matmul(b["dY"].t(), b["X"], out=b["dW"])
 
     for _ in range(warmup):
         step()
-    ms = time_steps(step, steps, torch.cuda.current_stream())
+    ms = time_steps(step, steps, torch.cuda.current_stream(), flush=flush)
     del bufs
     return {"ms_per_step": round(ms, 4), "tflops": round(flops / (ms / 1e3) / 1e12, 1), "flops": flops,
             "impl": "torch.matmul (cuBLAS) bf16"}
@@ -514,6 +558,8 @@ def run_cola(args, wl):
     peaks = _peaks()
     ridge = peaks["bf16_tflops"] * 1e12 / (peaks["hbm_gbs"] * 1e9)
     mode = args.mode or wl.modes[0]
+    if (mode == "infer") != (wl.phase == "infer"):
+        raise SystemExit(f"mode {mode} does not fit the {wl.phase} workload {wl.name}")
     blk = Block(wl, mode, device, seed=args.seed + rank)
     stream = torch.cuda.current_stream()
 
@@ -526,9 +572,27 @@ def run_cola(args, wl):
     for _ in range(args.warmup):
         blk.step()
     torch.cuda.synchronize()
+    # short steps replay as one CUDA graph: the launches of a step are
+    # recorded once (after the eager warm-up, which set every kernel's
+    # attributes) and replayed with no host work per launch
+    use_graph = args.graph == "on" or (args.graph == "auto" and wl.graph)
+    step_fn = blk.step
+    if use_graph:
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph):
+            blk.step()
+        step_fn = graph.replay
+        for _ in range(args.warmup):
+            step_fn()
+        torch.cuda.synchronize()
+        blk.check()
+    # a working set that fits in L2 is timed step by step with L2 rewritten
+    # between steps
+    ws_bytes = blk.working_set_bytes()
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=device) if ws_bytes < L2_BYTES else None
     sampler = ClockSampler(local)
     sampler.start()
-    ms = time_steps(blk.step, args.steps, stream, dist)
+    ms = time_steps(step_fn, args.steps, stream, dist, flush=flush)
     clocks = sampler.stop()
     blk.check()
 
@@ -543,13 +607,18 @@ def run_cola(args, wl):
 
     flops = wl.flops
     value = flops * world / (ms / 1e3) / 1e12
-    line = {"metric": METRIC, "value": round(value, 2), "unit": "TFLOP/s", "n_gpus": world, "steps": args.steps,
+    line = {"metric": METRIC if blk.train else METRIC_INFER, "value": round(value, 2), "unit": "TFLOP/s", "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": round(ms, 4), "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
             "config": {"workload": wl.desc, "n_tokens": wl.n, "mode": mode, "sigma": "silu",
                        "layers": [f"{L.name}:{L.d_in}->{L.d_out},r={L.r}" for L in wl.layers],
-                       "shared_x_groups": ["+".join(m["L"].name for m in g["members"]) for g in blk.groups], "parallelism": "replicas" if world > 1 else "single-gpu",
-                       "l2": f"no flush: working set {blk.working_set_bytes() / 1e9:.2f} GB > 129 MB L2"},
+                       "shared_x_groups": ["+".join(m["L"].name for m in g["members"]) for g in blk.groups],
+                       "parallelism": "replicas" if world > 1 else "single-gpu",
+                       "phase": "fwd+bwd" if blk.train else "fwd only (inference)",
+                       "cuda_graph": use_graph,
+                       "l2": (f"flushed between steps (256 MB write): working set {ws_bytes / 1e6:.1f} MB < L2"
+                              if flush is not None else
+                              f"no flush: working set {ws_bytes / 1e9:.2f} GB > 129 MB L2")},
             "tokens_per_s": round(wl.n * world / (ms / 1e3), 1),
             "pct_dense_bf16_peak": round(100.0 * value / world / peaks["bf16_tflops"], 2),
             "pct_dense_bf16_peak_sustained": round(100.0 * value / world / peaks["bf16_tflops_sustained"], 2),
@@ -557,8 +626,9 @@ def run_cola(args, wl):
             "gpu_launches": blk.launches_per_step * args.steps, "clocks": clocks}
 
     if not args.no_extras:
-        # end to end: each step's activations and upstream gradients come from
-        # pinned host memory; the weight gradients go back to pinned host memory
+        # end to end: each step's activations (and, training, upstream
+        # gradients) come from pinned host memory; the weight gradients (or,
+        # inference, the outputs) go back to pinned host memory
         def full_rows(t):   # the whole padded row-major buffer behind a view
             return torch.as_strided(t, (t.shape[0], t.stride(0)), (t.stride(0), 1))
 
@@ -572,7 +642,7 @@ def run_cola(args, wl):
         def e2e_step():
             for h, t in zip(h_in, ins):
                 t.copy_(h, non_blocking=True)
-            blk.step()
+            step_fn()
             for h, t in zip(h_out, outs):
                 h.copy_(t, non_blocking=True)
 
@@ -588,7 +658,7 @@ def run_cola(args, wl):
                        "d2h_bytes_per_step": bo}
         del h_in, h_out
         if rank == 0 and world == 1:
-            fr = full_rank_baseline(wl, device, max(3, args.steps // 2), 2, seed=args.seed)
+            fr = full_rank_baseline(wl, device, max(3, args.steps // 2), 3, seed=args.seed, flush=flush)
             fr["speedup_cola_vs_full_rank"] = round(fr["ms_per_step"] / ms, 3)
             line["full_rank"] = fr
             line["cpu_baseline"] = cpu_baseline(wl)
@@ -608,7 +678,9 @@ def main(argv=None):
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="cola", choices=["cola", "reference"])
     ap.add_argument("--workload", default="60m", choices=sorted(WORKLOADS))
-    ap.add_argument("--mode", default=None, choices=["cola", "cola_m"])
+    ap.add_argument("--mode", default=None, choices=["cola", "cola_m", "infer"])
+    ap.add_argument("--graph", default="auto", choices=["auto", "on", "off"],
+                    help="replay each step as one CUDA graph (auto: for the short, launch-bound workloads)")
     ap.add_argument("--seed", type=int, default=0)
     ap.add_argument("--no-extras", action="store_true", help="skip e2e, full-rank and CPU baselines")
     args = ap.parse_args(argv)

@@ -77,7 +77,9 @@ typedef enum {
 
 typedef enum {
     COLA_MODE_COLA = 0,          /* forward stores Z and H; backward reads both */
-    COLA_MODE_COLA_M = 1         /* forward stores Z only; backward recomputes H = sigma(Z) */
+    COLA_MODE_COLA_M = 1,        /* forward stores Z only; backward recomputes H = sigma(Z) */
+    COLA_MODE_INFER = 2          /* forward only (inference, Table 10): nothing is saved, H lives
+                                    in the workspace; the backward entry points reject it */
 } cola_mode_t;
 
 /* The layer of Eq. (main-fwd) as the paper states it: (d_in, d_out, rank r,
@@ -111,9 +113,10 @@ cola_status_t cola_workspace_init(void* ws, void* stream);
 /* Forward, Eq. (main-fwd):  Z = X A^T,  H = sigma(Z),  Y = H B^T.
  *   X [n x d_in] (ld_x), A [r x d_in] (ld_a), B [d_out x r]: inputs.
  *   Y [n x d_out] (ld_y): output.
- *   Z_save [n x r]: output, saved for the backward (both modes).
+ *   Z_save [n x r]: output, saved for the backward (COLA, COLA_M); must be
+ *                   NULL under COLA_MODE_INFER (Z is then never stored).
  *   H_save [n x r]: output under COLA_MODE_COLA; must be NULL under COLA_M
- *                   (H is then formed in the workspace and not kept).
+ *                   and INFER (H is then formed in the workspace and not kept).
  * Two tensor-core GEMMs: Z/H (sigma fused in the epilogue), then Y. */
 cola_status_t cola_fwd(const cola_desc_t* desc, const void* X, const void* A, const void* B, void* Y,
                        void* Z_save, void* H_save, void* ws, size_t ws_bytes, void* stream);
@@ -136,7 +139,8 @@ cola_status_t cola_bwd(const cola_desc_t* desc, const void* X, const void* A, co
  * layers of one shape (desc: d_in, d_out, r per projection) on one X.
  *   A_cat [count r x d_in] (ld_a): the A_j stacked by rows.  One GEMM with
  *     N = count r reads X once and writes Z_cat [n x count r] = [Z_1 .. Z_c]
- *     and, under COLA, H_cat [n x count r] (NULL under COLA_M).
+ *     and, under COLA, H_cat [n x count r] (NULL under COLA_M; under
+ *     COLA_MODE_INFER both Z_cat and H_cat are NULL).
  *   B[j] [d_out x r], Y[j] [n x d_out] (ld_y): host arrays of `count` device
  *     pointers; the count output GEMMs Y_j = H_j B_j^T run as one launch. */
 cola_status_t cola_fwd_shared_x(const cola_desc_t* desc, int32_t count, const void* X, const void* A_cat,

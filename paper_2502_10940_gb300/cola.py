@@ -17,7 +17,7 @@ _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "libcola.so")
 
 SIGMA = {"identity": 0, "silu": 1, "gelu": 2}
-MODE = {"cola": 0, "cola_m": 1}
+MODE = {"cola": 0, "cola_m": 1, "infer": 2}
 STATUS = {0: "COLA_OK", 1: "COLA_ERR_INVALID", 2: "COLA_ERR_ALIGN", 3: "COLA_ERR_UNSUPPORTED",
           4: "COLA_ERR_WORKSPACE", 5: "COLA_ERR_LAUNCH", 6: "COLA_ERR_DEVICE_TIMEOUT"}
 

@@ -58,7 +58,8 @@ cola_status_t check_desc(const cola_desc_t* d, Shape* s)
     if (!d) return COLA_ERR_INVALID;
     if (d->n < 1 || d->d_in < 1 || d->d_out < 1 || d->r < 1) return COLA_ERR_INVALID;
     if (d->sigma < COLA_SIGMA_IDENTITY || d->sigma > COLA_SIGMA_GELU) return COLA_ERR_INVALID;
-    if (d->mode != COLA_MODE_COLA && d->mode != COLA_MODE_COLA_M) return COLA_ERR_INVALID;
+    if (d->mode != COLA_MODE_COLA && d->mode != COLA_MODE_COLA_M && d->mode != COLA_MODE_INFER)
+        return COLA_ERR_INVALID;
     if (d->wgrad_fp32 != 0 && d->wgrad_fp32 != 1) return COLA_ERR_INVALID;
     if (d->reserved != 0) return COLA_ERR_INVALID;
     if (d->r % 64 != 0) return COLA_ERR_UNSUPPORTED;
@@ -84,6 +85,17 @@ cola_status_t check_ptrs(std::initializer_list<const void*> required)
         if (!p) return COLA_ERR_INVALID;
         if (!aligned16(p)) return COLA_ERR_ALIGN;
     }
+    return COLA_OK;
+}
+
+// The saved activations a forward call is given: Z under the training modes,
+// H under CoLA only, neither under inference.
+cola_status_t check_saved(int mode, const void* Z, const void* H)
+{
+    const bool want_z = mode != COLA_MODE_INFER;
+    const bool want_h = mode == COLA_MODE_COLA;
+    if ((Z != nullptr) != want_z || (H != nullptr) != want_h) return COLA_ERR_INVALID;
+    if ((Z && !aligned16(Z)) || (H && !aligned16(H))) return COLA_ERR_ALIGN;
     return COLA_OK;
 }
 
@@ -113,18 +125,22 @@ WgradPlan wgrad_plan(const cola_desc_t& d, int nproj, int sms)
     return plan_wgrad(M, N, nb + 1, d.n, sms);
 }
 
-// dZ [n x R] bf16, H [n x R] bf16 (CoLA-M only), the fp32 split partials of
-// the weight-gradient group.
+// dZ [n x R] bf16 (training modes), H [n x R] bf16 (CoLA-M and inference),
+// the fp32 split partials of the weight-gradient group (training modes).
 WsLayout ws_layout(const cola_desc_t& d, int nproj, int sms)
 {
     const int64_t R = nproj * d.r;
     WsLayout L;
     size_t off = WS_HEADER;
     L.dz_off = off;
-    off += align_up(static_cast<size_t>(d.n) * R * 2);
+    if (d.mode != COLA_MODE_INFER) off += align_up(static_cast<size_t>(d.n) * R * 2);
     L.h_off = off;
-    if (d.mode == COLA_MODE_COLA_M) off += align_up(static_cast<size_t>(d.n) * R * 2);
+    if (d.mode != COLA_MODE_COLA) off += align_up(static_cast<size_t>(d.n) * R * 2);
     L.part_off = off;
+    if (d.mode == COLA_MODE_INFER) {
+        L.total = off;
+        return L;
+    }
     const WgradPlan w = wgrad_plan(d, nproj, sms);
     if (w.splits > 1 || d.wgrad_fp32) off += align_up(static_cast<size_t>(w.part_elems) * 4);
     L.total = off;
@@ -213,11 +229,13 @@ cola_status_t run_f1(const Shape& s, int sigma, int64_t N, const void* X, const 
     pr.p = base_params(s.n, N, s.d_in, bn, ms);
     COLA_MAP(map_kmajor(&pr.map_a, X, s.d_in, s.n, s.ld_x, BM * ms));
     COLA_MAP(map_kmajor(&pr.map_b, A, s.d_in, N, s.ld_a, bn));
-    COLA_MAP(map_box32(&pr.map_d, Z, N, s.n, ldz));
+    // Z == nullptr (inference): the epilogue stores H alone, through map_d
+    COLA_MAP(map_box32(&pr.map_d, Z ? Z : H, N, s.n, ldz));
     pr.map_d2 = pr.map_d;
-    if (H) COLA_MAP(map_box32(&pr.map_d2, H, N, s.n, ldz));
+    if (Z && H) COLA_MAP(map_box32(&pr.map_d2, H, N, s.n, ldz));
     pr.map_z = pr.map_d;
-    pr.p.has_d2 = H != nullptr;
+    pr.p.has_d2 = Z && H;
+    pr.p.h_only = Z == nullptr;
     pr.p.sigma = sigma;
     pr.p.status = status;
     const int64_t mnk[1][3] = {{s.n, N, s.d_in}};
@@ -400,17 +418,15 @@ cola_status_t cola_fwd(const cola_desc_t* desc, const void* X, const void* A, co
 {
     Shape s;
     COLA_TRY(check_desc(desc, &s));
-    COLA_TRY(check_ptrs({X, A, B, Y, Z_save}));
-    const bool cola_m = desc->mode == COLA_MODE_COLA_M;
-    if (cola_m ? H_save != nullptr : H_save == nullptr) return COLA_ERR_INVALID;
-    if (H_save && !aligned16(H_save)) return COLA_ERR_ALIGN;
+    COLA_TRY(check_ptrs({X, A, B, Y}));
+    COLA_TRY(check_saved(desc->mode, Z_save, H_save));
     int sms = 0;
     COLA_TRY(device_info(&sms));
     WsLayout L;
     COLA_TRY(check_ws(*desc, 1, sms, ws, ws_bytes, &L));
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     unsigned int* status = ws_status(ws);
-    void* H = cola_m ? static_cast<void*>(wsb(ws) + L.h_off) : H_save;
+    void* H = desc->mode != COLA_MODE_COLA ? static_cast<void*>(wsb(ws) + L.h_off) : H_save;
     COLA_TRY(run_f1(s, desc->sigma, s.r, X, A, Z_save, H, s.r, status, sms, st));
     const void* Hs[1] = {H};
     const void* Bs[1] = {B};
@@ -424,6 +440,7 @@ cola_status_t cola_bwd(const cola_desc_t* desc, const void* X, const void* A, co
 {
     Shape s;
     COLA_TRY(check_desc(desc, &s));
+    if (desc->mode == COLA_MODE_INFER) return COLA_ERR_INVALID;
     COLA_TRY(check_ptrs({X, A, B, dY, Z_save, dX, dA, dB}));
     const bool cola_m = desc->mode == COLA_MODE_COLA_M;
     if (cola_m ? H_save != nullptr : H_save == nullptr) return COLA_ERR_INVALID;
@@ -459,11 +476,9 @@ cola_status_t cola_fwd_shared_x(const cola_desc_t* desc, int32_t count, const vo
     Shape s;
     COLA_TRY(check_desc(desc, &s));
     if (count < 2 || count > 3 || !B || !Y) return COLA_ERR_INVALID;
-    COLA_TRY(check_ptrs({X, A_cat, Z_cat}));
+    COLA_TRY(check_ptrs({X, A_cat}));
     for (int j = 0; j < count; ++j) COLA_TRY(check_ptrs({B[j], Y[j]}));
-    const bool cola_m = desc->mode == COLA_MODE_COLA_M;
-    if (cola_m ? H_cat != nullptr : H_cat == nullptr) return COLA_ERR_INVALID;
-    if (H_cat && !aligned16(H_cat)) return COLA_ERR_ALIGN;
+    COLA_TRY(check_saved(desc->mode, Z_cat, H_cat));
     int sms = 0;
     COLA_TRY(device_info(&sms));
     WsLayout L;
@@ -472,7 +487,7 @@ cola_status_t cola_fwd_shared_x(const cola_desc_t* desc, int32_t count, const vo
     unsigned int* status = ws_status(ws);
     const int64_t R = count * s.r;
     const size_t slice = static_cast<size_t>(s.r) * 2;   // bytes between the projections' column blocks
-    uint8_t* H = cola_m ? wsb(ws) + L.h_off : static_cast<uint8_t*>(H_cat);
+    uint8_t* H = desc->mode != COLA_MODE_COLA ? wsb(ws) + L.h_off : static_cast<uint8_t*>(H_cat);
     COLA_TRY(run_f1(s, desc->sigma, R, X, A_cat, Z_cat, H, R, status, sms, st));
     const void* Hs[3] = {H, H + slice, H + 2 * slice};
     return run_f2(s, count, Hs, R, B, Y, status, sms, st);
@@ -484,7 +499,7 @@ cola_status_t cola_bwd_shared_x(const cola_desc_t* desc, int32_t count, const vo
 {
     Shape s;
     COLA_TRY(check_desc(desc, &s));
-    if (count < 2 || count > 3 || !B || !dY || !dB) return COLA_ERR_INVALID;
+    if (count < 2 || count > 3 || !B || !dY || !dB || desc->mode == COLA_MODE_INFER) return COLA_ERR_INVALID;
     COLA_TRY(check_ptrs({X, A_cat, Z_cat, dX, dA_cat}));
     for (int j = 0; j < count; ++j) COLA_TRY(check_ptrs({B[j], dY[j], dB[j]}));
     const bool cola_m = desc->mode == COLA_MODE_COLA_M;

@@ -68,6 +68,7 @@ struct GemmParams {
     long long ldd;         // EPI_F32: row pitch of a slab in elements
     long long part_stride; // EPI_F32: elements per split slab
     int has_d2;            // EPI_ZH / EPI_DSIGMA: also store H through map_d2
+    int h_only;            // EPI_ZH: store H = sigma(bf16(acc)) through map_d and nothing else
     // The bf16 output behind map_d, for the one 32-column chunk per row block
     // that holds a ragged right edge (N % 8 != 0): a TMA store clips at
     // 16-byte granularity and would write the row padding past column N, so
@@ -591,15 +592,15 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 #pragma unroll
                     for (int j = 0; j < 16; ++j)
                         w[j] = pack_bf16x2(__uint_as_float(v[2 * j]), __uint_as_float(v[2 * j + 1]));
-                    emit(map_d, w, col0, row0);
-                    if (p.has_d2) {
+                    if (!p.h_only) emit(map_d, w, col0, row0);
+                    if (p.has_d2 || p.h_only) {
                         with_sigma(p.sigma, [&](auto tag) {
                             constexpr int S = decltype(tag)::value;
 #pragma unroll
                             for (int j = 0; j < 16; ++j)
                                 w[j] = pack_bf16x2(act_sigma<S>(bf16_lo(w[j])), act_sigma<S>(bf16_hi(w[j])));
                         });
-                        emit(map_d2, w, col0, row0);
+                        emit(p.h_only ? map_d : map_d2, w, col0, row0);
                     }
                 } else if (EPI == EPI_DSIGMA) {
                     const int b = zuse & 1;

@@ -33,10 +33,13 @@ class Workload:
     desc: str = ""
     seqs: int = 0
     seq_len: int = 256
+    phase: str = "train"    # "train": forward + backward; "infer": forward only, nothing saved
+    graph: bool = False     # replay each step as one CUDA graph (short, launch-bound steps)
 
     @property
     def flops(self) -> float:
-        return float(sum(layer_flops(self.n, l.d_in, l.d_out, l.r) for l in self.layers))
+        f = fwd_flops if self.phase == "infer" else layer_flops
+        return float(sum(f(self.n, l.d_in, l.d_out, l.r) for l in self.layers))
 
 
 def layer_flops(n: int, d_in: int, d_out: int, r: int) -> int:
@@ -73,7 +76,7 @@ def paper_flops_cola(n: int, d: int, d_ff: int, r: int) -> float:
 WORKLOADS = {
     "60m-q": Workload("60m-q", 2048, (Layer("q", 512, 512, 128, "x_attn"),), fused_qkv=False,
                       desc="single CoLA layer, LLaMA-60M q-proj shape, n=2048, 512->512, r=128",
-                      seqs=8),
+                      seqs=8, graph=True),
     "60m": Workload("60m", 65536, llama_block(512, 1376, 128),
                     desc="LLaMA-60M-shaped CoLA block, 7 layers, d=512, d_ff=1376, r=128, "
                          "65536 tokens (256 x 256)", seqs=256),
@@ -86,4 +89,11 @@ WORKLOADS = {
     "7b": Workload("7b", 32768, llama_block(4096, 11008, 1024), modes=("cola_m", "cola"),
                    desc="LLaMA-7B-shaped CoLA block, d=4096, d_ff=11008, r=1024, 32768 tokens "
                         "(128 x 256)", seqs=128),
+    # inference at the pre-training shapes with 32 sequences of 256 tokens (Table 10)
+    "1b-infer": Workload("1b-infer", 8192, llama_block(2048, 5461, 512), modes=("infer",), phase="infer",
+                         graph=True, desc="LLaMA-1B-shaped CoLA block, forward only (inference), d=2048, "
+                                          "d_ff=5461, r=512, 8192 tokens (32 x 256)", seqs=32),
+    "7b-infer": Workload("7b-infer", 8192, llama_block(4096, 11008, 1024), modes=("infer",), phase="infer",
+                         graph=True, desc="LLaMA-7B-shaped CoLA block, forward only (inference), d=4096, "
+                                          "d_ff=11008, r=1024, 8192 tokens (32 x 256)", seqs=32),
 }

@@ -148,6 +148,22 @@ def test_shared_x_argument_errors(L):
     assert g(ctypes.byref(dm), 2, FAKE, FAKE, ok2, ok2, FAKE, None, FAKE, FAKE, bad, FAKE, 1 << 20, None) == 2
 
 
+def test_infer_mode_argument_errors(L):
+    d = L.desc(256, 128, 128, 64, mode="infer")
+    f = L.lib().cola_fwd
+    # inference saves nothing: Z_save and H_save must both be NULL
+    assert f(ctypes.byref(d), FAKE, FAKE, FAKE, FAKE, FAKE, None, FAKE, 1 << 20, None) == 1
+    assert f(ctypes.byref(d), FAKE, FAKE, FAKE, FAKE, None, FAKE, FAKE, 1 << 20, None) == 1
+    # the backward entry points reject the inference mode
+    assert L.lib().cola_bwd(ctypes.byref(d), *([FAKE] * 5), None, *([FAKE] * 4), 1 << 20, None) == 1
+    ok2 = (ctypes.c_void_p * 2)(FAKE, FAKE)
+    assert L.lib().cola_bwd_shared_x(ctypes.byref(d), 2, FAKE, FAKE, ok2, ok2, FAKE, None, FAKE, FAKE, ok2, FAKE,
+                                     1 << 20, None) == 1
+    # a training-mode forward still needs Z_save
+    dc = L.desc(256, 128, 128, 64, mode="cola_m")
+    assert f(ctypes.byref(dc), FAKE, FAKE, FAKE, FAKE, None, None, FAKE, 1 << 20, None) == 1
+
+
 def test_workspace_init_and_check_reject_null(L):
     assert L.lib().cola_workspace_init(None, None) == 1
     assert L.lib().cola_workspace_init(FAKE + 16, None) == 2   # not 256-byte aligned

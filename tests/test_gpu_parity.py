@@ -186,3 +186,47 @@ def test_shared_x_pair_matches_oracle(shape, mode):
         assert_close(f"dA{j}", to64(dA[j * r:(j + 1) * r]), dAo[j])
     assert_close("dX", to64(dX), dXo)
     assert padding_intact(dX, d_in) and padding_intact(Ys[0], d_out)
+
+
+@pytest.mark.parametrize("shape", [(300, 200, 328, 128), (257, 520, 136, 256), (1, 64, 64, 64)], ids=str)
+def test_infer_forward_matches_training_forward(shape):
+    # the inference forward stores H alone; Y is bit for bit the training
+    # forward's Y (the same kernels round Z, apply sigma and run the Y GEMM),
+    # and within tolerance of the oracle
+    from paper_2502_10940_gb300 import cola
+    n, d_in, d_out, r = shape
+    inp = make_inputs(n, d_in, d_out, r, seed=40)
+    ref = gpu_layer(inp, "silu", "cola")
+    d = cola.desc(n, d_in, d_out, r, ld_x=cola.ld_of(inp["X"]), ld_y=cola.ld_of(inp["dY"]),
+                  ld_a=cola.ld_of(inp["A"]), sigma="silu", mode="infer")
+    ws = cola.workspace(d)
+    Y = padded_empty(n, d_out, cola.ld_of(inp["dY"]))
+    cola.cola_fwd(d, inp["X"], inp["A"], inp["B"], Y, None, None, ws)
+    assert cola.cola_check_status(ws)[0] == 0
+    assert torch.equal(Y, ref["Y"])
+    assert_close("Y", to64(Y), oracle_layer(inp, "silu", "cola")["Y"])
+    assert padding_intact(Y, d_out)
+
+
+def test_infer_shared_x_matches_training_forward():
+    from paper_2502_10940_gb300 import cola
+    n, d, r = 2048, 512, 128
+    X = make_inputs(n, d, d, r, seed=41)["X"]
+    parts = [make_inputs(n, d, d, r, seed=42 + j) for j in range(3)]
+    ldx = cola.ld_of(X)
+    A_cat = padded_empty(3 * r, d, ldx)
+    A_cat.copy_(torch.cat([p["A"] for p in parts], 0))
+    Bs = [p["B"] for p in parts]
+    ldy = cola.ld_of(parts[0]["dY"])
+    outs = {}
+    for mode in ("cola", "infer"):
+        desc = cola.desc(n, d, d, r, ld_x=ldx, ld_y=ldy, ld_a=ldx, sigma="silu", mode=mode)
+        ws = cola.workspace(desc, nproj=3)
+        Ys = [padded_empty(n, d, ldy) for _ in range(3)]
+        Z = torch.empty((n, 3 * r), dtype=torch.bfloat16, device="cuda") if mode == "cola" else None
+        H = torch.empty((n, 3 * r), dtype=torch.bfloat16, device="cuda") if mode == "cola" else None
+        cola.cola_fwd_shared_x(desc, X, A_cat, Bs, Ys, Z, H, ws)
+        assert cola.cola_check_status(ws)[0] == 0
+        outs[mode] = Ys
+    for a, b in zip(outs["cola"], outs["infer"]):
+        assert torch.equal(a, b)
