@@ -196,10 +196,12 @@ def launch_cost(kind, shapes, splits, flags):
             b = e * (m * k + n * k + m * n)
         elif kind == "reduce":
             b = e * m * n
+        elif kind == "sigma":
+            b = e * 2 * m * n
         else:
             b = 0
         tb += b
-        tf += 0.0 if kind == "reduce" else 2.0 * m * n * k
+        tf += 0.0 if kind in ("reduce", "sigma") else 2.0 * m * n * k
     return tb, tf
 
 
@@ -615,6 +617,8 @@ def run_cola(args, wl):
                        "shared_x_groups": ["+".join(m["L"].name for m in g["members"]) for g in blk.groups],
                        "parallelism": "replicas" if world > 1 else "single-gpu",
                        "phase": "fwd+bwd" if blk.train else "fwd only (inference)",
+                       "saved_activation_elems": sum(g[k].numel() for g in blk.groups for k in ("Z", "H")
+                                                     if g.get(k) is not None),
                        "cuda_graph": use_graph,
                        "l2": (f"flushed between steps (256 MB write): working set {ws_bytes / 1e6:.1f} MB < L2"
                               if flush is not None else

@@ -177,6 +177,20 @@ cola_status_t cola_bwd_qkv_fused(const cola_desc_t* desc, const void* X, const v
                                  const void* dY_v, const void* Z_qkv, const void* H_qkv, void* dX, void* dA_qkv,
                                  void* dB_q, void* dB_k, void* dB_v, void* ws, size_t ws_bytes, void* stream);
 
+/* Block-level CoLA-M recompute of the up-projections (Sec. 4.2, App. C:
+ * in the backward, CoLA-M recomputes B sigma(.) from the saved low-rank
+ * activation instead of keeping the layer output):
+ *   Y_j = sigma(Z_j) B_j^T        for j < count (1..3 projections)
+ * Z_cat [n x count r]: the Z saved by cola_fwd / cola_fwd_shared_x under
+ * COLA_MODE_COLA_M (column block j = Z_j).  B[j] [d_out x r], Y[j]
+ * [n x d_out] (ld_y): host arrays of `count` device pointers.  desc->mode
+ * must be COLA_MODE_COLA_M; ws must be sized by cola_workspace_size(desc,
+ * count), and H = sigma(Z) is formed in it (one elementwise launch) before
+ * the count output GEMMs run as one launch.  Y_j is bit for bit the Y_j of
+ * the forward call that saved Z_cat. */
+cola_status_t cola_recompute_up(const cola_desc_t* desc, int32_t count, const void* Z_cat, const void* const* B,
+                                void* const* Y, void* ws, size_t ws_bytes, void* stream);
+
 /* Synchronise `stream`, read and clear the workspace status word.
  * Returns COLA_OK, or COLA_ERR_DEVICE_TIMEOUT if a kernel that used this
  * workspace gave up on a wait since the last check (*code_out, if not NULL,
@@ -236,7 +250,8 @@ typedef enum {
     COLA_KERNEL_BWD_DZ = 2,      /* dZ = (dY B) * sigma'(Z)               (M=n, N=r, K=d_out) */
     COLA_KERNEL_WGRAD = 3,       /* dB = dY^T H and dA = dZ^T X, token split (M=d_out | r, N=r | d_in, K=n) */
     COLA_KERNEL_REDUCE = 4,      /* fixed-order sum of the partials       (M, N of the gradient, K=splits) */
-    COLA_KERNEL_BWD_DX = 5       /* dX = dZ A                             (M=n, N=d_in, K=r or 3r) */
+    COLA_KERNEL_BWD_DX = 5,      /* dX = dZ A                             (M=n, N=d_in, K=r or 3r) */
+    COLA_KERNEL_SIGMA = 6        /* H = sigma(Z), elementwise             (M=n, N=count r, K=0) */
 } cola_kernel_t;
 
 typedef struct {

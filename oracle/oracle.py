@@ -11,6 +11,8 @@ Definitions followed (arXiv 2502.10940):
     recomputed from it in the backward.
   * fused q/k/v -- Fig. 4: the q, k and v auto-encoders read the same x, so
     they are three independent layers sharing X, and dX is their sum.
+  * CoLA-M block recompute -- Sec. 4.2 / App. C: the up-projection B sigma(.)
+    is recomputed in the backward from the saved Z: Y = sigma(Z) B^T.
 
 Every function takes / returns numpy arrays.  Full routines take float64;
 the *_bf16 routines take bf16 bit patterns (uint16) and widen them exactly.
@@ -24,7 +26,7 @@ from .build import build as _build
 
 __all__ = [
     "SIGMA", "MODE", "lib", "sigma", "dsigma", "round_bf16", "widen_bf16",
-    "fwd", "bwd", "fwd_qkv", "bwd_qkv", "rows_bf16", "dA_entries_bf16",
+    "fwd", "bwd", "fwd_qkv", "bwd_qkv", "recompute_up", "rows_bf16", "dA_entries_bf16",
     "dB_entries_bf16", "num_threads",
 ]
 
@@ -161,6 +163,16 @@ def bwd(X, A, B, dY, Z, H=None, sigma="silu", mode="cola", round_store=False):
     lib().oracle_bwd(n, d_in, d_out, r, _sig(sigma), m, int(bool(round_store)), px, pa, pb, pdy,
                      pz, ph, pdx, pda, pdb, pdz)
     return dX, dA, dB, dZ
+
+
+def recompute_up(Z, B, sigma_kind="silu"):
+    """CoLA-M's recompute of a layer output from its saved rank-r activation
+    (Sec. 4.2, App. C): Y = sigma(Z) B^T, sigma from the oracle's own fp64
+    routine, the product by numpy.  Returns Y [n x d_out]."""
+    Z, _ = _f64(Z)
+    B, _ = _f64(B)
+    assert Z.shape[1] == B.shape[1]
+    return sigma(sigma_kind, Z) @ B.T
 
 
 def fwd_qkv(X, As, Bs, sigma="silu", round_store=False):

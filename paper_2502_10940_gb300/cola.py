@@ -23,10 +23,10 @@ STATUS = {0: "COLA_OK", 1: "COLA_ERR_INVALID", 2: "COLA_ERR_ALIGN", 3: "COLA_ERR
 
 # the entry points include/cola.h declares
 SYMBOLS = ("cola_workspace_size", "cola_workspace_init", "cola_fwd", "cola_bwd", "cola_fwd_shared_x",
-           "cola_bwd_shared_x", "cola_fwd_qkv_fused", "cola_bwd_qkv_fused", "cola_check_status",
+           "cola_bwd_shared_x", "cola_recompute_up", "cola_fwd_qkv_fused", "cola_bwd_qkv_fused", "cola_check_status",
            "cola_wgrad_static_scratch", "cola_trace_attach", "cola_trace_detach", "cola_status_string")
 STATIC_SCRATCH_BYTES = 64 * 1024 * 1024
-KERNELS = {0: "fwd_zh", 1: "fwd_y", 2: "bwd_dz", 3: "wgrad", 4: "reduce", 5: "bwd_dx"}
+KERNELS = {0: "fwd_zh", 1: "fwd_y", 2: "bwd_dz", 3: "wgrad", 4: "reduce", 5: "bwd_dx", 6: "sigma"}
 
 
 class ColaError(RuntimeError):
@@ -75,6 +75,8 @@ def lib():
         l.cola_bwd_shared_x.argtypes = [D, ctypes.c_int32, _vp, _vp, PP, PP, _vp, _vp, _vp, _vp, PP, _vp,
                                         ctypes.c_size_t, _vp]
         l.cola_bwd_shared_x.restype = st
+        l.cola_recompute_up.argtypes = [D, ctypes.c_int32, _vp, PP, PP, _vp, ctypes.c_size_t, _vp]
+        l.cola_recompute_up.restype = st
         l.cola_fwd_qkv_fused.argtypes = [D] + [_vp] * 11 + [ctypes.c_size_t, _vp]
         l.cola_fwd_qkv_fused.restype = st
         l.cola_bwd_qkv_fused.argtypes = [D] + [_vp] * 16 + [ctypes.c_size_t, _vp]
@@ -177,6 +179,11 @@ def cola_bwd_shared_x(d, X, A_cat, Bs, dYs, Z_cat, H_cat, dX, dA_cat, dBs, ws, s
     _check(lib().cola_bwd_shared_x(ctypes.byref(d), len(Bs), _ptr(X), _ptr(A_cat), _ptr_array(Bs), _ptr_array(dYs),
                                    _ptr(Z_cat), _ptr(H_cat), _ptr(dX), _ptr(dA_cat), _ptr_array(dBs), _ptr(ws),
                                    _nbytes(ws), _stream(stream)), "cola_bwd_shared_x")
+
+
+def cola_recompute_up(d, Z_cat, Bs, Ys, ws, stream=None):
+    _check(lib().cola_recompute_up(ctypes.byref(d), len(Bs), _ptr(Z_cat), _ptr_array(Bs), _ptr_array(Ys), _ptr(ws),
+                                   _nbytes(ws), _stream(stream)), "cola_recompute_up")
 
 
 def cola_fwd_qkv_fused(d, X, A_qkv, B_q, B_k, B_v, Y_q, Y_k, Y_v, Z_qkv, H_qkv, ws, stream=None):

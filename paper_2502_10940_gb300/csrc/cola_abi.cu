@@ -239,7 +239,7 @@ cola_status_t run_f1(const Shape& s, int sigma, int64_t N, const void* X, const 
     pr.p.sigma = sigma;
     pr.p.status = status;
     const int64_t mnk[1][3] = {{s.n, N, s.d_in}};
-    return run_batch<false, false, EPI_ZH>(COLA_KERNEL_FWD_ZH, bn, ms, &pr, mnk, 1, H != nullptr, sms, st);
+    return run_batch<false, false, EPI_ZH>(COLA_KERNEL_FWD_ZH, bn, ms, &pr, mnk, 1, Z && H, sms, st);
 }
 
 // F2: Y_j = H_j B_j^T for `count` projections of one shape (H_j [n x r] with
@@ -555,6 +555,31 @@ cola_status_t cola_bwd_qkv_fused(const cola_desc_t* desc, const void* X, const v
     const void* dY[3] = {dY_q, dY_k, dY_v};
     void* dB[3] = {dB_q, dB_k, dB_v};
     return cola_bwd_shared_x(desc, 3, X, A_qkv, B, dY, Z_qkv, H_qkv, dX, dA_qkv, dB, ws, ws_bytes, stream);
+}
+
+cola_status_t cola_recompute_up(const cola_desc_t* desc, int32_t count, const void* Z_cat, const void* const* B,
+                                void* const* Y, void* ws, size_t ws_bytes, void* stream)
+{
+    Shape s;
+    COLA_TRY(check_desc(desc, &s));
+    if (desc->mode != COLA_MODE_COLA_M || count < 1 || count > 3 || !B || !Y) return COLA_ERR_INVALID;
+    COLA_TRY(check_ptrs({Z_cat}));
+    for (int j = 0; j < count; ++j) COLA_TRY(check_ptrs({B[j], Y[j]}));
+    int sms = 0;
+    COLA_TRY(device_info(&sms));
+    WsLayout L;
+    COLA_TRY(check_ws(*desc, count, sms, ws, ws_bytes, &L));
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    unsigned int* status = ws_status(ws);
+    const int64_t R = count * s.r;
+    uint8_t* H = wsb(ws) + L.h_off;
+    const int64_t mnk[1][3] = {{s.n, R, 0}};
+    COLA_TRY(launched(traced(COLA_KERNEL_SIGMA, 1, mnk, 1, 0, st, [&] {
+        return launch_sigma(Z_cat, H, static_cast<long long>(s.n) * R, desc->sigma, sms, st);
+    })));
+    const size_t slice = static_cast<size_t>(s.r) * 2;
+    const void* Hs[3] = {H, H + slice, H + 2 * slice};
+    return run_f2(s, count, Hs, R, B, Y, status, sms, st);
 }
 
 cola_status_t cola_check_status(void* ws, void* stream, uint32_t* code_out)

@@ -34,6 +34,10 @@ struct ReduceBatch {
 
 cudaError_t launch_splitk_reduce(ReduceBatch& batch, cudaStream_t stream);
 
+// H = bf16(sigma(Z)) elementwise over `elems` bf16 values (a multiple of 8;
+// both pointers 16-byte aligned).
+cudaError_t launch_sigma(const void* Z, void* H, long long elems, int sigma, int sms, cudaStream_t stream);
+
 #ifdef COLA_DEFINE_LAUNCHERS
 template <int BN, int MSUB, bool A_MN, bool B_MN, int EPI>
 cudaError_t launch_gemm(const GemmBatch& batch, int grid, bool pdl, cudaStream_t stream)

@@ -51,6 +51,16 @@ def fwd_flops(n: int, d_in: int, d_out: int, r: int) -> int:
     return 2 * n * r * (d_in + d_out)
 
 
+def saved_activation_elems(wl: "Workload", mode: str) -> int:
+    """Elements the layer path keeps from the forward for the backward: Z and
+    H (n r each) per layer under CoLA, Z alone under CoLA-M, nothing for
+    inference.  For a block with one rank r that is App. C's low-rank terms:
+    +14nr for CoLA, 7nr for CoLA-M (whose 2nd of block inputs lies outside
+    the layers)."""
+    per = {"cola": 2, "cola_m": 1, "infer": 0}[mode]
+    return sum(per * wl.n * l.r for l in wl.layers)
+
+
 def llama_block(d: int, d_ff: int, r: int) -> tuple:
     return (
         Layer("q", d, d, r, "x_attn"),

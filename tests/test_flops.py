@@ -71,3 +71,16 @@ def test_workload_flops():
     assert W.WORKLOADS["1b"].flops == pytest.approx(7.83e12, rel=2e-3)
     assert W.WORKLOADS["7b"].flops == pytest.approx(1.572e13, rel=2e-3)
     assert W.WORKLOADS["60m-q"].flops == pytest.approx(1.61e9, rel=2e-3)
+
+
+@pytest.mark.parametrize("name", ["60m", "1b", "7b"])
+def test_saved_activations_app_c(name):
+    # App. C: CoLA adds 14nr of low-rank activations per block (nr for Ax and
+    # nr for sigma(Ax) in each of the 7 layers); CoLA-M keeps 7nr (plus the
+    # 2nd of block inputs, which the layers do not hold)
+    wl = W.WORKLOADS[name]
+    r = wl.layers[0].r
+    assert all(l.r == r for l in wl.layers) and len(wl.layers) == 7
+    assert W.saved_activation_elems(wl, "cola") == 14 * wl.n * r
+    assert W.saved_activation_elems(wl, "cola_m") == 7 * wl.n * r
+    assert W.saved_activation_elems(wl, "infer") == 0

@@ -326,3 +326,22 @@ def test_sampled_oracle_padded_row_pitch():
                                dA[ii, kk], rtol=1e-13)
     oo, ii2 = np.array([10, 0]), np.array([3, 2])
     np.testing.assert_allclose(oracle.dB_entries_bf16(Xp, Ab, dYp, oo, ii2, "silu"), dB[oo, ii2], rtol=1e-13)
+
+
+# --- CoLA-M block-level recompute of the up-projection (Sec. 4.2, App. C) ---
+
+@pytest.mark.parametrize("kind", SIGMAS)
+def test_recompute_up_reproduces_forward_output(kind):
+    # recomputing B sigma(.) from the saved Z gives the forward's Y: the C
+    # forward's loops against sigma + a numpy product
+    X, A, B, _ = _rand_layer(23, 17, 31, 5)
+    Z, _, Y = oracle.fwd(X, A, B, kind)
+    np.testing.assert_allclose(oracle.recompute_up(Z, B, kind), Y, rtol=1e-12, atol=1e-12)
+
+
+def test_recompute_up_worked_example():
+    # one token, r = 2: Z = [0, 1], B = [[1, 2], [-3, 0.5]], SiLU:
+    # sigma(0) = 0 and sigma(1) = 1 / (1 + e^-1), so Y = [2 s, 0.5 s] with s = sigma(1)
+    s = 1.0 / (1.0 + math.exp(-1.0))
+    Y = oracle.recompute_up(np.array([[0.0, 1.0]]), np.array([[1.0, 2.0], [-3.0, 0.5]]), "silu")
+    np.testing.assert_allclose(Y, [[2.0 * s, 0.5 * s]], rtol=1e-15)
