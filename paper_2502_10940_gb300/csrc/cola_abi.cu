@@ -222,13 +222,13 @@ cola_status_t run_batch(int kind, int bn, int msub, const GemmProblem* probs, co
 cola_status_t run_f1(const Shape& s, int sigma, int64_t N, const void* X, const void* A, void* Z, void* H,
                      int64_t ldz, unsigned int* status, int sms, cudaStream_t st)
 {
-    const int bn = choose_bn(N);
+    const int bn = choose_bn_for(s.n, N, s.d_in);
     const int ms = choose_msub(s.n, N, s.d_in, bn);
     GemmProblem pr;
     std::memset(&pr, 0, sizeof pr);
     pr.p = base_params(s.n, N, s.d_in, bn, ms);
-    COLA_MAP(map_kmajor(&pr.map_a, X, s.d_in, s.n, s.ld_x, BM * ms));
-    COLA_MAP(map_kmajor(&pr.map_b, A, s.d_in, N, s.ld_a, bn));
+    COLA_MAP(map_kmajor(&pr.map_a, X, s.d_in, s.n, s.ld_x, a_box_rows(ms)));
+    COLA_MAP(map_kmajor(&pr.map_b, A, s.d_in, N, s.ld_a, b_box_rows(bn, ms)));
     // Z == nullptr (inference): the epilogue stores H alone, through map_d
     COLA_MAP(map_box32(&pr.map_d, Z ? Z : H, N, s.n, ldz));
     pr.map_d2 = pr.map_d;
@@ -247,15 +247,15 @@ cola_status_t run_f1(const Shape& s, int sigma, int64_t N, const void* X, const 
 cola_status_t run_f2(const Shape& s, int count, const void* const* H, int64_t ldh, const void* const* B,
                      void* const* Y, unsigned int* status, int sms, cudaStream_t st)
 {
-    const int bn = choose_bn(s.d_out);
+    const int bn = choose_bn_for(s.n, s.d_out, s.r);
     const int ms = choose_msub(s.n, s.d_out, s.r, bn);
     GemmProblem pr[MAX_GROUP];
     int64_t mnk[MAX_GROUP][3];
     std::memset(pr, 0, sizeof pr);
     for (int j = 0; j < count; ++j) {
         pr[j].p = base_params(s.n, s.d_out, s.r, bn, ms);
-        COLA_MAP(map_kmajor(&pr[j].map_a, H[j], s.r, s.n, ldh, BM * ms));
-        COLA_MAP(map_kmajor(&pr[j].map_b, B[j], s.r, s.d_out, s.r, bn));
+        COLA_MAP(map_kmajor(&pr[j].map_a, H[j], s.r, s.n, ldh, a_box_rows(ms)));
+        COLA_MAP(map_kmajor(&pr[j].map_b, B[j], s.r, s.d_out, s.r, b_box_rows(bn, ms)));
         COLA_MAP(map_box32(&pr[j].map_d, Y[j], s.d_out, s.n, s.ld_y));
         pr[j].map_d2 = pr[j].map_z = pr[j].map_d;
         pr[j].p.d_ptr = static_cast<__nv_bfloat16*>(Y[j]);
@@ -274,14 +274,14 @@ cola_status_t run_b1(const Shape& s, int sigma, int count, const void* const* dY
                      const void* const* Z, int64_t ldz, void* const* dZ, void* const* Hout, unsigned int* status,
                      int sms, cudaStream_t st)
 {
-    const int bn = choose_bn(s.r);
+    const int bn = choose_bn_for(s.n, s.r, s.d_out);
     const int ms = choose_msub(s.n, s.r, s.d_out, bn);
     GemmProblem pr[MAX_GROUP];
     int64_t mnk[MAX_GROUP][3];
     std::memset(pr, 0, sizeof pr);
     for (int j = 0; j < count; ++j) {
         pr[j].p = base_params(s.n, s.r, s.d_out, bn, ms);
-        COLA_MAP(map_kmajor(&pr[j].map_a, dY[j], s.d_out, s.n, s.ld_y, BM * ms));
+        COLA_MAP(map_kmajor(&pr[j].map_a, dY[j], s.d_out, s.n, s.ld_y, a_box_rows(ms)));
         COLA_MAP(map_mnmajor(&pr[j].map_b, B[j], s.r, s.d_out, s.r));
         COLA_MAP(map_box32(&pr[j].map_d, dZ[j], s.r, s.n, ldz));
         COLA_MAP(map_box32(&pr[j].map_z, Z[j], s.r, s.n, ldz));
@@ -372,12 +372,12 @@ cola_status_t run_wgrad(const WgradPlan& w, int64_t ntok, const WgradJob* jobs, 
 cola_status_t run_b4(const Shape& s, int64_t K, const void* dZ, int64_t ldz, const void* A, void* dX,
                      unsigned int* status, int sms, cudaStream_t st)
 {
-    const int bn = choose_bn(s.d_in);
+    const int bn = choose_bn_for(s.n, s.d_in, K);
     const int ms = choose_msub(s.n, s.d_in, K, bn);
     GemmProblem pr;
     std::memset(&pr, 0, sizeof pr);
     pr.p = base_params(s.n, s.d_in, K, bn, ms);
-    COLA_MAP(map_kmajor(&pr.map_a, dZ, K, s.n, ldz, BM * ms));
+    COLA_MAP(map_kmajor(&pr.map_a, dZ, K, s.n, ldz, a_box_rows(ms)));
     COLA_MAP(map_mnmajor(&pr.map_b, A, s.d_in, K, s.ld_a));
     COLA_MAP(map_box32(&pr.map_d, dX, s.d_in, s.n, s.ld_x));
     pr.map_d2 = pr.map_z = pr.map_d;

@@ -8,6 +8,16 @@
 // swizzled shared memory and consumed by tcgen05.mma directly, so no
 // operand is ever transposed in memory.
 //
+// CTA pairs (PAIR = true): two CTAs of a cluster run one 256-row tile with
+// tcgen05 cta_group::2.  Each CTA loads its own 128 rows of A and half of the
+// tile's B columns; the even CTA issues M = 256 MMAs that read both CTAs'
+// shared memory and accumulate each CTA's 128 rows in that CTA's TMEM.  The
+// per-CTA B traffic (TMA fills and MMA operand reads) halves, which relieves
+// the shared-memory bandwidth that bounds a single-CTA M = 128 GEMM.  Both
+// CTAs' TMA loads count on the even CTA's stage barrier; its MMA commits
+// arrive on the stage and accumulator barriers of both CTAs; the odd CTA's
+// epilogue arrives on the even CTA's accumulator-free barrier.
+//
 // Warp roles (320 threads, one CTA per SM, persistent over output tiles):
 //   warp 0      TMA producer: fills a STAGES-deep ring of (A, B) k-blocks.
 //   warp 1      MMA issuer:  tcgen05.mma M=128, N=BN, K=16 into one of two
@@ -92,15 +102,18 @@ constexpr int EPI_SMEM_BYTES = NUM_EPI_WARPS * EPI_WARP_BYTES;
 // A CTA tile is MSUB x 128 rows by BN columns: MSUB = 2 runs two M = 128
 // MMAs per k-step that share one B tile (halving the B-operand traffic per
 // output row), into two TMEM accumulators of BN columns each.
-template <int BN, int MSUB>
+template <int BN, int MSUB, bool PAIR = false>
 struct GemmCfg {
     static_assert(BN % 64 == 0 && BN >= 64 && BN <= 256, "BN must be 64..256 in steps of 64");
     static_assert(MSUB == 1 || MSUB == 2, "one or two 128-row sub-tiles");
-    static constexpr int TILE_M = BM * MSUB;
+    static_assert(!PAIR || (MSUB == 1 && BN >= 128), "a CTA pair runs 128 rows and BN / 2 >= 64 B columns per CTA");
+    static constexpr int TILE_M = PAIR ? 2 * BM : BM * MSUB;   // rows of one unit
+    static constexpr int CTA_ROWS = PAIR ? BM : TILE_M;          // rows of A this CTA loads
+    static constexpr int B_ROWS = PAIR ? BN / 2 : BN;           // columns of B this CTA loads
     static constexpr int ACC_COLS = MSUB * BN;   // TMEM columns of one tile's accumulator
     static_assert(2 * ACC_COLS <= 512, "double-buffered accumulator must fit TMEM");
-    static constexpr int A_BYTES = TILE_M * BK * 2;
-    static constexpr int B_BYTES = BN * BK * 2;
+    static constexpr int A_BYTES = CTA_ROWS * BK * 2;
+    static constexpr int B_BYTES = B_ROWS * BK * 2;
     static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
     static constexpr int BAR_BYTES = 256;
     static constexpr int SMEM_LIMIT = 232448;   // opt-in maximum per CTA
@@ -167,12 +180,21 @@ struct WaitCtx {
     unsigned int* status;
 };
 
+template <bool CLUSTER = false>
+__device__ __forceinline__ bool try_wait_scoped(uint64_t* bar, uint32_t parity)
+{
+    return CLUSTER ? mbar_try_wait_cluster(bar, parity) : mbar_try_wait(bar, parity);
+}
+
+// CLUSTER: the barrier receives arrivals from the peer CTA of a pair
+// (acquire at cluster scope).
+template <bool CLUSTER = false>
 __device__ __forceinline__ bool wait_bounded(uint64_t* bar, uint32_t parity, const WaitCtx& w, unsigned int code)
 {
-    if (mbar_try_wait(bar, parity)) return true;
+    if (try_wait_scoped<CLUSTER>(bar, parity)) return true;
     const uint64_t t0 = global_timer_ns();
     while (true) {
-        if (mbar_try_wait(bar, parity)) return true;
+        if (try_wait_scoped<CLUSTER>(bar, parity)) return true;
         if (*w.abort_flag) return false;
         if (global_timer_ns() - t0 > WAIT_LIMIT_NS) {
             *w.abort_flag = 1;
@@ -262,11 +284,11 @@ __device__ __forceinline__ void stage_row(uint32_t box, int lane, const uint32_t
 }
 
 // ------------------------------------------------------------ the kernel
-template <int BN, int MSUB, bool A_MN, bool B_MN, int EPI>
+template <int BN, int MSUB, bool A_MN, bool B_MN, int EPI, bool PAIR = false>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
     gemm_kernel(const __grid_constant__ GemmBatch batch)
 {
-    using C = GemmCfg<BN, MSUB>;
+    using C = GemmCfg<BN, MSUB, PAIR>;
     constexpr int STAGES = C::STAGES;
     constexpr int TILE_M = C::TILE_M;
     extern __shared__ uint8_t smem_raw[];
@@ -288,6 +310,11 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     const int lane = threadIdx.x & 31;
     unsigned int* const status = batch.prob[0].p.status;
     const WaitCtx wc{abort_flag, status};
+    // units: one per CTA, or one per CTA pair (both CTAs of a pair take the same units)
+    const uint32_t rank = PAIR ? cluster_ctarank() : 0u;
+    const bool leader = rank == 0;
+    const int first_unit = PAIR ? static_cast<int>(blockIdx.x >> 1) : static_cast<int>(blockIdx.x);
+    const int unit_step = PAIR ? static_cast<int>(gridDim.x >> 1) : static_cast<int>(gridDim.x);
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < STAGES; ++s) {
@@ -296,7 +323,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(&tfull_bar[b], 1);
-            mbar_init(&tempty_bar[b], NUM_EPI_WARPS * 32);
+            mbar_init(&tempty_bar[b], NUM_EPI_WARPS * 32 * (PAIR ? 2 : 1));   // PAIR: both CTAs' epilogues
         }
         mbar_init(drain_bar, 1);
         for (int j = 0; j < 2 * NUM_EPI_WARPS; ++j) mbar_init(&zfull_bar[j], 1);
@@ -310,11 +337,19 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         }
     }
     if (warp == 1) {
-        tmem_alloc(tmem_slot, C::TMEM_COLS);
-        tmem_relinquish();
+        if (PAIR) {
+            tmem_alloc_pair(tmem_slot, C::TMEM_COLS);
+            tmem_relinquish_pair();
+        } else {
+            tmem_alloc(tmem_slot, C::TMEM_COLS);
+            tmem_relinquish();
+        }
     }
     tc_fence_before();
-    __syncthreads();
+    if (PAIR)
+        cluster_sync();   // both CTAs' barriers initialised before any cross-CTA arrive
+    else
+        __syncthreads();
     tc_fence_after();
     const uint32_t tmem_base = *tmem_slot;
     // The prologue above overlaps the previous kernel's tail; global memory is
@@ -329,11 +364,13 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             uint32_t phase = 0;
             long long issued = 0;
             bool ok = true;
-            for (int u = blockIdx.x; u < batch.units && ok; u += gridDim.x) {
+            for (int u = first_unit; u < batch.units && ok; u += unit_step) {
                 const Unit x = decode(batch, u);
                 const CUtensorMap* map_a = &batch.prob[x.g].map_a;
                 const CUtensorMap* map_b = &batch.prob[x.g].map_b;
-                const int m0 = x.m_blk * TILE_M, n0 = x.n_blk * BN;
+                // this CTA's rows of A and columns of B
+                const int m0 = x.m_blk * TILE_M + static_cast<int>(rank) * C::CTA_ROWS;
+                const int n0 = x.n_blk * BN + static_cast<int>(rank) * C::B_ROWS;
                 for (int kb = x.kb0; kb < x.kb1; ++kb) {
                     if (!wait_bounded(&empty_bar[stage], phase ^ 1u, wc, ST_TIMEOUT_PRODUCER)) {
                         ok = false;
@@ -341,21 +378,41 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                     }
                     uint8_t* sa = smem_a + stage * C::A_BYTES;
                     uint8_t* sb = smem_b + stage * C::B_BYTES;
-                    mbar_arrive_expect_tx(&full_bar[stage], C::STAGE_BYTES);
                     const int k0 = kb * BK;
-                    if (A_MN) {                 // 64-row boxes along M
+                    if (PAIR) {
+                        // both CTAs' boxes count on the even CTA's stage barrier
+                        const uint32_t fb = mapa_shared(smem_u32(&full_bar[stage]), 0);
+                        if (leader) mbar_arrive_expect_tx(&full_bar[stage], 2 * C::STAGE_BYTES);
+                        if (A_MN) {
 #pragma unroll
-                        for (int j = 0; j < TILE_M / 64; ++j)
-                            tma_load_2d(map_a, &full_bar[stage], sa + j * 64 * BK * 2, m0 + 64 * j, k0);
-                    } else {                    // one box of TILE_M rows
-                        tma_load_2d(map_a, &full_bar[stage], sa, k0, m0);
-                    }
-                    if (B_MN) {
+                            for (int j = 0; j < C::CTA_ROWS / 64; ++j)
+                                tma_load_2d_pair(map_a, fb, sa + j * 64 * BK * 2, m0 + 64 * j, k0);
+                        } else {
+                            tma_load_2d_pair(map_a, fb, sa, k0, m0);
+                        }
+                        if (B_MN) {
 #pragma unroll
-                        for (int j = 0; j < BN / 64; ++j)
-                            tma_load_2d(map_b, &full_bar[stage], sb + j * 64 * BK * 2, n0 + 64 * j, k0);
+                            for (int j = 0; j < C::B_ROWS / 64; ++j)
+                                tma_load_2d_pair(map_b, fb, sb + j * 64 * BK * 2, n0 + 64 * j, k0);
+                        } else {
+                            tma_load_2d_pair(map_b, fb, sb, k0, n0);
+                        }
                     } else {
-                        tma_load_2d(map_b, &full_bar[stage], sb, k0, n0);
+                        mbar_arrive_expect_tx(&full_bar[stage], C::STAGE_BYTES);
+                        if (A_MN) {                 // 64-row boxes along M
+#pragma unroll
+                            for (int j = 0; j < TILE_M / 64; ++j)
+                                tma_load_2d(map_a, &full_bar[stage], sa + j * 64 * BK * 2, m0 + 64 * j, k0);
+                        } else {                    // one box of TILE_M rows
+                            tma_load_2d(map_a, &full_bar[stage], sa, k0, m0);
+                        }
+                        if (B_MN) {
+#pragma unroll
+                            for (int j = 0; j < BN / 64; ++j)
+                                tma_load_2d(map_b, &full_bar[stage], sb + j * 64 * BK * 2, n0 + 64 * j, k0);
+                        } else {
+                            tma_load_2d(map_b, &full_bar[stage], sb, k0, n0);
+                        }
                     }
                     ++issued;
                     if (++stage == STAGES) {
@@ -375,7 +432,15 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                     }
                 }
             } else {
-                // drain: the last min(issued, STAGES) loads may still be landing
+                // drain: the last min(issued, STAGES) loads may still be landing.
+                // The odd CTA of a pair cannot observe its loads (they count on
+                // the even CTA's barriers): it gives them a fixed 50 us.
+                if (PAIR && !leader) {
+                    const uint64_t t0 = global_timer_ns();
+                    while (global_timer_ns() - t0 < 50000ull) {
+                    }
+                    issued = 0;
+                }
                 const int outstanding = issued < STAGES ? static_cast<int>(issued) : STAGES;
                 int s = stage;
                 uint32_t ph = phase;
@@ -396,18 +461,18 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         }
     } else if (warp == 1) {
         // ------------------------------------------------ MMA issuer
-        if (lane == 0) {
-            constexpr uint32_t idesc = idesc_bf16_f32(BM, BN, A_MN ? 1 : 0, B_MN ? 1 : 0);
+        if (lane == 0 && leader) {   // a pair's MMAs are issued by its even CTA alone
+            constexpr uint32_t idesc = idesc_bf16_f32(PAIR ? 2 * BM : BM, BN, A_MN ? 1 : 0, B_MN ? 1 : 0);
             int stage = 0;
             uint32_t phase = 0;
             int buf = 0;
             uint32_t bphase = 0;
             bool ok = true;
             bool issued_any = false;
-            for (int u = blockIdx.x; u < batch.units && ok; u += gridDim.x) {
+            for (int u = first_unit; u < batch.units && ok; u += unit_step) {
                 const Unit x = decode(batch, u);
                 const int kb0 = x.kb0, kb1 = x.kb1;
-                if (!wait_bounded(&tempty_bar[buf], bphase ^ 1u, wc, ST_TIMEOUT_MMA)) {
+                if (!wait_bounded<PAIR>(&tempty_bar[buf], bphase ^ 1u, wc, ST_TIMEOUT_MMA)) {
                     ok = false;
                     break;
                 }
@@ -433,25 +498,39 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                             const uint32_t sas = sa + sub * BM * BK * 2;
                             const uint64_t da = A_MN ? smem_desc_sw128(sas + ks * UMMA_K * 128, 64 * BK * 2, 1024)
                                                      : smem_desc_sw128(sas + ks * UMMA_K * 2, 16, 1024);
-                            umma_f16(d_tmem + sub * BN, da, db, idesc, (kb > kb0 || ks > 0) ? 1u : 0u);
+                            if (PAIR)
+                                umma_f16_pair(d_tmem, da, db, idesc, (kb > kb0 || ks > 0) ? 1u : 0u);
+                            else
+                                umma_f16(d_tmem + sub * BN, da, db, idesc, (kb > kb0 || ks > 0) ? 1u : 0u);
                         }
                     }
                     issued_any = true;
-                    umma_commit(&empty_bar[stage]);   // frees the smem stage once these MMAs are done
+                    // frees the smem stage (of both CTAs of a pair) once these MMAs are done
+                    if (PAIR)
+                        umma_commit_pair(&empty_bar[stage], 0x3);
+                    else
+                        umma_commit(&empty_bar[stage]);
                     if (++stage == STAGES) {
                         stage = 0;
                         phase ^= 1u;
                     }
                 }
                 if (!ok) break;
-                umma_commit(&tfull_bar[buf]);         // accumulator ready for the epilogue
+                // accumulator ready for the epilogue (of both CTAs of a pair)
+                if (PAIR)
+                    umma_commit_pair(&tfull_bar[buf], 0x3);
+                else
+                    umma_commit(&tfull_bar[buf]);
                 if (++buf == 2) {
                     buf = 0;
                     bphase ^= 1u;
                 }
             }
             if ((!ok || *abort_flag) && issued_any) {
-                umma_commit(drain_bar);
+                if (PAIR)
+                    umma_commit_pair(drain_bar, 0x1);
+                else
+                    umma_commit(drain_bar);
                 const uint64_t t0 = global_timer_ns();
                 while (!mbar_try_wait(drain_bar, 0)) {
                     if (global_timer_ns() - t0 > WAIT_LIMIT_NS) {
@@ -470,7 +549,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         const int sub = (MSUB == 2) ? half : 0;
         const int c_first = (MSUB == 2) ? 0 : half;
         constexpr int C_STEP = (MSUB == 2) ? 1 : 2;
-        const int row_in_tile = sub * BM + q * 32 + lane;
+        const int row_off = PAIR ? static_cast<int>(rank) * BM : 0;   // this CTA's rows of a pair's tile
+        const int row_in_tile = row_off + sub * BM + q * 32 + lane;
         uint8_t* ep_gen = smem_epi + (warp - 2) * EPI_WARP_BYTES;
         const uint32_t ep = smem_u32(ep_gen);
         uint64_t* zbar = zfull_bar + 2 * (warp - 2);
@@ -484,7 +564,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             const Unit x = decode(batch, u);
             const GemmParams& pu = batch.prob[x.g].p;
             if (EPI == EPI_F32) return BN / 32;
-            if (x.m_blk * TILE_M + sub * BM + q * 32 >= pu.M) return 0;   // this warp's 32 rows are all past the end
+            if (x.m_blk * TILE_M + row_off + sub * BM + q * 32 >= pu.M) return 0;   // this warp's 32 rows are all past the end
             const int left = pu.N - x.n_blk * BN;
             return left >= BN ? BN / 32 : (left + 31) / 32;
         };
@@ -511,12 +591,12 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         };
 
         // EPI_DSIGMA: Z boxes run one (tile, chunk) item ahead of their use
-        int zu = blockIdx.x, zc = c_first;      // next item whose Z box is to be loaded
+        int zu = first_unit, zc = c_first;      // next item whose Z box is to be loaded
         uint32_t zphase = 0;                    // bit b: parity of the next wait on zbar[b]
         int zload = 0, zuse = 0;
         auto z_advance = [&]() {                // move (zu, zc) to the next item that has a chunk
             while (zu < batch.units && zc >= chunk_count(zu)) {
-                zu += gridDim.x;
+                zu += unit_step;
                 zc = c_first;
             }
         };
@@ -528,7 +608,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                 bulk_wait_group_read<0>();      // the stores that last read box b are done with it
                 mbar_arrive_expect_tx(&zbar[b], EPI_BOX_BYTES);
                 tma_load_2d(&batch.prob[x.g].map_z, &zbar[b], ep_gen + b * EPI_BOX_BYTES, x.n_blk * BN + zc * 32,
-                            x.m_blk * TILE_M + sub * BM + q * 32);
+                            x.m_blk * TILE_M + row_off + sub * BM + q * 32);
             }
             ++zload;
             zc += C_STEP;
@@ -539,14 +619,14 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             z_issue();
         }
 
-        for (int u = blockIdx.x; u < batch.units && ok; u += gridDim.x) {
+        for (int u = first_unit; u < batch.units && ok; u += unit_step) {
             const Unit x = decode(batch, u);
             const GemmParams& p = batch.prob[x.g].p;
             const CUtensorMap* map_d = &batch.prob[x.g].map_d;
             const CUtensorMap* map_d2 = &batch.prob[x.g].map_d2;
             const int m_blk = x.m_blk, n_blk = x.n_blk, split = x.split;
             cur_M = p.M;
-            const int row0 = m_blk * TILE_M + sub * BM + q * 32;
+            const int row0 = m_blk * TILE_M + row_off + sub * BM + q * 32;
             const int row = row0 + lane;
             const int nch = chunk_count(u);
             if (!wait_bounded(&tfull_bar[buf], bphase, wc, ST_TIMEOUT_EPILOGUE)) break;
@@ -647,7 +727,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                 }
             }
             tc_fence_before();
-            mbar_arrive(&tempty_bar[buf]);
+            if (PAIR)   // the even CTA's barrier collects both CTAs' epilogues
+                mbar_arrive_cluster(mapa_shared(smem_u32(&tempty_bar[buf]), 0));
+            else
+                mbar_arrive(&tempty_bar[buf]);
             if (++buf == 2) {
                 buf = 0;
                 bphase ^= 1u;
@@ -670,10 +753,16 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     }
 
     tc_fence_before();
-    __syncthreads();
+    if (PAIR)
+        cluster_sync();   // neither CTA leaves while the pair's MMAs may still read its shared memory
+    else
+        __syncthreads();
     if (warp == 1) {
         tc_fence_after();
-        tmem_dealloc(tmem_base, C::TMEM_COLS);
+        if (PAIR)
+            tmem_dealloc_pair(tmem_base, C::TMEM_COLS);
+        else
+            tmem_dealloc(tmem_base, C::TMEM_COLS);
     }
 }
 

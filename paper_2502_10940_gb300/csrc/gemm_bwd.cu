@@ -8,7 +8,9 @@ namespace cola {
 template cudaError_t launch_gemm<128, 1, false, true, EPI_DSIGMA>(const GemmBatch&, int, bool, cudaStream_t);
 template cudaError_t launch_gemm<256, 1, false, true, EPI_DSIGMA>(const GemmBatch&, int, bool, cudaStream_t);
 template cudaError_t launch_gemm<128, 2, false, true, EPI_DSIGMA>(const GemmBatch&, int, bool, cudaStream_t);
+template cudaError_t launch_gemm<256, 1, false, true, EPI_DSIGMA, true>(const GemmBatch&, int, bool, cudaStream_t);
 template cudaError_t launch_gemm<128, 1, false, true, EPI_STORE>(const GemmBatch&, int, bool, cudaStream_t);
 template cudaError_t launch_gemm<256, 1, false, true, EPI_STORE>(const GemmBatch&, int, bool, cudaStream_t);
 template cudaError_t launch_gemm<128, 2, false, true, EPI_STORE>(const GemmBatch&, int, bool, cudaStream_t);
+template cudaError_t launch_gemm<256, 1, false, true, EPI_STORE, true>(const GemmBatch&, int, bool, cudaStream_t);
 }  // namespace cola

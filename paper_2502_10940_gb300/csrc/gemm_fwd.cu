@@ -8,9 +8,11 @@ namespace cola {
 template cudaError_t launch_gemm<128, 1, false, false, EPI_ZH>(const GemmBatch&, int, bool, cudaStream_t);
 template cudaError_t launch_gemm<256, 1, false, false, EPI_ZH>(const GemmBatch&, int, bool, cudaStream_t);
 template cudaError_t launch_gemm<128, 2, false, false, EPI_ZH>(const GemmBatch&, int, bool, cudaStream_t);
+template cudaError_t launch_gemm<256, 1, false, false, EPI_ZH, true>(const GemmBatch&, int, bool, cudaStream_t);
 template cudaError_t launch_gemm<128, 1, false, false, EPI_STORE>(const GemmBatch&, int, bool, cudaStream_t);
 template cudaError_t launch_gemm<256, 1, false, false, EPI_STORE>(const GemmBatch&, int, bool, cudaStream_t);
 template cudaError_t launch_gemm<128, 2, false, false, EPI_STORE>(const GemmBatch&, int, bool, cudaStream_t);
+template cudaError_t launch_gemm<256, 1, false, false, EPI_STORE, true>(const GemmBatch&, int, bool, cudaStream_t);
 
 // H = bf16(sigma(Z)) over `vecs` groups of 8 bf16, each a 16-byte vector;
 // sigma is evaluated exactly as in the Z/H epilogue (same function on the

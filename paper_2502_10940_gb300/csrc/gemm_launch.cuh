@@ -10,8 +10,9 @@ namespace cola {
 
 // Launch the GEMM kernel over a batch of problems (see GemmBatch).  pdl:
 // launch with programmatic stream serialization (the prologue overlaps the
-// previous kernel's tail).
-template <int BN, int MSUB, bool A_MN, bool B_MN, int EPI>
+// previous kernel's tail).  PAIR: clusters of two CTAs (grid even), each
+// pair running one 256-row tile with tcgen05 cta_group::2.
+template <int BN, int MSUB, bool A_MN, bool B_MN, int EPI, bool PAIR = false>
 cudaError_t launch_gemm(const GemmBatch& batch, int grid, bool pdl, cudaStream_t stream);
 
 // One fixed-order reduction of fp32 split partials into a gradient.
@@ -39,11 +40,11 @@ cudaError_t launch_splitk_reduce(ReduceBatch& batch, cudaStream_t stream);
 cudaError_t launch_sigma(const void* Z, void* H, long long elems, int sigma, int sms, cudaStream_t stream);
 
 #ifdef COLA_DEFINE_LAUNCHERS
-template <int BN, int MSUB, bool A_MN, bool B_MN, int EPI>
+template <int BN, int MSUB, bool A_MN, bool B_MN, int EPI, bool PAIR>
 cudaError_t launch_gemm(const GemmBatch& batch, int grid, bool pdl, cudaStream_t stream)
 {
-    constexpr int smem = GemmCfg<BN, MSUB>::SMEM_BYTES;
-    auto kern = gemm_kernel<BN, MSUB, A_MN, B_MN, EPI>;
+    constexpr int smem = GemmCfg<BN, MSUB, PAIR>::SMEM_BYTES;
+    auto kern = gemm_kernel<BN, MSUB, A_MN, B_MN, EPI, PAIR>;
     // the opt-in shared-memory size is a per-device function attribute
     static unsigned long long configured = 0;   // bit d: set on device d
     int dev = 0;
@@ -59,11 +60,18 @@ cudaError_t launch_gemm(const GemmBatch& batch, int grid, bool pdl, cudaStream_t
     cfg.blockDim = dim3(NUM_THREADS);
     cfg.dynamicSmemBytes = smem;
     cfg.stream = stream;
-    cudaLaunchAttribute attr[1];
+    cudaLaunchAttribute attr[2];
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
     attr[0].val.programmaticStreamSerializationAllowed = pdl ? 1 : 0;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
+    if (PAIR) {
+        attr[1].id = cudaLaunchAttributeClusterDimension;
+        attr[1].val.clusterDim.x = 2;
+        attr[1].val.clusterDim.y = 1;
+        attr[1].val.clusterDim.z = 1;
+        cfg.numAttrs = 2;
+    }
     return cudaLaunchKernelEx(&cfg, kern, batch);
 }
 #endif

@@ -83,9 +83,11 @@ __global__ void __launch_bounds__(RED_GROUPS * RED_WAYS) splitk_reduce_kernel(co
 template cudaError_t launch_gemm<128, 1, true, true, EPI_STORE>(const GemmBatch&, int, bool, cudaStream_t);
 template cudaError_t launch_gemm<256, 1, true, true, EPI_STORE>(const GemmBatch&, int, bool, cudaStream_t);
 template cudaError_t launch_gemm<128, 2, true, true, EPI_STORE>(const GemmBatch&, int, bool, cudaStream_t);
+template cudaError_t launch_gemm<256, 1, true, true, EPI_STORE, true>(const GemmBatch&, int, bool, cudaStream_t);
 template cudaError_t launch_gemm<128, 1, true, true, EPI_F32>(const GemmBatch&, int, bool, cudaStream_t);
 template cudaError_t launch_gemm<256, 1, true, true, EPI_F32>(const GemmBatch&, int, bool, cudaStream_t);
 template cudaError_t launch_gemm<128, 2, true, true, EPI_F32>(const GemmBatch&, int, bool, cudaStream_t);
+template cudaError_t launch_gemm<256, 1, true, true, EPI_F32, true>(const GemmBatch&, int, bool, cudaStream_t);
 
 cudaError_t launch_splitk_reduce(ReduceBatch& rb, cudaStream_t stream)
 {

@@ -72,23 +72,49 @@ bool map_mnmajor(CUtensorMap* m, const void* base, int64_t mn_extent, int64_t k_
 }
 
 // ------------------------------------------------------------ planning
-int choose_bn(int64_t N)
+// Column tile: the width that pads N least; a compute-heavy GEMM (see
+// heavy_gemm) takes 256 whenever that pads N by at most 5 %, because only
+// 256-column tiles run on CTA pairs.
+int choose_bn(int64_t N, bool heavy = false)
 {
     if (N <= 128) return 128;
     const int64_t pad256 = (N + 255) / 256 * 256;
     const int64_t pad128 = (N + 127) / 128 * 128;
+    if (heavy && N >= 1024 && pad256 * 100 <= N * 105) return 256;
     return pad256 <= pad128 ? 256 : 128;
 }
 
-// Rows per CTA tile: two 128-row sub-tiles sharing each B tile when the
-// accumulator fits TMEM twice over (BN = 128), M spans more than one and the
-// launch is compute-heavy (>= 64 GFLOP).  Measured: it lifts the tensor-bound
-// 1B/7B blocks by 4-6 % but slows the HBM-bound 60M block, whose short GEMMs
-// are limited by the epilogue, which a taller tile makes longer.
-int choose_msub(int64_t M, int64_t N, int64_t K, int bn)
+// >= 64 GFLOP over more than one 128-row block: tensor-bound at every rank
+// the workloads use.
+bool heavy_gemm(int64_t M, int64_t N, int64_t K)
 {
     const double flops = 2.0 * static_cast<double>(M) * static_cast<double>(N) * static_cast<double>(K);
-    return (bn == 128 && M > BM && flops >= 64e9) ? 2 : 1;
+    return M > 128 && flops >= 64e9;
+}
+
+int choose_bn_for(int64_t M, int64_t N, int64_t K) { return choose_bn(N, heavy_gemm(M, N, K)); }
+
+// Tile modes ("msub" below): 1 = one CTA runs a 128-row tile; 2 = one CTA
+// runs two 128-row sub-tiles sharing each B tile; TILE_PAIR = a CTA pair runs
+// a 256-row tile with tcgen05 cta_group::2 (each CTA loads half of B).
+constexpr int TILE_PAIR = 3;
+
+int tile_rows(int msub) { return msub == 1 ? BM : 2 * BM; }        // rows of one unit
+int a_box_rows(int msub) { return msub == TILE_PAIR ? BM : BM * msub; }   // rows of A one CTA loads
+int b_box_rows(int bn, int msub) { return msub == TILE_PAIR ? bn / 2 : bn; }   // K-major B rows one CTA loads
+int unit_slots(int msub, int sms) { return msub == TILE_PAIR ? sms / 2 : sms; }   // units in flight
+
+// Compute-heavy GEMMs with 256-column tiles run on CTA pairs: halving each
+// CTA's B traffic relieves the shared-memory bandwidth that a single CTA's
+// M = 128 MMAs, its TMA fills and its epilogue stores saturate (measured:
+// -10 to -25 % per GEMM on the 1B layers).  With 128-column tiles a pair was
+// slower than one CTA running two 128-row sub-tiles (+12 to +23 %), which
+// they keep.  The HBM-bound short GEMMs keep single-CTA 128-row tiles (a
+// taller tile lengthens the epilogue they are limited by).
+int choose_msub(int64_t M, int64_t N, int64_t K, int bn)
+{
+    if (!heavy_gemm(M, N, K)) return 1;
+    return bn == 256 ? TILE_PAIR : 2;
 }
 
 // Tile grid of one GEMM, without a token split.
@@ -99,7 +125,7 @@ GemmParams base_params(int64_t M, int64_t N, int64_t K, int bn, int msub)
     p.M = static_cast<int>(M);
     p.N = static_cast<int>(N);
     p.k_blocks = static_cast<int>((K + BK - 1) / BK);
-    p.m_tiles = static_cast<int>((M + BM * msub - 1) / (BM * msub));
+    p.m_tiles = static_cast<int>((M + tile_rows(msub) - 1) / tile_rows(msub));
     p.n_tiles = static_cast<int>((N + bn - 1) / bn);
     p.kb_per_split = p.k_blocks;
     p.splits = 1;
@@ -110,12 +136,14 @@ GemmParams base_params(int64_t M, int64_t N, int64_t K, int bn, int msub)
 // Token split of weight-gradient GEMMs sharing one launch (same K): minimise
 // (waves of persistent CTAs) x (k-blocks per unit + the cost of writing and
 // re-reading its fp32 partial tile, counted in k-blocks of operand bytes:
-// 8 BN msub / (128 msub + BN), plus 2 for the reduction pass), with at least
+// 8 BN rows / (128 (rows + BN)), plus 2 for the reduction pass), with at least
 // 4 k-blocks per split.
 int choose_splits(int tiles, int k_blocks, int bn, int msub, int sms)
 {
     const int max_s = k_blocks / 4 > 1 ? k_blocks / 4 : 1;
-    const double c_part = 8.0 * bn * msub / (128.0 * msub + bn) + 2.0;
+    const int rows = tile_rows(msub);
+    const double c_part = 8.0 * bn * rows / (128.0 * (rows + bn)) + 2.0;
+    sms = unit_slots(msub, sms);
     double best = -1.0;
     int S = 1;
     for (int s = 1; s <= max_s; ++s) {
@@ -140,7 +168,7 @@ void set_splits(GemmParams& p, int S)
 
 int64_t partial_elems(const GemmParams& p, int bn, int msub)
 {
-    return static_cast<int64_t>(p.m_tiles) * BM * msub * p.n_tiles * bn;
+    return static_cast<int64_t>(p.m_tiles) * tile_rows(msub) * p.n_tiles * bn;
 }
 
 // Weight-gradient group plan: count GEMMs D_i[M_i x N_i] = sum over the same
@@ -158,11 +186,14 @@ WgradPlan plan_wgrad(const int64_t* M, const int64_t* N, int count, int64_t ntok
     std::memset(&w, 0, sizeof w);
     w.count = count;
     w.bn = 256;
-    for (int i = 0; i < count; ++i) w.bn = choose_bn(N[i]) < w.bn ? choose_bn(N[i]) : w.bn;
-    w.msub = 2;
+    for (int i = 0; i < count; ++i) {
+        const int b = choose_bn_for(M[i], N[i], ntok);
+        w.bn = b < w.bn ? b : w.bn;
+    }
+    w.msub = TILE_PAIR;   // the smallest tile any GEMM of the group would take
     for (int i = 0; i < count; ++i) {
         const int ms = choose_msub(M[i], N[i], ntok, w.bn);
-        w.msub = ms < w.msub ? ms : w.msub;
+        if (ms == 1 || (ms == 2 && w.msub == TILE_PAIR)) w.msub = ms;
     }
     int tiles = 0;
     for (int i = 0; i < count; ++i) {
@@ -195,10 +226,15 @@ cudaError_t dispatch(int bn, int msub, GemmBatch& b, int sms, cudaStream_t s)
         flops += 2.0 * b.prob[g].p.M * b.prob[g].p.N * (static_cast<double>(b.prob[g].p.k_blocks) * BK);
     }
     b.units = units;
-    const int grid = units < sms ? units : sms;
     const bool pdl = flops < 64e9;
+    if (msub == TILE_PAIR && bn == 256) {
+        const int pairs = units < sms / 2 ? units : sms / 2;
+        return launch_gemm<256, 1, A_MN, B_MN, EPI, true>(b, 2 * pairs, pdl, s);
+    }
+    if (msub != 1 && bn == 256) return cudaErrorInvalidValue;   // planned tiles exist as above only
+    const int grid = units < sms ? units : sms;
     if (bn == 256) return launch_gemm<256, 1, A_MN, B_MN, EPI>(b, grid, pdl, s);
-    if (msub == 2) return launch_gemm<128, 2, A_MN, B_MN, EPI>(b, grid, pdl, s);
+    if (msub != 1) return launch_gemm<128, 2, A_MN, B_MN, EPI>(b, grid, pdl, s);
     return launch_gemm<128, 1, A_MN, B_MN, EPI>(b, grid, pdl, s);
 }
 
