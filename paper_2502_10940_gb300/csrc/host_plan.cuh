@@ -104,17 +104,20 @@ int a_box_rows(int msub) { return msub == TILE_PAIR ? BM : BM * msub; }   // row
 int b_box_rows(int bn, int msub) { return msub == TILE_PAIR ? bn / 2 : bn; }   // K-major B rows one CTA loads
 int unit_slots(int msub, int sms) { return msub == TILE_PAIR ? sms / 2 : sms; }   // units in flight
 
-// Compute-heavy GEMMs with 256-column tiles run on CTA pairs: halving each
-// CTA's B traffic relieves the shared-memory bandwidth that a single CTA's
-// M = 128 MMAs, its TMA fills and its epilogue stores saturate (measured:
-// -10 to -25 % per GEMM on the 1B layers).  With 128-column tiles a pair was
-// slower than one CTA running two 128-row sub-tiles (+12 to +23 %), which
-// they keep.  The HBM-bound short GEMMs keep single-CTA 128-row tiles (a
-// taller tile lengthens the epilogue they are limited by).
+// Compute-heavy GEMMs with 256-column tiles and K >= 512 run on CTA pairs:
+// halving each CTA's B traffic relieves the shared-memory bandwidth that a
+// single CTA's M = 128 MMAs, its TMA fills and its epilogue stores saturate
+// (measured: -5 to -25 % per GEMM on the 1B layers, K = 512 to 65536).  With
+// K = 256 (4 k-blocks per tile, the store-bound Y and dX GEMMs at rank 256)
+// a pair was 20-40 % slower, and with 128-column tiles slower than one CTA
+// running two 128-row sub-tiles (+12 to +23 %), which those keep.  The
+// HBM-bound short GEMMs keep single-CTA 128-row tiles (a taller tile
+// lengthens the epilogue they are limited by).
 int choose_msub(int64_t M, int64_t N, int64_t K, int bn)
 {
     if (!heavy_gemm(M, N, K)) return 1;
-    return bn == 256 ? TILE_PAIR : 2;
+    if (bn == 256) return K >= 512 ? TILE_PAIR : 1;
+    return 2;
 }
 
 // Tile grid of one GEMM, without a token split.
