@@ -99,6 +99,8 @@ WORKLOADS = {
     "7b": Workload("7b", 32768, llama_block(4096, 11008, 1024), modes=("cola_m", "cola"),
                    desc="LLaMA-7B-shaped CoLA block, d=4096, d_ff=11008, r=1024, 32768 tokens "
                         "(128 x 256)", seqs=128),
+    "1b-o": Workload("1b-o", 65536, (Layer("o", 2048, 2048, 512, "x_o"),), fused_qkv=False,
+                     desc="single CoLA layer, LLaMA-1B o-proj shape, 65536 tokens, 2048->2048, r=512", seqs=256),
     # inference at the pre-training shapes with 32 sequences of 256 tokens (Table 10)
     "1b-infer": Workload("1b-infer", 8192, llama_block(2048, 5461, 512), modes=("infer",), phase="infer",
                          graph=True, desc="LLaMA-1B-shaped CoLA block, forward only (inference), d=2048, "
