@@ -84,12 +84,17 @@ int choose_bn(int64_t N, bool heavy = false)
     return pad256 <= pad128 ? 256 : 128;
 }
 
-// >= 64 GFLOP over more than one 128-row block: tensor-bound at every rank
-// the workloads use.
+// Compute-heavy: more than one 128-row block and either >= 64 GFLOP, or
+// >= 16 GFLOP at an arithmetic intensity (each operand read once, the
+// result written once) of >= 300 FLOP/B, above the ridge of the GB300 bf16
+// roofline (~287).  The second clause takes the tensor-bound GEMMs of the
+// 8192-token inference workloads (measured: 1B forward -14 %).
 bool heavy_gemm(int64_t M, int64_t N, int64_t K)
 {
-    const double flops = 2.0 * static_cast<double>(M) * static_cast<double>(N) * static_cast<double>(K);
-    return M > 128 && flops >= 64e9;
+    const double m = static_cast<double>(M), n = static_cast<double>(N), k = static_cast<double>(K);
+    const double flops = 2.0 * m * n * k;
+    const double bytes = 2.0 * (m * k + n * k + m * n);
+    return M > 128 && (flops >= 64e9 || (flops >= 16e9 && flops / bytes >= 300.0));
 }
 
 int choose_bn_for(int64_t M, int64_t N, int64_t K) { return choose_bn(N, heavy_gemm(M, N, K)); }
