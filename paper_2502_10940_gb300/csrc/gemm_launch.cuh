@@ -23,7 +23,7 @@ struct ReduceJob {
     int M, N;
     void* out;                  // bf16 (or fp32 when accumulating)
     long long ldo;
-    long long block_begin;      // first block of this job in the launch
+    long long group_begin;      // first 4-column group of this job in the launch (set by the launcher)
 };
 
 struct ReduceBatch {
@@ -31,6 +31,7 @@ struct ReduceBatch {
     int count;
     int splits;
     int accumulate_f32;
+    long long groups;           // 4-column groups of all jobs (set by the launcher)
 };
 
 cudaError_t launch_splitk_reduce(ReduceBatch& batch, cudaStream_t stream);
