@@ -5,8 +5,9 @@ Y and dX (row-local), random entries of dA and dB (each a full reduction
 over all n tokens).
 
 The shapes exercise the tile configurations the production workloads select
-and the small parity cases do not reach: the two-sub-tile (256-row) CTA tiles
-of compute-heavy launches in every epilogue, 256-column tiles, ragged widths
+and the small parity cases do not reach: CTA-pair (cta_group::2) tiles of
+compute-heavy launches in every epilogue, including a ragged last pair tile,
+the two-sub-tile (256-row) single-CTA tiles, 256-column tiles, ragged widths
 with padded pitches (5461 -> 5464), and multi-wave token splits.
 """
 import numpy as np
@@ -23,6 +24,9 @@ SHAPES = [
     (65536, 2048, 5461, 512),    # LLaMA-1B gate/up: Y with 5461 columns on 256-row tiles
     (65536, 5461, 2048, 512),    # LLaMA-1B down: K = 5461 forward, dA / dX with 5461 columns
     (32768, 8192, 8192, 128),    # r = 128 at 68.7 GFLOP per GEMM: 256-row tiles for Z/H, dZ and dB
+    # CTA-pair tiles with a ragged last tile (1B widths, tensor-bound at a few thousand tokens):
+    (8320, 2048, 2048, 512),     # the last pair tile's odd CTA holds only rows past the end
+    (8200, 2048, 2048, 512),     # the last pair tile ends inside its even CTA's rows
 ]
 
 
@@ -50,8 +54,9 @@ def test_full_size_layer_sampled(shape):
     Xb, dYb = _full_bits(inp["X"]), _full_bits(inp["dY"])
     Ab, Bb = I.bf16_bits(inp["A"]), I.bf16_bits(inp["B"])
     rng = np.random.default_rng(1234)
-    rows = np.sort(rng.choice(n, 48, replace=False))
-    rows[-1] = n - 1                                    # the last (possibly ragged) tile
+    # random rows plus rows of the last (possibly ragged) 256-row tile
+    tail = [n - 1 - k for k in (0, 1, 63, 64, 127, 128, 200) if n - 1 - k >= 0]
+    rows = np.unique(np.concatenate([rng.choice(n, 44, replace=False), tail]))
     Z, H, Y, dZ, dX = oracle.rows_bf16(Xb, Ab, Bb, rows, dYb, "silu", d_in=d_in, d_out=d_out)
     ridx = torch.from_numpy(rows).cuda()
     assert_close("Z rows", to64(g["Z"][ridx]), Z)
