@@ -480,12 +480,26 @@ def time_steps(fn, steps, stream, dist=None, flush=None):
         total = sum(a.elapsed_time(b) for a, b in ev)
     if dist:
         dist.barrier()
-    ms = total / steps
-    if dist:
-        t = torch.tensor([ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
-    return ms
+    return max_over_ranks(total / steps, dist, "cuda")
+
+
+def max_over_ranks(value, dist=None, device="cpu"):
+    """The largest of the ranks' values (the job's step time is its slowest
+    rank's); the value itself without a process group."""
+    if not dist:
+        return value
+    import torch
+
+    t = torch.tensor([float(value)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def whole_job_tflops(flops_per_rank_step, world, ms_per_step):
+    """Weak scaling: every rank runs the whole workload on its own batch, so
+    the job processes world x the per-rank work in the (max-over-ranks) step
+    time."""
+    return flops_per_rank_step * world / (ms_per_step / 1e3) / 1e12
 
 
 def full_rank_baseline(wl, device, steps, warmup, seed=0, flush=None):
@@ -608,7 +622,7 @@ def run_cola(args, wl):
                                                roofline["algorithmic_bytes_per_launch"])
 
     flops = wl.flops
-    value = flops * world / (ms / 1e3) / 1e12
+    value = whole_job_tflops(flops, world, ms)
     line = {"metric": METRIC if blk.train else METRIC_INFER, "value": round(value, 2), "unit": "TFLOP/s", "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": round(ms, 4), "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
