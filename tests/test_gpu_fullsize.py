@@ -77,3 +77,28 @@ def test_full_size_layer_sampled(shape):
     dB_o = oracle.dB_entries_bf16(Xb, Ab, dYb, oo, jj, "silu")
     dB_g = to64(g["dB"])[oo, jj]
     assert_close("dB entries", dB_g, dB_o)
+
+
+def test_pair_tiles_cola_m_bitwise_and_fp32_accumulate():
+    # On the CTA-pair path (1B widths, ragged last pair tile): CoLA and CoLA-M
+    # give the same gradients bit for bit, and fp32 accumulation adds the same
+    # gradient onto existing values (sampled against the oracle).
+    n, d_in, d_out, r = 8320, 2048, 2048, 512
+    inp = I.layer_inputs(n, d_in, d_out, r, seed=9, device="cuda")
+    a = gpu_layer(inp, "silu", "cola")
+    b = gpu_layer(inp, "silu", "cola_m")
+    for k in ["Y", "Z", "dX", "dA", "dB"]:
+        assert torch.equal(a[k], b[k]), k
+    g0 = torch.Generator(device="cuda").manual_seed(11)
+    dA0 = torch.randn((r, d_in), generator=g0, device="cuda")
+    dB0 = torch.randn((d_out, r), generator=g0, device="cuda")
+    f = gpu_layer(inp, "silu", "cola", wgrad_fp32=True, dA0=dA0, dB0=dB0)
+    Xb, dYb = _full_bits(inp["X"]), _full_bits(inp["dY"])
+    Ab, Bb = I.bf16_bits(inp["A"]), I.bf16_bits(inp["B"])
+    rng = np.random.default_rng(99)
+    ii, kk = rng.integers(0, r, 24), rng.integers(0, d_in, 24)
+    dA_o = oracle.dA_entries_bf16(Xb, Ab, Bb, dYb, ii, kk, "silu", d_out=d_out)
+    assert_close("dA += entries", (to64(f["dA"]) - to64(dA0))[ii, kk], dA_o)
+    oo, jj = rng.integers(0, d_out, 24), rng.integers(0, r, 24)
+    dB_o = oracle.dB_entries_bf16(Xb, Ab, dYb, oo, jj, "silu")
+    assert_close("dB += entries", (to64(f["dB"]) - to64(dB0))[oo, jj], dB_o)
