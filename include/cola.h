@@ -194,8 +194,28 @@ cola_status_t cola_recompute_up(const cola_desc_t* desc, int32_t count, const vo
 /* Synchronise `stream`, read and clear the workspace status word.
  * Returns COLA_OK, or COLA_ERR_DEVICE_TIMEOUT if a kernel that used this
  * workspace gave up on a wait since the last check (*code_out, if not NULL,
- * receives the raw status bits), or COLA_ERR_LAUNCH on a CUDA error. */
+ * receives the raw status bits below), or COLA_ERR_LAUNCH on a CUDA error.
+ * Every wait in the kernels is bounded (2 s of GPU global time); a wait that
+ * runs out raises an abort flag that ends its CTA's other waits, and the
+ * kernel drains its own copies and MMAs (bounded), frees its TMEM and exits,
+ * leaving the results of that launch undefined and the context usable. */
+#define COLA_STATUS_PRODUCER_TIMEOUT 0x1u   /* a TMA producer gave up waiting for a free stage */
+#define COLA_STATUS_MMA_TIMEOUT 0x2u        /* an MMA issuer gave up waiting for operands or TMEM */
+#define COLA_STATUS_EPILOGUE_TIMEOUT 0x4u   /* an epilogue gave up waiting for an accumulator or saved Z */
+#define COLA_STATUS_DRAIN_TIMEOUT 0x8u      /* a CTA gave up waiting for its own copies or MMAs to drain */
 cola_status_t cola_check_status(void* ws, void* stream, uint32_t* code_out);
+
+/* ---- failure detection self-test ----
+ * The paper has no counterpart.  Launches one 128 x 128 x 64 GEMM (operands
+ * and output in ws after its 256-byte status header; ws_bytes >= 256 + 96 KB)
+ * whose TMA producer issues no loads, so that its MMA issuer's first wait
+ * runs out after 2 s: the next cola_check_status on ws then returns
+ * COLA_ERR_DEVICE_TIMEOUT with COLA_STATUS_MMA_TIMEOUT set (and, if the
+ * epilogue's wait for that accumulator ran out first, also
+ * COLA_STATUS_EPILOGUE_TIMEOUT; no other bit).  No copy or MMA
+ * is ever in flight, nothing in ws beyond the status word is touched, and the
+ * CUDA context stays usable.  Async on `stream`. */
+cola_status_t cola_selftest_wait_timeout(void* ws, size_t ws_bytes, void* stream);
 
 /* ---- weight gradient without any workspace or allocation ----
  * The paper has no counterpart to this entry point.  It serves callers that

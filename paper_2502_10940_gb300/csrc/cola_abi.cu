@@ -582,6 +582,37 @@ cola_status_t cola_recompute_up(const cola_desc_t* desc, int32_t count, const vo
     return run_f2(s, count, Hs, R, B, Y, status, sms, st);
 }
 
+static_assert(COLA_STATUS_PRODUCER_TIMEOUT == ST_TIMEOUT_PRODUCER && COLA_STATUS_MMA_TIMEOUT == ST_TIMEOUT_MMA &&
+                  COLA_STATUS_EPILOGUE_TIMEOUT == ST_TIMEOUT_EPILOGUE && COLA_STATUS_DRAIN_TIMEOUT == ST_TIMEOUT_DRAIN,
+              "status bits of the header and the kernels agree");
+
+cola_status_t cola_selftest_wait_timeout(void* ws, size_t ws_bytes, void* stream)
+{
+    if (!ws) return COLA_ERR_INVALID;
+    if (reinterpret_cast<uintptr_t>(ws) & (WS_ALIGN - 1)) return COLA_ERR_ALIGN;
+    constexpr size_t tile_bytes = 128 * 128 * 2;
+    if (ws_bytes < WS_HEADER + 3 * tile_bytes) return COLA_ERR_WORKSPACE;
+    int sms = 0;
+    COLA_TRY(device_info(&sms));
+    // one 128 x 128 x 64 GEMM whose operands and output lie in the workspace;
+    // its producer issues no loads, so nothing is ever read or written there
+    uint8_t* base = wsb(ws) + WS_HEADER;
+    GemmProblem pr;
+    std::memset(&pr, 0, sizeof pr);
+    pr.p = base_params(128, 128, 64, 128, 1);
+    COLA_MAP(map_kmajor(&pr.map_a, base, 64, 128, 64, BM));
+    COLA_MAP(map_kmajor(&pr.map_b, base + tile_bytes, 64, 128, 64, 128));
+    COLA_MAP(map_box32(&pr.map_d, base + 2 * tile_bytes, 128, 128, 128));
+    pr.map_d2 = pr.map_z = pr.map_d;
+    pr.p.d_ptr = reinterpret_cast<__nv_bfloat16*>(base + 2 * tile_bytes);
+    pr.p.d_ld = 128;
+    pr.p.status = ws_status(ws);
+    pr.p.selftest_no_loads = 1;
+    const int64_t mnk[1][3] = {{128, 128, 64}};
+    return run_batch<false, false, EPI_STORE>(COLA_KERNEL_FWD_Y, 128, 1, &pr, mnk, 1, 0, sms,
+                                              static_cast<cudaStream_t>(stream));
+}
+
 cola_status_t cola_check_status(void* ws, void* stream, uint32_t* code_out)
 {
     if (!ws) return COLA_ERR_INVALID;

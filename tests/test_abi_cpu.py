@@ -164,6 +164,13 @@ def test_infer_mode_argument_errors(L):
     assert f(ctypes.byref(dc), FAKE, FAKE, FAKE, FAKE, None, None, FAKE, 1 << 20, None) == 1
 
 
+def test_selftest_argument_errors(L):
+    f = L.lib().cola_selftest_wait_timeout
+    assert f(None, 1 << 20, None) == 1
+    assert f(FAKE + 16, 1 << 20, None) == 2      # not 256-byte aligned
+    assert f(FAKE, 1024, None) == 4              # smaller than the status word plus three tiles
+
+
 def test_workspace_init_and_check_reject_null(L):
     assert L.lib().cola_workspace_init(None, None) == 1
     assert L.lib().cola_workspace_init(FAKE + 16, None) == 2   # not 256-byte aligned
