@@ -417,7 +417,9 @@ def cpu_baseline(wl, target_s=10.0):
     dt, fl = oracle_block_sample(wl, n_s)
     return {"value": round(fl / dt / 1e12, 6), "unit": "TFLOP/s", "cores": oracle.num_threads(), "kind": "oracle",
             "sample": f"{wl.name} block, all {len(wl.layers)} layers {phase_words(wl)} on {n_s} of {wl.n} tokens "
-                      f"({dt:.1f} s, fp64 loops, OpenMP)"}
+                      f"({dt:.1f} s, fp64 loops, OpenMP)",
+            # every token costs the same, so the full step scales with the token count
+            "full_step_s_extrapolated": round(dt * wl.n / n_s, 2)}
 
 
 # ---------------------------------------------------------------- arms
@@ -679,6 +681,26 @@ def run_cola(args, wl):
             fr = full_rank_baseline(wl, device, max(3, args.steps // 2), 3, seed=args.seed, flush=flush)
             fr["speedup_cola_vs_full_rank"] = round(fr["ms_per_step"] / ms, 3)
             line["full_rank"] = fr
+            other = [m for m in wl.modes if m != mode]
+            if other:
+                # the same workload in the other mode: CoLA-M's time over CoLA's,
+                # the two modes timed alternately (3 rounds each, medians) so
+                # that both see the same clocks
+                ob = Block(wl, other[0], device, seed=args.seed + rank)
+                for _ in range(args.warmup):
+                    ob.step()
+                t_this, t_other = [], []
+                for _ in range(3):
+                    t_this.append(time_steps(blk.step, args.steps, stream))
+                    t_other.append(time_steps(ob.step, args.steps, stream))
+                ob.check()
+                blk.check()
+                ms_a, ms_o = statistics.median(t_this), statistics.median(t_other)
+                ms_m, ms_c = (ms_a, ms_o) if mode == "cola_m" else (ms_o, ms_a)
+                line["modes"] = {mode: round(ms_a, 4), other[0]: round(ms_o, 4),
+                                 "cola_m_over_cola": round(ms_m / ms_c, 4),
+                                 "how": "alternating, 3 rounds each, medians"}
+                del ob
             line["cpu_baseline"] = cpu_baseline(wl)
     if rank == 0:
         print(json.dumps(line), flush=True)
