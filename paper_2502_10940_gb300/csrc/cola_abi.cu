@@ -4,6 +4,8 @@
 #include <cuda.h>
 #include <cuda_runtime.h>
 
+#include <algorithm>
+#include <cmath>
 #include <cstdint>
 #include <cstring>
 #include <mutex>
@@ -75,6 +77,14 @@ cola_status_t check_desc(const cola_desc_t* d, Shape* s)
     const int64_t lim = (int64_t(1) << 31) - 256;
     if (s->n > lim || s->d_in > lim || s->d_out > lim || 3 * s->r > lim || s->ld_x > lim || s->ld_y > lim ||
         s->ld_a > lim)
+        return COLA_ERR_UNSUPPORTED;
+    // the work units of one launch are numbered in 32 bits: up to 3 projections
+    // of (n / 128) x (width / 128) output tiles, or up to 4 weight gradients of
+    // (width / 128)^2 tiles split up to n / 256 ways
+    const double w = static_cast<double>(std::max({s->d_in, s->d_out, 3 * s->r}));
+    const double row_tiles = std::ceil(static_cast<double>(s->n) / 128.0), col_tiles = std::ceil(w / 128.0);
+    const double cap = 2147483647.0 / 2.0;
+    if (3.0 * row_tiles * col_tiles > cap || 4.0 * col_tiles * col_tiles * std::ceil(s->n / 256.0) > cap)
         return COLA_ERR_UNSUPPORTED;
     return COLA_OK;
 }

@@ -64,6 +64,7 @@ def _ws_size(L, d, nproj=1):
     (dict(ld_y=132), 1),                  # pitch not a multiple of 8
     (dict(sigma=7), 1),
     (dict(mode=5), 1),
+    (dict(n=1 << 30, d_in=1 << 20, d_out=1 << 20, r=128), 3),   # more work units than 32 bits number
 ])
 def test_workspace_size_rejects_bad_desc(L, kw, code):
     args = dict(n=256, d_in=128, d_out=128, r=64)
