@@ -122,6 +122,31 @@ class Block:
     def step_inputs(self):
         return list(self.X.values()) + ([s["dY"] for s in self.layers] if self.train else [])
 
+    def add_input_set(self):
+        """A second set of the step's input buffers (same shapes and pitches),
+        so that the next step's inputs can be copied in while this step runs;
+        bind(i) selects the set the next step reads."""
+        torch = self.torch
+
+        def twin(t):
+            full = torch.as_strided(t, (t.shape[0], t.stride(0)), (t.stride(0), 1))
+            return full.clone()[:, :t.shape[1]]
+
+        if not hasattr(self, "input_sets"):
+            self.input_sets = [(dict(self.X), [s["dY"] for s in self.layers])]
+        X2 = {k: twin(v) for k, v in self.X.items()}
+        dY2 = [twin(s["dY"]) if s["dY"] is not None else None for s in self.layers]
+        self.input_sets.append((X2, dY2))
+
+    def bind(self, i):
+        X, dY = self.input_sets[i]
+        self.X = dict(X)
+        for s, d in zip(self.layers, dY):
+            s["X"] = X[s["L"].x]
+            s["dY"] = d
+        for g in self.groups:
+            g["X"] = X[g["members"][0]["L"].x]
+
     # what a step hands back: the weight gradients (training) or the outputs
     def step_results(self):
         if not self.train:
@@ -652,30 +677,80 @@ def run_cola(args, wl):
         def full_rows(t):   # the whole padded row-major buffer behind a view
             return torch.as_strided(t, (t.shape[0], t.stride(0)), (t.stride(0), 1))
 
-        ins = [full_rows(t) for t in blk.step_inputs()]
         outs = [full_rows(t) for t in blk.step_results()]
-        h_in = [torch.empty(t.shape, dtype=t.dtype, pin_memory=True) for t in ins]
-        for h, t in zip(h_in, ins):
-            h.copy_(t)
         h_out = [torch.empty(t.shape, dtype=t.dtype, pin_memory=True) for t in outs]
+        # Without a graph, the inputs are double-buffered: step k+1's inputs are
+        # copied on a second stream while step k runs (it waits for them before
+        # it starts, and the copy into a buffer waits for the step that last
+        # read it).  A graph replays fixed buffers, so there every step copies
+        # its inputs and then runs.
+        pipelined = not use_graph
+        if pipelined:
+            blk.add_input_set()
+        sets_in = []
+        for i in range(2 if pipelined else 1):
+            if pipelined:
+                blk.bind(i)
+            sets_in.append([full_rows(t) for t in blk.step_inputs()])
+        h_in = [torch.empty(t.shape, dtype=t.dtype, pin_memory=True) for t in sets_in[0]]
+        for h, t in zip(h_in, sets_in[0]):
+            h.copy_(t)
+        copy_stream = torch.cuda.Stream()
 
-        def e2e_step():
-            for h, t in zip(h_in, ins):
+        def copy_in(dst):
+            for h, t in zip(h_in, dst):
                 t.copy_(h, non_blocking=True)
-            step_fn()
-            for h, t in zip(h_out, outs):
-                h.copy_(t, non_blocking=True)
 
-        for _ in range(max(1, args.warmup // 2)):
-            e2e_step()
+        def e2e_run(K):
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            ev_in = [torch.cuda.Event(), torch.cuda.Event()]
+            ev_done = [torch.cuda.Event(), torch.cuda.Event()]
+            if dist:
+                dist.barrier()
+            torch.cuda.synchronize()
+            e0.record(stream)
+            if pipelined:
+                copy_stream.wait_event(e0)
+                with torch.cuda.stream(copy_stream):
+                    copy_in(sets_in[0])
+                ev_in[0].record(copy_stream)
+            for k in range(K):
+                cur, nxt = k % 2, (k + 1) % 2
+                if pipelined:
+                    if k + 1 < K:
+                        if k >= 1:
+                            copy_stream.wait_event(ev_done[nxt])
+                        with torch.cuda.stream(copy_stream):
+                            copy_in(sets_in[nxt])
+                        ev_in[nxt].record(copy_stream)
+                    stream.wait_event(ev_in[cur])
+                    blk.bind(cur)
+                    blk.step()
+                    ev_done[cur].record(stream)
+                else:
+                    copy_in(sets_in[0])
+                    step_fn()
+                for h, t in zip(h_out, outs):
+                    h.copy_(t, non_blocking=True)
+            e1.record(stream)
+            torch.cuda.synchronize()
+            if dist:
+                dist.barrier()
+            return max_over_ranks(e0.elapsed_time(e1) / K, dist, "cuda")
+
+        e2e_run(2)
         e2e_steps = max(3, args.steps // 2)
-        ms_e2e = time_steps(e2e_step, e2e_steps, stream, dist)
+        ms_e2e = e2e_run(e2e_steps)
+        if pipelined:
+            blk.bind(0)
         blk.check()
-        bi = sum(t.numel() * t.element_size() for t in ins)
+        bi = sum(t.numel() * t.element_size() for t in sets_in[0])
         bo = sum(t.numel() * t.element_size() for t in outs)
-        line["e2e"] = {"value": round(flops * world / (ms_e2e / 1e3) / 1e12, 2), "unit": "TFLOP/s",
+        line["e2e"] = {"value": round(whole_job_tflops(flops, world, ms_e2e), 2), "unit": "TFLOP/s",
                        "ms_per_step": round(ms_e2e, 4), "steps": e2e_steps, "h2d_bytes_per_step": bi,
-                       "d2h_bytes_per_step": bo}
+                       "d2h_bytes_per_step": bo,
+                       "inputs": "double-buffered, next step's copies overlap this step" if pipelined
+                       else "copied before each graph replay"}
         del h_in, h_out
         if rank == 0 and world == 1:
             fr = full_rank_baseline(wl, device, max(3, args.steps // 2), 3, seed=args.seed, flush=flush)
