@@ -209,7 +209,9 @@ def launch_cost(kind, shapes, splits, flags):
     e = 2
     tb, tf = 0.0, 0.0
     for (m, n, k) in shapes:
-        if kind == "fwd_zh":
+        if kind in ("fwd_zh", "fwd_y") and flags & 2:
+            b = e * (m * k + n * k)   # split-K partials; the reduce writes the output
+        elif kind == "fwd_zh":
             b = e * (m * k + n * k + m * n * (2 if flags & 1 else 1))
         elif kind == "fwd_y":
             b = e * (m * k + n * k + m * n)
@@ -220,7 +222,7 @@ def launch_cost(kind, shapes, splits, flags):
         elif kind == "bwd_dx":
             b = e * (m * k + n * k + m * n)
         elif kind == "reduce":
-            b = e * m * n
+            b = e * m * n * (2 if flags & 1 else 1)   # flag: the Z/H reduce writes Z and H
         elif kind == "sigma":
             b = e * 2 * m * n
         else:

@@ -135,6 +135,33 @@ WgradPlan wgrad_plan(const cola_desc_t& d, int nproj, int sms)
     return plan_wgrad(M, N, nb + 1, d.n, sms);
 }
 
+// fp32 partial elements the forward of `nproj` projections needs when its
+// GEMMs are small enough to be split over K (small_launch_splits)
+int64_t fwd_part_elems(const cola_desc_t& d, int nproj, int sms)
+{
+    int64_t need = 0;
+    const int64_t R = nproj * d.r;
+    const int bn1 = choose_bn_for(d.n, R, d.d_in);
+    if (choose_msub(d.n, R, d.d_in, bn1) == 1) {
+        GemmParams p = base_params(d.n, R, d.d_in, bn1, 1);
+        const int S = small_launch_splits(p.m_tiles * p.n_tiles, p.k_blocks, sms);
+        if (S > 1) {
+            set_splits(p, S);
+            need = std::max<int64_t>(need, p.splits * partial_elems(p, bn1, 1));
+        }
+    }
+    const int bn2 = choose_bn_for(d.n, d.d_out, d.r);
+    if (choose_msub(d.n, d.d_out, d.r, bn2) == 1) {
+        GemmParams p = base_params(d.n, d.d_out, d.r, bn2, 1);
+        const int S = small_launch_splits(nproj * p.m_tiles * p.n_tiles, p.k_blocks, sms);
+        if (S > 1) {
+            set_splits(p, S);
+            need = std::max<int64_t>(need, nproj * p.splits * partial_elems(p, bn2, 1));
+        }
+    }
+    return need;
+}
+
 // dZ [n x R] bf16 (training modes), H [n x R] bf16 (CoLA-M and inference),
 // the fp32 split partials of the weight-gradient group (training modes).
 WsLayout ws_layout(const cola_desc_t& d, int nproj, int sms)
@@ -147,12 +174,14 @@ WsLayout ws_layout(const cola_desc_t& d, int nproj, int sms)
     L.h_off = off;
     if (d.mode != COLA_MODE_COLA) off += align_up(static_cast<size_t>(d.n) * R * 2);
     L.part_off = off;
-    if (d.mode == COLA_MODE_INFER) {
-        L.total = off;
-        return L;
+    // fp32 partials: of the split-K forward GEMMs of small launches, or of the
+    // weight gradients (the forward and backward calls use them in turn)
+    size_t part = static_cast<size_t>(fwd_part_elems(d, nproj, sms)) * 4;
+    if (d.mode != COLA_MODE_INFER) {
+        const WgradPlan w = wgrad_plan(d, nproj, sms);
+        if (w.splits > 1 || d.wgrad_fp32) part = std::max(part, static_cast<size_t>(w.part_elems) * 4);
     }
-    const WgradPlan w = wgrad_plan(d, nproj, sms);
-    if (w.splits > 1 || d.wgrad_fp32) off += align_up(static_cast<size_t>(w.part_elems) * 4);
+    off += align_up(part);
     L.total = off;
     return L;
 }
@@ -230,7 +259,7 @@ cola_status_t run_batch(int kind, int bn, int msub, const GemmProblem* probs, co
 // F1: Z = X A^T, H = sigma(Z)  (N = r, or 3r for the fused q/k/v factors;
 // Z / H pitch ldz)
 cola_status_t run_f1(const Shape& s, int sigma, int64_t N, const void* X, const void* A, void* Z, void* H,
-                     int64_t ldz, unsigned int* status, int sms, cudaStream_t st)
+                     int64_t ldz, float* part, size_t part_bytes, unsigned int* status, int sms, cudaStream_t st)
 {
     const int bn = choose_bn_for(s.n, N, s.d_in);
     const int ms = choose_msub(s.n, N, s.d_in, bn);
@@ -239,6 +268,39 @@ cola_status_t run_f1(const Shape& s, int sigma, int64_t N, const void* X, const 
     pr.p = base_params(s.n, N, s.d_in, bn, ms);
     COLA_MAP(map_kmajor(&pr.map_a, X, s.d_in, s.n, s.ld_x, a_box_rows(ms)));
     COLA_MAP(map_kmajor(&pr.map_b, A, s.d_in, N, s.ld_a, b_box_rows(bn, ms)));
+    const int S = ms == 1 ? small_launch_splits(pr.p.m_tiles * pr.p.n_tiles, pr.p.k_blocks, sms) : 1;
+    if (S > 1) {
+        // a small launch: K split across CTAs into fp32 partials, then the
+        // reduce applies the Z/H epilogue (Z = bf16(sum), H = bf16(sigma(Z)))
+        set_splits(pr.p, S);
+        const int64_t slab = partial_elems(pr.p, bn, 1);
+        if (static_cast<size_t>(pr.p.splits * slab) * 4 > part_bytes) return COLA_ERR_WORKSPACE;
+        pr.map_d = pr.map_d2 = pr.map_z = pr.map_a;
+        pr.p.D = part;
+        pr.p.ldd = static_cast<long long>(pr.p.n_tiles) * bn;
+        pr.p.part_stride = slab;
+        pr.p.status = status;
+        const int64_t mnk[1][3] = {{s.n, N, s.d_in}};
+        COLA_TRY((run_batch<false, false, EPI_F32>(COLA_KERNEL_FWD_ZH, bn, 1, &pr, mnk, 1, 2, sms, st)));
+        ReduceBatch rb;
+        std::memset(&rb, 0, sizeof rb);
+        rb.count = 1;
+        rb.splits = pr.p.splits;
+        rb.zh = 1;
+        rb.sigma = sigma;
+        ReduceJob& rj = rb.job[0];
+        rj.part = part;
+        rj.part_stride = slab;
+        rj.ldp = pr.p.n_tiles * bn;
+        rj.M = static_cast<int>(s.n);
+        rj.N = static_cast<int>(N);
+        rj.out = Z;
+        rj.out2 = H;
+        rj.ldo = ldz;
+        const int64_t rmnk[1][3] = {{s.n, N, pr.p.splits}};
+        return launched(traced(COLA_KERNEL_REDUCE, 1, rmnk, pr.p.splits, Z ? 1 : 0, st,
+                               [&] { return launch_splitk_reduce(rb, st); }));
+    }
     // Z == nullptr (inference): the epilogue stores H alone, through map_d
     COLA_MAP(map_box32(&pr.map_d, Z ? Z : H, N, s.n, ldz));
     pr.map_d2 = pr.map_d;
@@ -255,13 +317,58 @@ cola_status_t run_f1(const Shape& s, int sigma, int64_t N, const void* X, const 
 // F2: Y_j = H_j B_j^T for `count` projections of one shape (H_j [n x r] with
 // pitch ldh; Y_j pitch ld_y), one launch
 cola_status_t run_f2(const Shape& s, int count, const void* const* H, int64_t ldh, const void* const* B,
-                     void* const* Y, unsigned int* status, int sms, cudaStream_t st)
+                     void* const* Y, float* part, size_t part_bytes, unsigned int* status, int sms, cudaStream_t st)
 {
     const int bn = choose_bn_for(s.n, s.d_out, s.r);
     const int ms = choose_msub(s.n, s.d_out, s.r, bn);
     GemmProblem pr[MAX_GROUP];
     int64_t mnk[MAX_GROUP][3];
     std::memset(pr, 0, sizeof pr);
+    {
+        const GemmParams p0 = base_params(s.n, s.d_out, s.r, bn, ms);
+        const int S = ms == 1 ? small_launch_splits(count * p0.m_tiles * p0.n_tiles, p0.k_blocks, sms) : 1;
+        if (S > 1) {
+            // a small launch: K split into fp32 partials, reduced into bf16 Y_j
+            ReduceBatch rb;
+            std::memset(&rb, 0, sizeof rb);
+            int64_t rmnk[MAX_GROUP][3];
+            float* slab_base = part;
+            for (int j = 0; j < count; ++j) {
+                pr[j].p = p0;
+                set_splits(pr[j].p, S);
+                const int64_t slab = partial_elems(pr[j].p, bn, 1);
+                if (static_cast<size_t>((slab_base - part) + pr[j].p.splits * slab) * 4 > part_bytes)
+                    return COLA_ERR_WORKSPACE;
+                COLA_MAP(map_kmajor(&pr[j].map_a, H[j], s.r, s.n, ldh, a_box_rows(1)));
+                COLA_MAP(map_kmajor(&pr[j].map_b, B[j], s.r, s.d_out, s.r, b_box_rows(bn, 1)));
+                pr[j].map_d = pr[j].map_d2 = pr[j].map_z = pr[j].map_a;
+                pr[j].p.D = slab_base;
+                pr[j].p.ldd = static_cast<long long>(pr[j].p.n_tiles) * bn;
+                pr[j].p.part_stride = slab;
+                pr[j].p.status = status;
+                mnk[j][0] = s.n;
+                mnk[j][1] = s.d_out;
+                mnk[j][2] = s.r;
+                ReduceJob& rj = rb.job[j];
+                rj.part = slab_base;
+                rj.part_stride = slab;
+                rj.ldp = pr[j].p.n_tiles * bn;
+                rj.M = static_cast<int>(s.n);
+                rj.N = static_cast<int>(s.d_out);
+                rj.out = Y[j];
+                rj.ldo = s.ld_y;
+                rmnk[j][0] = s.n;
+                rmnk[j][1] = s.d_out;
+                rmnk[j][2] = pr[j].p.splits;
+                slab_base += pr[j].p.splits * slab;
+            }
+            COLA_TRY((run_batch<false, false, EPI_F32>(COLA_KERNEL_FWD_Y, bn, 1, pr, mnk, count, 2, sms, st)));
+            rb.count = count;
+            rb.splits = pr[0].p.splits;
+            return launched(traced(COLA_KERNEL_REDUCE, count, rmnk, pr[0].p.splits, 0, st,
+                                   [&] { return launch_splitk_reduce(rb, st); }));
+        }
+    }
     for (int j = 0; j < count; ++j) {
         pr[j].p = base_params(s.n, s.d_out, s.r, bn, ms);
         COLA_MAP(map_kmajor(&pr[j].map_a, H[j], s.r, s.n, ldh, a_box_rows(ms)));
@@ -437,11 +544,13 @@ cola_status_t cola_fwd(const cola_desc_t* desc, const void* X, const void* A, co
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     unsigned int* status = ws_status(ws);
     void* H = desc->mode != COLA_MODE_COLA ? static_cast<void*>(wsb(ws) + L.h_off) : H_save;
-    COLA_TRY(run_f1(s, desc->sigma, s.r, X, A, Z_save, H, s.r, status, sms, st));
+    float* part = reinterpret_cast<float*>(wsb(ws) + L.part_off);
+    const size_t part_bytes = L.total - L.part_off;
+    COLA_TRY(run_f1(s, desc->sigma, s.r, X, A, Z_save, H, s.r, part, part_bytes, status, sms, st));
     const void* Hs[1] = {H};
     const void* Bs[1] = {B};
     void* Ys[1] = {Y};
-    return run_f2(s, 1, Hs, s.r, Bs, Ys, status, sms, st);
+    return run_f2(s, 1, Hs, s.r, Bs, Ys, part, part_bytes, status, sms, st);
 }
 
 cola_status_t cola_bwd(const cola_desc_t* desc, const void* X, const void* A, const void* B, const void* dY,
@@ -498,9 +607,11 @@ cola_status_t cola_fwd_shared_x(const cola_desc_t* desc, int32_t count, const vo
     const int64_t R = count * s.r;
     const size_t slice = static_cast<size_t>(s.r) * 2;   // bytes between the projections' column blocks
     uint8_t* H = desc->mode != COLA_MODE_COLA ? wsb(ws) + L.h_off : static_cast<uint8_t*>(H_cat);
-    COLA_TRY(run_f1(s, desc->sigma, R, X, A_cat, Z_cat, H, R, status, sms, st));
+    float* part = reinterpret_cast<float*>(wsb(ws) + L.part_off);
+    const size_t part_bytes = L.total - L.part_off;
+    COLA_TRY(run_f1(s, desc->sigma, R, X, A_cat, Z_cat, H, R, part, part_bytes, status, sms, st));
     const void* Hs[3] = {H, H + slice, H + 2 * slice};
-    return run_f2(s, count, Hs, R, B, Y, status, sms, st);
+    return run_f2(s, count, Hs, R, B, Y, part, part_bytes, status, sms, st);
 }
 
 cola_status_t cola_bwd_shared_x(const cola_desc_t* desc, int32_t count, const void* X, const void* A_cat,
@@ -589,7 +700,8 @@ cola_status_t cola_recompute_up(const cola_desc_t* desc, int32_t count, const vo
     })));
     const size_t slice = static_cast<size_t>(s.r) * 2;
     const void* Hs[3] = {H, H + slice, H + 2 * slice};
-    return run_f2(s, count, Hs, R, B, Y, status, sms, st);
+    float* part = reinterpret_cast<float*>(wsb(ws) + L.part_off);
+    return run_f2(s, count, Hs, R, B, Y, part, L.total - L.part_off, status, sms, st);
 }
 
 static_assert(COLA_STATUS_PRODUCER_TIMEOUT == ST_TIMEOUT_PRODUCER && COLA_STATUS_MMA_TIMEOUT == ST_TIMEOUT_MMA &&

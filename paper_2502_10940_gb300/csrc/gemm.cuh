@@ -643,13 +643,15 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                 tmem_ld_32x32b_x32(tbase + c * 32, v);
                 tmem_ld_wait();
                 if (EPI == EPI_F32) {
-                    float* dst = reinterpret_cast<float*>(p.D) + split * p.part_stride +
-                                 static_cast<long long>(m_blk * TILE_M + row_in_tile) * p.ldd + col0;
-                    float4* d4 = reinterpret_cast<float4*>(dst);
+                    if (row < p.M) {                // rows past the last one: the reduce never reads them
+                        float* dst = reinterpret_cast<float*>(p.D) + split * p.part_stride +
+                                     static_cast<long long>(m_blk * TILE_M + row_in_tile) * p.ldd + col0;
+                        float4* d4 = reinterpret_cast<float4*>(dst);
 #pragma unroll
-                    for (int j = 0; j < 8; ++j)
-                        d4[j] = make_float4(__uint_as_float(v[4 * j]), __uint_as_float(v[4 * j + 1]),
-                                            __uint_as_float(v[4 * j + 2]), __uint_as_float(v[4 * j + 3]));
+                        for (int j = 0; j < 8; ++j)
+                            d4[j] = make_float4(__uint_as_float(v[4 * j]), __uint_as_float(v[4 * j + 1]),
+                                                __uint_as_float(v[4 * j + 2]), __uint_as_float(v[4 * j + 3]));
+                    }
                     continue;
                 }
                 uint32_t w[16];

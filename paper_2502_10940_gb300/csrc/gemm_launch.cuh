@@ -15,14 +15,17 @@ namespace cola {
 template <int BN, int MSUB, bool A_MN, bool B_MN, int EPI, bool PAIR = false>
 cudaError_t launch_gemm(const GemmBatch& batch, int grid, bool pdl, cudaStream_t stream);
 
-// One fixed-order reduction of fp32 split partials into a gradient.
+// One fixed-order reduction of fp32 split partials into a result: a weight
+// gradient, a split-K output GEMM (bf16), or the split-K Z/H GEMM (zh: Z =
+// bf16(sum) into `out` when not null, H = bf16(sigma(Z)) into `out2`).
 struct ReduceJob {
     const float* part;          // splits slabs of part_stride elements
     long long part_stride;
     int ldp;                    // row pitch of a slab
     int M, N;
     void* out;                  // bf16 (or fp32 when accumulating)
-    long long ldo;
+    void* out2;                 // zh: H
+    long long ldo;              // row pitch of out and out2
     long long group_begin;      // first 4-column group of this job in the launch (set by the launcher)
 };
 
@@ -31,6 +34,8 @@ struct ReduceBatch {
     int count;
     int splits;
     int accumulate_f32;
+    int zh;                     // 1: the Z/H epilogue (out = Z or null, out2 = H)
+    int sigma;                  // zh: the activation
     long long groups;           // 4-column groups of all jobs (set by the launcher)
 };
 

@@ -53,7 +53,19 @@ __global__ void __launch_bounds__(RED_THREADS) splitk_reduce_kernel(const __grid
         }
         const float v[4] = {acc.x, acc.y, acc.z, acc.w};
         const int valid = min(4, job.N - j);
-        if (rb.accumulate_f32) {
+        if (rb.zh) {
+            // Z = bf16(sum), H = bf16(sigma(bf16 Z)): the split-K form of the Z/H epilogue
+            const uint32_t z01 = pack_bf16x2(v[0], v[1]), z23 = pack_bf16x2(v[2], v[3]);
+            uint32_t h01 = 0, h23 = 0;
+            with_sigma(rb.sigma, [&](auto tag) {
+                constexpr int S = decltype(tag)::value;
+                h01 = pack_bf16x2(act_sigma<S>(bf16_lo(z01)), act_sigma<S>(bf16_hi(z01)));
+                h23 = pack_bf16x2(act_sigma<S>(bf16_lo(z23)), act_sigma<S>(bf16_hi(z23)));
+            });
+            const long long off = static_cast<long long>(i) * job.ldo + j;   // N = count r: 4 | N
+            if (job.out) *reinterpret_cast<uint2*>(reinterpret_cast<__nv_bfloat16*>(job.out) + off) = make_uint2(z01, z23);
+            *reinterpret_cast<uint2*>(reinterpret_cast<__nv_bfloat16*>(job.out2) + off) = make_uint2(h01, h23);
+        } else if (rb.accumulate_f32) {
             float* o = reinterpret_cast<float*>(job.out) + static_cast<long long>(i) * job.ldo + j;
             for (int e = 0; e < valid; ++e) o[e] += v[e];
         } else {
@@ -68,6 +80,9 @@ __global__ void __launch_bounds__(RED_THREADS) splitk_reduce_kernel(const __grid
 }
 
 template cudaError_t launch_gemm<128, 1, true, true, EPI_STORE>(const GemmBatch&, int, bool, cudaStream_t);
+// split-K output GEMMs of small launches (both operands K-major)
+template cudaError_t launch_gemm<128, 1, false, false, EPI_F32>(const GemmBatch&, int, bool, cudaStream_t);
+template cudaError_t launch_gemm<256, 1, false, false, EPI_F32>(const GemmBatch&, int, bool, cudaStream_t);
 template cudaError_t launch_gemm<256, 1, true, true, EPI_STORE>(const GemmBatch&, int, bool, cudaStream_t);
 template cudaError_t launch_gemm<128, 2, true, true, EPI_STORE>(const GemmBatch&, int, bool, cudaStream_t);
 template cudaError_t launch_gemm<256, 1, true, true, EPI_STORE, true>(const GemmBatch&, int, bool, cudaStream_t);

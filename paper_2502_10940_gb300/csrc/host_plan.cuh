@@ -174,6 +174,20 @@ void set_splits(GemmParams& p, int S)
     p.units = p.m_tiles * p.n_tiles * p.splits;
 }
 
+// Split-K for the forward GEMMs of small launches: with fewer output tiles
+// than half the SMs (a few hundred tokens or less) and K >= 1024, the K range
+// of each tile is split (>= 4 k-blocks per split, up to about one unit per
+// SM); the fp32 partials are reduced, and the epilogue applied, by the reduce
+// kernel.  A shorter K streams too little per tile for the extra reduce
+// launch to pay off (measured: the 2048-token 60M layer, K = 512 / 128, got
+// slower).  1 = no split.
+int small_launch_splits(int tiles, int k_blocks, int sms)
+{
+    if (2 * tiles >= sms || k_blocks < 16) return 1;
+    const int s = (sms + tiles - 1) / tiles;
+    return s < k_blocks / 4 ? s : k_blocks / 4;
+}
+
 int64_t partial_elems(const GemmParams& p, int bn, int msub)
 {
     return static_cast<int64_t>(p.m_tiles) * tile_rows(msub) * p.n_tiles * bn;
@@ -235,14 +249,21 @@ cudaError_t dispatch(int bn, int msub, GemmBatch& b, int sms, cudaStream_t s)
     }
     b.units = units;
     const bool pdl = flops < 64e9;
-    if (msub == TILE_PAIR && bn == 256) {
-        const int pairs = units < sms / 2 ? units : sms / 2;
-        return launch_gemm<256, 1, A_MN, B_MN, EPI, true>(b, 2 * pairs, pdl, s);
+    // the split-K forward GEMMs of small launches (K-major fp32 partials) run
+    // on single-CTA 128-row tiles only
+    constexpr bool small_only = EPI == EPI_F32 && !A_MN;
+    if constexpr (!small_only) {
+        if (msub == TILE_PAIR && bn == 256) {
+            const int pairs = units < sms / 2 ? units : sms / 2;
+            return launch_gemm<256, 1, A_MN, B_MN, EPI, true>(b, 2 * pairs, pdl, s);
+        }
     }
-    if (msub != 1 && bn == 256) return cudaErrorInvalidValue;   // planned tiles exist as above only
+    if (msub != 1 && (bn == 256 || small_only)) return cudaErrorInvalidValue;   // planned tiles exist as above only
     const int grid = units < sms ? units : sms;
     if (bn == 256) return launch_gemm<256, 1, A_MN, B_MN, EPI>(b, grid, pdl, s);
-    if (msub != 1) return launch_gemm<128, 2, A_MN, B_MN, EPI>(b, grid, pdl, s);
+    if constexpr (!small_only) {
+        if (msub != 1) return launch_gemm<128, 2, A_MN, B_MN, EPI>(b, grid, pdl, s);
+    }
     return launch_gemm<128, 1, A_MN, B_MN, EPI>(b, grid, pdl, s);
 }
 

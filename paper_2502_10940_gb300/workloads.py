@@ -108,4 +108,12 @@ WORKLOADS = {
     "7b-infer": Workload("7b-infer", 8192, llama_block(4096, 11008, 1024), modes=("infer",), phase="infer",
                          graph=True, desc="LLaMA-7B-shaped CoLA block, forward only (inference), d=4096, "
                                           "d_ff=11008, r=1024, 8192 tokens (32 x 256)", seqs=32),
+    # one new token for each of 32 sequences: every GEMM has a few output tiles
+    # (split over K across the SMs) and streams its weights
+    "1b-decode": Workload("1b-decode", 32, llama_block(2048, 5461, 512), modes=("infer",), phase="infer",
+                          graph=True, desc="LLaMA-1B-shaped CoLA block, forward only, 32 tokens (one per sequence)",
+                          seqs=32, seq_len=1),
+    "7b-decode": Workload("7b-decode", 32, llama_block(4096, 11008, 1024), modes=("infer",), phase="infer",
+                          graph=True, desc="LLaMA-7B-shaped CoLA block, forward only, 32 tokens (one per sequence)",
+                          seqs=32, seq_len=1),
 }
