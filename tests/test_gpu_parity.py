@@ -258,3 +258,34 @@ def test_small_n_infer_matches_training_forward():
     cola.cola_fwd(d, inp["X"], inp["A"], inp["B"], Y, None, None, ws)
     assert cola.cola_check_status(ws)[0] == 0
     assert torch.equal(Y, ref["Y"])
+
+
+@pytest.mark.parametrize("mode", ["cola", "infer"])
+def test_small_n_shared_x_split_k(mode):
+    # three projections on one X at 40 tokens with K = 1024 in both forward
+    # GEMMs: the Z/H GEMM (N = 3r) and the three Y GEMMs run split over K and
+    # are finished by the reduce (one Z/H job; three Y jobs in one launch)
+    import oracle
+    from paper_2502_10940_gb300 import cola
+    n, d, r = 40, 1024, 1024
+    X = make_inputs(n, d, d, r, seed=70)["X"]
+    parts = [make_inputs(n, d, d, r, seed=71 + j) for j in range(3)]
+    ldx = cola.ld_of(X)
+    A_cat = padded_empty(3 * r, d, ldx)
+    A_cat.copy_(torch.cat([p["A"] for p in parts], 0))
+    Bs = [p["B"] for p in parts]
+    ldy = cola.ld_of(parts[0]["dY"])
+    desc = cola.desc(n, d, d, r, ld_x=ldx, ld_y=ldy, ld_a=ldx, sigma="silu", mode=mode)
+    ws = cola.workspace(desc, nproj=3)
+    Ys = [padded_empty(n, d, ldy) for _ in range(3)]
+    Z = torch.empty((n, 3 * r), dtype=torch.bfloat16, device="cuda") if mode == "cola" else None
+    H = torch.empty((n, 3 * r), dtype=torch.bfloat16, device="cuda") if mode == "cola" else None
+    cola.cola_fwd_shared_x(desc, X, A_cat, Bs, Ys, Z, H, ws)
+    assert cola.cola_check_status(ws)[0] == 0
+    Zs, Hs, Yo = oracle.fwd_qkv(to64(X), [to64(p["A"]) for p in parts], [to64(b) for b in Bs], "silu")
+    for j in range(3):
+        assert_close(f"Y{j}", to64(Ys[j]), Yo[j])
+        if Z is not None:
+            assert_close(f"Z{j}", to64(Z[:, j * r:(j + 1) * r]), Zs[j])
+            assert_close(f"H{j}", to64(H[:, j * r:(j + 1) * r]), Hs[j])
+        assert padding_intact(Ys[j], d)
