@@ -7,7 +7,7 @@ h = B sigma(A x) each, Sec. 3.2 / Fig. 4) followed by their backward
 (Sec. 3.4), every GEMM on the library's tcgen05 kernels through the C ABI.
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--workload 60m|350m|1b|7b|60m-q]
-                    [--mode cola|cola_m|infer] [--impl cola|reference] [--graph auto|on|off]
+                    [--mode cola|cola_m|infer] [--impl cola|reference] [--graph on|off]
 
 Prints ONE JSON line (rank 0).  `value` is whole-job TFLOP/s (algorithmic
 6 n r (d_in + d_out) per layer), device-timed with CUDA events, inputs
@@ -617,10 +617,11 @@ def run_cola(args, wl):
     for _ in range(args.warmup):
         blk.step()
     torch.cuda.synchronize()
-    # short steps replay as one CUDA graph: the launches of a step are
-    # recorded once (after the eager warm-up, which set every kernel's
-    # attributes) and replayed with no host work per launch
-    use_graph = args.graph == "on" or (args.graph == "auto" and wl.graph)
+    # each step replays as one CUDA graph: its launches are recorded once
+    # (after the eager warm-up, which set every kernel's attributes) and
+    # replayed with no host work per launch and less launch overhead on the
+    # GPU (measured: -2 % step time on the 60M and 1B blocks)
+    use_graph = args.graph != "off"
     step_fn = blk.step
     if use_graph:
         graph = torch.cuda.CUDAGraph()
@@ -681,19 +682,23 @@ def run_cola(args, wl):
 
         outs = [full_rows(t) for t in blk.step_results()]
         h_out = [torch.empty(t.shape, dtype=t.dtype, pin_memory=True) for t in outs]
-        # Without a graph, the inputs are double-buffered: step k+1's inputs are
-        # copied on a second stream while step k runs (it waits for them before
-        # it starts, and the copy into a buffer waits for the step that last
-        # read it).  A graph replays fixed buffers, so there every step copies
-        # its inputs and then runs.
-        pipelined = not use_graph
-        if pipelined:
-            blk.add_input_set()
+        # The inputs are double-buffered: step k+1's inputs are copied on a
+        # second stream while step k runs (it waits for them before it starts,
+        # and the copy into a buffer waits for the step that last read it).
+        # With graphs, one graph per buffer set.
+        blk.add_input_set()
         sets_in = []
-        for i in range(2 if pipelined else 1):
-            if pipelined:
-                blk.bind(i)
+        for i in range(2):
+            blk.bind(i)
             sets_in.append([full_rows(t) for t in blk.step_inputs()])
+        run_set = [blk.step, blk.step]
+        if use_graph:
+            g1 = torch.cuda.CUDAGraph()
+            blk.bind(1)
+            with torch.cuda.graph(g1):
+                blk.step()
+            run_set = [graph.replay, g1.replay]
+        blk.bind(0)
         h_in = [torch.empty(t.shape, dtype=t.dtype, pin_memory=True) for t in sets_in[0]]
         for h, t in zip(h_in, sets_in[0]):
             h.copy_(t)
@@ -711,27 +716,23 @@ def run_cola(args, wl):
                 dist.barrier()
             torch.cuda.synchronize()
             e0.record(stream)
-            if pipelined:
-                copy_stream.wait_event(e0)
-                with torch.cuda.stream(copy_stream):
-                    copy_in(sets_in[0])
-                ev_in[0].record(copy_stream)
+            copy_stream.wait_event(e0)
+            with torch.cuda.stream(copy_stream):
+                copy_in(sets_in[0])
+            ev_in[0].record(copy_stream)
             for k in range(K):
                 cur, nxt = k % 2, (k + 1) % 2
-                if pipelined:
-                    if k + 1 < K:
-                        if k >= 1:
-                            copy_stream.wait_event(ev_done[nxt])
-                        with torch.cuda.stream(copy_stream):
-                            copy_in(sets_in[nxt])
-                        ev_in[nxt].record(copy_stream)
-                    stream.wait_event(ev_in[cur])
+                if k + 1 < K:
+                    if k >= 1:
+                        copy_stream.wait_event(ev_done[nxt])
+                    with torch.cuda.stream(copy_stream):
+                        copy_in(sets_in[nxt])
+                    ev_in[nxt].record(copy_stream)
+                stream.wait_event(ev_in[cur])
+                if not use_graph:
                     blk.bind(cur)
-                    blk.step()
-                    ev_done[cur].record(stream)
-                else:
-                    copy_in(sets_in[0])
-                    step_fn()
+                run_set[cur]()
+                ev_done[cur].record(stream)
                 for h, t in zip(h_out, outs):
                     h.copy_(t, non_blocking=True)
             e1.record(stream)
@@ -743,16 +744,14 @@ def run_cola(args, wl):
         e2e_run(2)
         e2e_steps = max(3, args.steps // 2)
         ms_e2e = e2e_run(e2e_steps)
-        if pipelined:
-            blk.bind(0)
+        blk.bind(0)
         blk.check()
         bi = sum(t.numel() * t.element_size() for t in sets_in[0])
         bo = sum(t.numel() * t.element_size() for t in outs)
         line["e2e"] = {"value": round(whole_job_tflops(flops, world, ms_e2e), 2), "unit": "TFLOP/s",
                        "ms_per_step": round(ms_e2e, 4), "steps": e2e_steps, "h2d_bytes_per_step": bi,
                        "d2h_bytes_per_step": bo,
-                       "inputs": "double-buffered, next step's copies overlap this step" if pipelined
-                       else "copied before each graph replay"}
+                       "inputs": "double-buffered, next step's copies overlap this step"}
         del h_in, h_out
         if rank == 0 and world == 1:
             fr = full_rank_baseline(wl, device, max(3, args.steps // 2), 3, seed=args.seed, flush=flush)
@@ -796,8 +795,8 @@ def main(argv=None):
     ap.add_argument("--impl", default="cola", choices=["cola", "reference"])
     ap.add_argument("--workload", default="60m", choices=sorted(WORKLOADS))
     ap.add_argument("--mode", default=None, choices=["cola", "cola_m", "infer"])
-    ap.add_argument("--graph", default="auto", choices=["auto", "on", "off"],
-                    help="replay each step as one CUDA graph (auto: for the short, launch-bound workloads)")
+    ap.add_argument("--graph", default="on", choices=["on", "off"],
+                    help="replay each step as one CUDA graph (off: launch every kernel from the host)")
     ap.add_argument("--seed", type=int, default=0)
     ap.add_argument("--no-extras", action="store_true", help="skip e2e, full-rank and CPU baselines")
     args = ap.parse_args(argv)

@@ -34,7 +34,6 @@ class Workload:
     seqs: int = 0
     seq_len: int = 256
     phase: str = "train"    # "train": forward + backward; "infer": forward only, nothing saved
-    graph: bool = False     # replay each step as one CUDA graph (short, launch-bound steps)
 
     @property
     def flops(self) -> float:
@@ -86,7 +85,7 @@ def paper_flops_cola(n: int, d: int, d_ff: int, r: int) -> float:
 WORKLOADS = {
     "60m-q": Workload("60m-q", 2048, (Layer("q", 512, 512, 128, "x_attn"),), fused_qkv=False,
                       desc="single CoLA layer, LLaMA-60M q-proj shape, n=2048, 512->512, r=128",
-                      seqs=8, graph=True),
+                      seqs=8),
     "60m": Workload("60m", 65536, llama_block(512, 1376, 128),
                     desc="LLaMA-60M-shaped CoLA block, 7 layers, d=512, d_ff=1376, r=128, "
                          "65536 tokens (256 x 256)", seqs=256),
@@ -102,18 +101,14 @@ WORKLOADS = {
     "1b-o": Workload("1b-o", 65536, (Layer("o", 2048, 2048, 512, "x_o"),), fused_qkv=False,
                      desc="single CoLA layer, LLaMA-1B o-proj shape, 65536 tokens, 2048->2048, r=512", seqs=256),
     # inference at the pre-training shapes with 32 sequences of 256 tokens (Table 10)
-    "1b-infer": Workload("1b-infer", 8192, llama_block(2048, 5461, 512), modes=("infer",), phase="infer",
-                         graph=True, desc="LLaMA-1B-shaped CoLA block, forward only (inference), d=2048, "
+    "1b-infer": Workload("1b-infer", 8192, llama_block(2048, 5461, 512), modes=("infer",), phase="infer", desc="LLaMA-1B-shaped CoLA block, forward only (inference), d=2048, "
                                           "d_ff=5461, r=512, 8192 tokens (32 x 256)", seqs=32),
-    "7b-infer": Workload("7b-infer", 8192, llama_block(4096, 11008, 1024), modes=("infer",), phase="infer",
-                         graph=True, desc="LLaMA-7B-shaped CoLA block, forward only (inference), d=4096, "
+    "7b-infer": Workload("7b-infer", 8192, llama_block(4096, 11008, 1024), modes=("infer",), phase="infer", desc="LLaMA-7B-shaped CoLA block, forward only (inference), d=4096, "
                                           "d_ff=11008, r=1024, 8192 tokens (32 x 256)", seqs=32),
     # one new token for each of 32 sequences: every GEMM has a few output tiles
     # (split over K across the SMs) and streams its weights
-    "1b-decode": Workload("1b-decode", 32, llama_block(2048, 5461, 512), modes=("infer",), phase="infer",
-                          graph=True, desc="LLaMA-1B-shaped CoLA block, forward only, 32 tokens (one per sequence)",
+    "1b-decode": Workload("1b-decode", 32, llama_block(2048, 5461, 512), modes=("infer",), phase="infer", desc="LLaMA-1B-shaped CoLA block, forward only, 32 tokens (one per sequence)",
                           seqs=32, seq_len=1),
-    "7b-decode": Workload("7b-decode", 32, llama_block(4096, 11008, 1024), modes=("infer",), phase="infer",
-                          graph=True, desc="LLaMA-7B-shaped CoLA block, forward only, 32 tokens (one per sequence)",
+    "7b-decode": Workload("7b-decode", 32, llama_block(4096, 11008, 1024), modes=("infer",), phase="infer", desc="LLaMA-7B-shaped CoLA block, forward only, 32 tokens (one per sequence)",
                           seqs=32, seq_len=1),
 }
