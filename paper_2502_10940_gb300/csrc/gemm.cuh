@@ -20,9 +20,10 @@
 //
 // Warp roles (320 threads, one CTA per SM, persistent over output tiles):
 //   warp 0      TMA producer: fills a STAGES-deep ring of (A, B) k-blocks.
-//   warp 1      MMA issuer:  tcgen05.mma M=128, N=BN, K=16 into one of two
-//               TMEM accumulators (double buffered, so the epilogue of tile
-//               i overlaps the main loop of tile i+1); allocates TMEM.
+//   warp 1      MMA issuer:  tcgen05.mma M=128 (M=256 on a CTA pair, issued
+//               by its even CTA), N=BN, K=16 into one of two TMEM
+//               accumulators (double buffered, so the epilogue of tile i
+//               overlaps the main loop of tile i+1); allocates TMEM.
 //   warps 2..9  epilogue, two warps per TMEM lane quarter taking alternate
 //               32-column chunks: tcgen05.ld -> fused elementwise -> 32x32
 //               boxes staged in shared memory (64-byte swizzle, bank-conflict
@@ -35,7 +36,9 @@
 //   EPI_ZH      Z = bf16(acc), H = bf16(sigma(Z))              (forward A-GEMM)
 //   EPI_DSIGMA  dZ = bf16(acc * sigma'(Z_saved)); with CoLA-M also
 //               H = bf16(sigma(Z_saved)) for the weight gradient of B
-//   EPI_F32     fp32 split-K partial slab (weight gradients, reduced later)
+//   EPI_F32     fp32 split-K partial slab, reduced (in a fixed order) by the
+//               reduce kernel: the weight gradients, and the forward GEMMs of
+//               small launches
 //
 // Every mbarrier wait is bounded (WAIT_LIMIT_NS of global time).  On expiry
 // the waiting thread records where it gave up in the status word, raises a

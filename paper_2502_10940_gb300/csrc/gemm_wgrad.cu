@@ -2,7 +2,9 @@
 // the n tokens, both operands are token-major activations read MN-major, and
 // the token range is split across CTAs into fp32 partial slabs that
 // splitk_reduce_kernel sums in a fixed order (or, unsplit, the epilogue
-// stores the bf16 gradient directly).
+// stores the bf16 gradient directly).  The same reduce finishes the split-K
+// forward GEMMs of small launches (instantiated here too), applying the Z/H
+// epilogue for the Z GEMM.
 #define COLA_DEFINE_LAUNCHERS
 #include "gemm_launch.cuh"
 
