@@ -267,24 +267,35 @@ def summarize_trace(records, peaks, ridge):
                       "tflops": round(v["flops"] / (v["ms"] / 1e3) / 1e12, 1)} for k, v in kinds.items()}
 
 
+def kernel_source_hash():
+    """sha256 of the GEMM kernel's code (gemm.cuh and ptx.cuh with comments
+    and whitespace removed): a committed ncu figure stays valid while this
+    hash, i.e. the code it was measured on, is unchanged."""
+    import hashlib
+    import re
+
+    h = hashlib.sha256()
+    for name in ("gemm.cuh", "ptx.cuh"):
+        with open(os.path.join(ROOT, "paper_2502_10940_gb300", "csrc", name)) as g:
+            src = g.read()
+        src = re.sub(r"//[^\n]*", "", src)
+        src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+        h.update(re.sub(r"\s+", "", src).encode())
+    return h.hexdigest()
+
+
 def traffic_from_profile(kernel_key, workload, algorithmic_bytes):
     """dram bytes per launch from a committed ncu summary, valid only while the
-    kernel sources are unchanged (hash match) and the launches it averaged
+    kernel code is unchanged (kernel_source_hash) and the launches it averaged
     carry the same algorithmic bytes as the ones timed now; else None."""
-    import hashlib
-
     path = os.path.join(ROOT, "profiles", "ncu_traffic.json")
     if not os.path.exists(path):
         return None
     try:
         with open(path) as f:
             rec = json.load(f)
-        h = hashlib.sha256()
-        for name in ("gemm.cuh", "ptx.cuh"):
-            with open(os.path.join(ROOT, "paper_2502_10940_gb300", "csrc", name), "rb") as g:
-                h.update(g.read())
         entry = rec.get(workload, {}).get(kernel_key)
-        if (entry and entry.get("src_sha256") == h.hexdigest()
+        if (entry and entry.get("src_sha256") == kernel_source_hash()
                 and entry.get("algorithmic_bytes_per_launch") == algorithmic_bytes):
             return entry["dram_bytes_per_launch"]
     except Exception:  # noqa: BLE001 -- a missing or stale summary means "no traffic figure"
