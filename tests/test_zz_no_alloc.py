@@ -23,7 +23,8 @@ def cola():
     return c
 
 
-@pytest.mark.parametrize("shape", [(4100, 136, 200, 64), (2048, 512, 1376, 128)], ids=str)
+# the last shape plans CTA-pair tiles (dB = dY^T H with M = 2048, N = 512 over 65536 tokens)
+@pytest.mark.parametrize("shape", [(4100, 136, 200, 64), (2048, 512, 1376, 128), (65536, 2048, 2048, 512)], ids=str)
 def test_matches_workspace_path_twice(cola, shape):
     n, d_in, d_out, r = shape
     inp = make_inputs(n, d_in, d_out, r, seed=21)
