@@ -46,9 +46,21 @@ def _full_bits(t):
 
 @pytest.mark.parametrize("shape", SHAPES, ids=lambda s: "x".join(map(str, s)))
 def test_full_size_layer_sampled(shape):
+    _check_sampled(shape, "silu", "cola")
+
+
+# The other activations on the CTA-pair path with a ragged last pair tile, in
+# CoLA-M mode: the pair Z/H epilogue applies sigma, the pair dZ epilogue applies
+# sigma' and recomputes H = sigma(Z) for dB.
+@pytest.mark.parametrize("sigma", ["gelu", "identity"])
+def test_pair_tiles_other_activations_cola_m(sigma):
+    _check_sampled((8200, 2048, 2048, 512), sigma, "cola_m")
+
+
+def _check_sampled(shape, sigma, mode):
     n, d_in, d_out, r = shape
     inp = I.layer_inputs(n, d_in, d_out, r, seed=7, device="cuda")
-    g = gpu_layer(inp, "silu", "cola")
+    g = gpu_layer(inp, sigma, mode)
     torch.cuda.synchronize()
 
     Xb, dYb = _full_bits(inp["X"]), _full_bits(inp["dY"])
@@ -57,24 +69,25 @@ def test_full_size_layer_sampled(shape):
     # random rows plus rows of the last (possibly ragged) 256-row tile
     tail = [n - 1 - k for k in (0, 1, 63, 64, 127, 128, 200) if n - 1 - k >= 0]
     rows = np.unique(np.concatenate([rng.choice(n, 44, replace=False), tail]))
-    Z, H, Y, dZ, dX = oracle.rows_bf16(Xb, Ab, Bb, rows, dYb, "silu", d_in=d_in, d_out=d_out)
+    Z, H, Y, dZ, dX = oracle.rows_bf16(Xb, Ab, Bb, rows, dYb, sigma, d_in=d_in, d_out=d_out)
     ridx = torch.from_numpy(rows).cuda()
     assert_close("Z rows", to64(g["Z"][ridx]), Z)
-    assert_close("H rows", to64(g["H"][ridx]), H)
+    if g["H"] is not None:
+        assert_close("H rows", to64(g["H"][ridx]), H)
     assert_close("Y rows", to64(g["Y"][ridx]), Y)
     assert_close("dX rows", to64(g["dX"][ridx]), dX)
 
     ii = rng.integers(0, r, 32)
     kk = rng.integers(0, d_in, 32)
     kk[-1] = d_in - 1
-    dA_o = oracle.dA_entries_bf16(Xb, Ab, Bb, dYb, ii, kk, "silu", d_out=d_out)
+    dA_o = oracle.dA_entries_bf16(Xb, Ab, Bb, dYb, ii, kk, sigma, d_out=d_out)
     dA_g = to64(g["dA"])[ii, kk]
     assert_close("dA entries", dA_g, dA_o)
 
     oo = rng.integers(0, d_out, 32)
     oo[-1] = d_out - 1
     jj = rng.integers(0, r, 32)
-    dB_o = oracle.dB_entries_bf16(Xb, Ab, dYb, oo, jj, "silu")
+    dB_o = oracle.dB_entries_bf16(Xb, Ab, dYb, oo, jj, sigma)
     dB_g = to64(g["dB"])[oo, jj]
     assert_close("dB entries", dB_g, dB_o)
 

@@ -147,6 +147,49 @@ def test_qkv_fused_matches_oracle(shape, mode):
 
 
 @pytest.mark.parametrize("mode", ["cola", "cola_m"])
+def test_qkv_fused_fp32_accumulate_gelu(mode):
+    # fp32 weight gradients through the shared-input backward: dA_qkv [3r x d]
+    # and each dB_j are added onto existing fp32 values (micro-batching), with
+    # the GELU activation and a ragged token count (a partial last token tile)
+    import oracle
+    from paper_2502_10940_gb300 import cola
+    n, d, r = 1100, 264, 64
+    X = make_inputs(n, d, d, r, seed=40)["X"]
+    parts = [make_inputs(n, d, d, r, seed=41 + j) for j in range(3)]
+    ldx = cola.ld_of(X)
+    A_pad = padded_empty(3 * r, d, ldx)
+    A_pad.copy_(torch.cat([p["A"] for p in parts], 0))
+    Bs = [p["B"] for p in parts]
+    dYs = [p["dY"] for p in parts]
+    ldy = cola.ld_of(dYs[0])
+    desc = cola.desc(n, d, d, r, ld_x=ldx, ld_y=ldy, ld_a=ldx, sigma="gelu", mode=mode, wgrad_fp32=True)
+    ws = cola.workspace(desc, nproj=3)
+    Ys = [padded_empty(n, d, ldy) for _ in range(3)]
+    Z = torch.empty((n, 3 * r), dtype=torch.bfloat16, device="cuda")
+    H = torch.empty((n, 3 * r), dtype=torch.bfloat16, device="cuda") if mode == "cola" else None
+    cola.cola_fwd_qkv_fused(desc, X, A_pad, *Bs, *Ys, Z, H, ws)
+    g0 = torch.Generator(device="cuda").manual_seed(42)
+    dA0 = torch.randn((3 * r, d), generator=g0, device="cuda")
+    dB0 = [torch.randn((d, r), generator=g0, device="cuda") for _ in range(3)]
+    dX = padded_empty(n, d, ldx)
+    dA = padded_empty(3 * r, d, ldx, torch.float32)
+    dA.copy_(dA0)
+    dBs = [b.clone() for b in dB0]
+    cola.cola_bwd_qkv_fused(desc, X, A_pad, *Bs, *dYs, Z, H, dX, dA, *dBs, ws)
+    assert cola.cola_check_status(ws)[0] == 0
+
+    X64 = to64(X)
+    As = [to64(p["A"]) for p in parts]
+    Bo = [to64(b) for b in Bs]
+    Zs, Hs, Yo = oracle.fwd_qkv(X64, As, Bo, "gelu")
+    dXo, dAo, dBo, _ = oracle.bwd_qkv(X64, As, Bo, [to64(t) for t in dYs], Zs, Hs, "gelu", "cola")
+    for j in range(3):
+        assert_close(f"dB{j}+=", to64(dBs[j]) - to64(dB0[j]), dBo[j])
+        assert_close(f"dA{j}+=", (to64(dA) - to64(dA0))[j * r:(j + 1) * r], dAo[j])
+    assert_close("dX", to64(dX), dXo)
+
+
+@pytest.mark.parametrize("mode", ["cola", "cola_m"])
 @pytest.mark.parametrize("shape", [(300, 200, 328, 128), (2048, 512, 1376, 128)], ids=str)
 def test_shared_x_pair_matches_oracle(shape, mode):
     # gate / up: two projections of one shape reading one X (Fig. 4); dX is
