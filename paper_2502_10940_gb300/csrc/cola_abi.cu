@@ -5,6 +5,7 @@
 #include <cuda_runtime.h>
 
 #include <algorithm>
+#include <atomic>
 #include <cmath>
 #include <cstdint>
 #include <cstring>
@@ -18,8 +19,10 @@ namespace cola {
 namespace {
 
 // ------------------------------------------------------------ device info
+// Queried once per device; `ok` is published (release) after `sms`, so a
+// thread that reads ok != 0 without the lock also sees sms.
 struct DevInfo {
-    int ok = 0;      // 1: queried, 2: unsupported device
+    std::atomic<int> ok{0};   // 1: queried, 2: unsupported device
     int sms = 0;
 };
 
@@ -31,19 +34,22 @@ cola_status_t device_info(int* sms)
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return COLA_ERR_LAUNCH;
     DevInfo& d = g_dev[dev];
-    if (d.ok == 0) {
+    int ok = d.ok.load(std::memory_order_acquire);
+    if (ok == 0) {
         std::lock_guard<std::mutex> lock(g_mu);
-        if (d.ok == 0) {
+        ok = d.ok.load(std::memory_order_relaxed);
+        if (ok == 0) {
             int major = 0, minor = 0, n = 0;
             if (cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev) != cudaSuccess ||
                 cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev) != cudaSuccess ||
                 cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
                 return COLA_ERR_LAUNCH;
             d.sms = n;
-            d.ok = (major == 10 && minor == 3) ? 1 : 2;   // kernels are built for sm_103a only
+            ok = (major == 10 && minor == 3) ? 1 : 2;   // kernels are built for sm_103a only
+            d.ok.store(ok, std::memory_order_release);
         }
     }
-    if (d.ok != 1) return COLA_ERR_UNSUPPORTED;
+    if (ok != 1) return COLA_ERR_UNSUPPORTED;
     *sms = d.sms;
     return COLA_OK;
 }

@@ -4,6 +4,8 @@
 #pragma once
 #include <cuda_runtime.h>
 
+#include <atomic>
+
 #include "gemm.cuh"
 
 namespace cola {
@@ -51,15 +53,16 @@ cudaError_t launch_gemm(const GemmBatch& batch, int grid, bool pdl, cudaStream_t
 {
     constexpr int smem = GemmCfg<BN, MSUB, PAIR>::SMEM_BYTES;
     auto kern = gemm_kernel<BN, MSUB, A_MN, B_MN, EPI, PAIR>;
-    // the opt-in shared-memory size is a per-device function attribute
-    static unsigned long long configured = 0;   // bit d: set on device d
+    // the opt-in shared-memory size is a per-device function attribute; host
+    // threads may launch concurrently, so the set of configured devices is atomic
+    static std::atomic<unsigned long long> configured{0};   // bit d: set on device d
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
-    if (dev >= 64 || !((configured >> dev) & 1ull)) {
+    if (dev >= 64 || !((configured.load(std::memory_order_acquire) >> dev) & 1ull)) {
         e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
         if (e != cudaSuccess) return e;
-        if (dev < 64) configured |= 1ull << dev;
+        if (dev < 64) configured.fetch_or(1ull << dev, std::memory_order_acq_rel);
     }
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(grid);

@@ -91,6 +91,39 @@ def test_deterministic():
         assert torch.equal(a[k], b[k]), k
 
 
+def test_two_host_threads_on_two_streams():
+    # The library keeps no per-call host state: two host threads, each with its
+    # own stream and workspace, run layers concurrently (their kernels overlap
+    # on the GPU) and get the results of a lone run bit for bit.
+    import threading
+    shapes = [(4100, 136, 200, 64), (2048, 512, 512, 128)]
+    inps = [make_inputs(*sh, seed=60 + i) for i, sh in enumerate(shapes)]
+    ref = [gpu_layer(inp, "silu", "cola") for inp in inps]
+    torch.cuda.synchronize()
+    out, err = [None, None], [None, None]
+
+    def work(i):
+        try:
+            s = torch.cuda.Stream()
+            with torch.cuda.stream(s):
+                res = [gpu_layer(inps[i], "silu", "cola") for _ in range(3)]
+            s.synchronize()
+            out[i] = res
+        except Exception as e:  # noqa: BLE001 -- reported by the assertion below
+            err[i] = e
+
+    threads = [threading.Thread(target=work, args=(i,)) for i in range(2)]
+    for t in threads:
+        t.start()
+    for t in threads:
+        t.join()
+    assert err == [None, None], err
+    for i in range(2):
+        for res in out[i]:
+            for k in ["Y", "Z", "H", "dX", "dA", "dB"]:
+                assert torch.equal(res[k], ref[i][k]), (i, k)
+
+
 def test_wgrad_fp32_accumulate():
     n, d_in, d_out, r = 300, 200, 328, 128
     inp = make_inputs(n, d_in, d_out, r, seed=5)
