@@ -45,6 +45,9 @@
  *     the device status word and must be zeroed once with
  *     cola_workspace_init() before first use.  One workspace must not be
  *     used by two calls that may run concurrently.
+ *   - The entry points may be called from several host threads at once, each
+ *     with its own workspace (and, typically, its own stream); the launch
+ *     tracing below is the one exception.
  *   - Every wait inside the kernels is bounded (about 2 s).  A wait that runs
  *     out records a code in the workspace status word and the kernel returns
  *     early (its outputs are then undefined); cola_check_status() reports it.
