@@ -242,9 +242,12 @@ cola_status_t cola_selftest_wait_timeout(void* ws, size_t ws_bytes, void* stream
  * cudaMalloc, cudaFree or other allocating routine.  A problem whose fp32
  * partial tile grid (M and N rounded up to the tile size) does not fit the
  * array even without a token split returns COLA_ERR_WORKSPACE before any
- * launch.  The first call on each device fetches the array's device address
- * (cudaGetSymbolAddress, which may load the library's device module): make
- * that first call before any stream capture begins on the device.  Every
+ * launch.  A problem the planner runs without a token split, with a bf16
+ * D, stores D straight from the GEMM epilogue and does not touch the array.
+ * The first call on each device that uses the array fetches its device
+ * address (cudaGetSymbolAddress, which may load the library's device module;
+ * a failed lookup returns COLA_ERR_LAUNCH and is retried by the next call):
+ * make that first call before any stream capture begins on the device.  Every
  * call shares the one array, so calls that may overlap on the GPU (other
  * streams, other host threads) race and must be serialised by the caller.
  * Nothing in the array needs to start at zero: each call overwrites the

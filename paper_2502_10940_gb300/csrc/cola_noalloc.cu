@@ -11,10 +11,11 @@
 //
 // The array's name is only a host-side stand-in in host code.  Its device
 // address is fetched with cudaGetSymbolAddress once per device, with that
-// device current, on the first call that runs on it; kernels only ever see
-// that address.
+// device current, on the first call that runs on it (a failed lookup is
+// retried by the next call); kernels only ever see that address.
 #include <cuda_runtime.h>
 
+#include <atomic>
 #include <cstdint>
 #include <cstring>
 #include <mutex>
@@ -32,24 +33,27 @@ constexpr size_t kStaticScratchBytes = static_cast<size_t>(COLA_STATIC_SCRATCH_B
 // on a device (calls that overlap on the GPU race on it).
 static __device__ __align__(256) unsigned char g_wgrad_scratch[kStaticScratchBytes];
 
-struct ScratchSlot {
-    std::once_flag once;
-    cudaError_t err = cudaSuccess;
-    void* ptr = nullptr;
-};
-ScratchSlot g_slots[64];
+// Per device, the array's device address once a lookup has succeeded; a
+// failed lookup is not cached, so the next call on that device tries again.
+std::atomic<void*> g_scratch_ptr[64];
+std::mutex g_scratch_mu;
 
-// Device address of g_wgrad_scratch on the current device (set up once per device).
+// Device address of g_wgrad_scratch on the current device `dev`.
 cudaError_t scratch_address(int dev, void** out)
 {
-    ScratchSlot& s = g_slots[dev];
-    std::call_once(s.once, [&] {
-        void* p = nullptr;
-        s.err = cudaGetSymbolAddress(&p, g_wgrad_scratch);
-        if (s.err == cudaSuccess) s.ptr = p;
-    });
-    *out = s.ptr;
-    return s.err;
+    void* p = g_scratch_ptr[dev].load(std::memory_order_acquire);
+    if (!p) {
+        std::lock_guard<std::mutex> lock(g_scratch_mu);
+        p = g_scratch_ptr[dev].load(std::memory_order_relaxed);
+        if (!p) {
+            const cudaError_t e = cudaGetSymbolAddress(&p, g_wgrad_scratch);
+            if (e != cudaSuccess) return e;
+            if (!p) return cudaErrorInvalidSymbol;
+            g_scratch_ptr[dev].store(p, std::memory_order_release);
+        }
+    }
+    *out = p;
+    return cudaSuccess;
 }
 
 }  // namespace
@@ -90,10 +94,7 @@ extern "C" cola_status_t cola_wgrad_static_scratch(int64_t n_tokens, int64_t M, 
     const int max_splits = static_cast<int>(kStaticScratchBytes / slab_bytes);
     if (w.p[0].splits > max_splits) set_splits(w.p[0], max_splits);
 
-    // ---- set-up: the scratch's device address on this device (first call only)
-    void* scratch = nullptr;
-    if (scratch_address(dev, &scratch) != cudaSuccess || scratch == nullptr) return COLA_ERR_LAUNCH;
-
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
     GemmBatch b;
     std::memset(&b, 0, sizeof b);
     b.count = 1;
@@ -101,13 +102,25 @@ extern "C" cola_status_t cola_wgrad_static_scratch(int64_t n_tokens, int64_t M, 
     pr.p = w.p[0];
     if (!map_mnmajor(&pr.map_a, P, M, n_tokens, ld_p) || !map_mnmajor(&pr.map_b, Q, N, n_tokens, ld_q))
         return COLA_ERR_LAUNCH;
+    pr.p.status = nullptr;   // no workspace to report a device-side timeout through
+    if (pr.p.splits == 1 && !accumulate_f32) {
+        // unsplit: the epilogue stores the bf16 gradient directly; no scratch
+        if (!map_box32(&pr.map_d, D, N, M, ld_d)) return COLA_ERR_LAUNCH;
+        pr.map_d2 = pr.map_z = pr.map_d;
+        pr.p.d_ptr = static_cast<__nv_bfloat16*>(D);
+        pr.p.d_ld = ld_d;
+        return dispatch<true, true, EPI_STORE>(w.bn, w.msub, b, sms, st) == cudaSuccess ? COLA_OK : COLA_ERR_LAUNCH;
+    }
+
+    // ---- set-up: the scratch's device address on this device (first call only)
+    void* scratch = nullptr;
+    if (scratch_address(dev, &scratch) != cudaSuccess || scratch == nullptr) return COLA_ERR_LAUNCH;
+
     pr.map_d = pr.map_d2 = pr.map_z = pr.map_a;
     float* part = static_cast<float*>(scratch);
     pr.p.D = part;
     pr.p.ldd = static_cast<long long>(pr.p.n_tiles) * w.bn;
     pr.p.part_stride = w.slab[0];
-    pr.p.status = nullptr;   // no workspace to report a device-side timeout through
-    cudaStream_t st = static_cast<cudaStream_t>(stream);
     if (dispatch<true, true, EPI_F32>(w.bn, w.msub, b, sms, st) != cudaSuccess) return COLA_ERR_LAUNCH;
     ReduceBatch rb;
     std::memset(&rb, 0, sizeof rb);
