@@ -6,15 +6,17 @@ seven CoLA layers of a LLaMA-shaped block (q/k/v fused, o, gate, up, down;
 h = B sigma(A x) each, Sec. 3.2 / Fig. 4) followed by their backward
 (Sec. 3.4), every GEMM on the library's tcgen05 kernels through the C ABI.
 
-    python bench.py [--gpus N] [--steps K] [--warmup W] [--workload 60m|350m|1b|7b|60m-q]
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--workload 7b|1b|350m|60m|60m-q|...]
                     [--mode cola|cola_m|infer] [--impl cola|reference] [--graph on|off]
 
-Prints ONE JSON line (rank 0).  `value` is whole-job TFLOP/s (algorithmic
-6 n r (d_in + d_out) per layer), device-timed with CUDA events, inputs
-resident in HBM; `e2e` is the same metric with each step's inputs copied
-from pinned host memory and the weight gradients copied back inside the
-timed region.  The working set of every block workload is larger than L2
-(129 MB), so no L2 flush is needed between steps.
+The default workload is the LLaMA-7B-shaped block in CoLA-M mode (32768
+tokens); its line also carries the 1B block (65536 tokens) timed in the same
+run.  Prints ONE JSON line (rank 0).  `value` is whole-job TFLOP/s
+(algorithmic 6 n r (d_in + d_out) per layer), device-timed with CUDA events,
+inputs resident in HBM; `e2e` is the same metric with each step's inputs
+copied from pinned host memory and its results (weight and input gradients)
+copied back inside the timed region.  The working set of every block
+workload is larger than L2 (129 MB), so no L2 flush is needed between steps.
 
 --impl reference times the fp64 CPU oracle (the only reference there is: the
 paper publishes no implementation) on the host cores, on a bounded sample of
@@ -147,11 +149,18 @@ class Block:
         for g in self.groups:
             g["X"] = X[g["members"][0]["L"].x]
 
-    # what a step hands back: the weight gradients (training) or the outputs
+    # what a step hands back: the weight gradients and the block's input
+    # gradients (training), or the outputs (inference)
     def step_results(self):
         if not self.train:
             return [s["Y"] for s in self.layers]
-        return [g["dA"] for g in self.groups] + [s["dB"] for s in self.layers]
+        return [g["dA"] for g in self.groups] + [s["dB"] for s in self.layers] + [g["dX"] for g in self.groups]
+
+    def results_words(self):
+        if not self.train:
+            return "Y of every layer"
+        return ("dA and dB of every layer and dX of every input group; Y, Z and H stay on the device "
+                "(they feed the block's attention / MLP ops and the backward)")
 
     def forward(self):
         c = self.cola
@@ -248,16 +257,21 @@ def summarize_trace(records, peaks, ridge):
     d = kinds[top]
     t = d["ms"] / 1e3
     intensity = d["flops"] / max(d["bytes"], 1.0)
+    # every traced launch is bracketed by its own events: a kernel timed
+    # alone, so the burst peak is its denominator (the sustained one beside it)
     if intensity >= ridge:
         achieved = d["flops"] / t / 1e12
-        peak = peaks["bf16_tflops_sustained"]
-        roof = {"bound": "tensor", "unit": "TFLOP/s"}
+        peak = peaks["bf16_tflops"]
+        roof = {"bound": "tensor", "unit": "TFLOP/s",
+                "frac_sustained": round(achieved / peaks["bf16_tflops_sustained"], 4),
+                "peak_sustained": peaks["bf16_tflops_sustained"]}
     else:
         achieved = d["bytes"] / t / 1e9
         peak = peaks["hbm_gbs"]
         roof = {"bound": "hbm", "unit": "GB/s"}
     roof.update({"kernel": f"gemm {top}", "achieved": round(achieved, 1), "peak": peak,
                  "frac": round(achieved / peak, 4), "peak_source": peaks["source"],
+                 "peak_kind": "burst (each launch timed alone)" if roof["bound"] == "tensor" else "copy",
                  "launches": d["launches"], "avg_launch_us": round(d["ms"] * 1e3 / d["launches"], 2),
                  "algorithmic_bytes_per_launch": int(d["bytes"] / d["launches"]),
                  "flop_per_launch": d["flops"] / d["launches"], "share": round(d["share"], 4)})
@@ -593,6 +607,75 @@ def full_rank_baseline(wl, device, steps, warmup, seed=0, flush=None):
             "impl": "torch.matmul (cuBLAS) bf16"}
 
 
+def timed_block(wl, mode, args, device, stream, dist=None, seed=0):
+    """Build the block, count its launches with the library trace, warm it
+    up, capture its step as a CUDA graph (unless --graph off) and time K
+    steps (clocks sampled meanwhile).  Returns a dict of what it built and
+    measured."""
+    import torch
+
+    from paper_2502_10940_gb300 import cola
+
+    blk = Block(wl, mode, device, seed=seed)
+    # launches per step, counted by the library's trace
+    with cola.Trace(512) as tr:
+        blk.step()
+    blk.launches_per_step = tr.count.value
+    blk.check()
+
+    for _ in range(args.warmup):
+        blk.step()
+    torch.cuda.synchronize()
+    # each step replays as one CUDA graph: its launches are recorded once
+    # (after the eager warm-up, which set every kernel's attributes) and
+    # replayed with no host work per launch and less launch overhead on the
+    # GPU (measured: -2 % step time on the 60M and 1B blocks)
+    use_graph = args.graph != "off"
+    step_fn, graph = blk.step, None
+    if use_graph:
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph):
+            blk.step()
+        step_fn = graph.replay
+        for _ in range(args.warmup):
+            step_fn()
+        torch.cuda.synchronize()
+        blk.check()
+    # a working set that fits in L2 is timed step by step with L2 rewritten
+    # between steps
+    ws_bytes = blk.working_set_bytes()
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=device) if ws_bytes < L2_BYTES else None
+    sampler = ClockSampler(torch.cuda.current_device())
+    sampler.start()
+    ms = time_steps(step_fn, args.steps, stream, dist, flush=flush)
+    clocks = sampler.stop()
+    blk.check()
+    return dict(blk=blk, graph=graph, step_fn=step_fn, use_graph=use_graph, ms=ms, clocks=clocks,
+                flush=flush, ws_bytes=ws_bytes)
+
+
+def modes_ratio(wl, mode, blk, args, device, stream, seed=0):
+    """The same workload in its other mode: CoLA-M's time over CoLA's, the two
+    modes timed alternately (3 rounds each, medians) so that both see the
+    same clocks.  None if the workload has one mode."""
+    other = [m for m in wl.modes if m != mode]
+    if not other:
+        return None
+    ob = Block(wl, other[0], device, seed=seed)
+    for _ in range(args.warmup):
+        ob.step()
+    t_this, t_other = [], []
+    for _ in range(3):
+        t_this.append(time_steps(blk.step, args.steps, stream))
+        t_other.append(time_steps(ob.step, args.steps, stream))
+    ob.check()
+    blk.check()
+    ms_a, ms_o = statistics.median(t_this), statistics.median(t_other)
+    ms_m, ms_c = (ms_a, ms_o) if mode == "cola_m" else (ms_o, ms_a)
+    return {mode: round(ms_a, 4), other[0]: round(ms_o, 4), "cola_m_over_cola": round(ms_m / ms_c, 4),
+            "how": "alternating, 3 rounds each, medians (eager launches)"}
+
+
 def run_cola(args, wl):
     import torch
 
@@ -609,6 +692,7 @@ def run_cola(args, wl):
 
     from paper_2502_10940_gb300 import build
     from paper_2502_10940_gb300 import cola
+    from paper_2502_10940_gb300.workloads import WORKLOADS
 
     build.build()
     peaks = _peaks()
@@ -616,42 +700,10 @@ def run_cola(args, wl):
     mode = args.mode or wl.modes[0]
     if (mode == "infer") != (wl.phase == "infer"):
         raise SystemExit(f"mode {mode} does not fit the {wl.phase} workload {wl.name}")
-    blk = Block(wl, mode, device, seed=args.seed + rank)
     stream = torch.cuda.current_stream()
-
-    # launches per step, counted by the library's trace
-    with cola.Trace(512) as tr:
-        blk.step()
-    blk.launches_per_step = tr.count.value
-    blk.check()
-
-    for _ in range(args.warmup):
-        blk.step()
-    torch.cuda.synchronize()
-    # each step replays as one CUDA graph: its launches are recorded once
-    # (after the eager warm-up, which set every kernel's attributes) and
-    # replayed with no host work per launch and less launch overhead on the
-    # GPU (measured: -2 % step time on the 60M and 1B blocks)
-    use_graph = args.graph != "off"
-    step_fn = blk.step
-    if use_graph:
-        graph = torch.cuda.CUDAGraph()
-        with torch.cuda.graph(graph):
-            blk.step()
-        step_fn = graph.replay
-        for _ in range(args.warmup):
-            step_fn()
-        torch.cuda.synchronize()
-        blk.check()
-    # a working set that fits in L2 is timed step by step with L2 rewritten
-    # between steps
-    ws_bytes = blk.working_set_bytes()
-    flush = torch.empty(256 << 20, dtype=torch.uint8, device=device) if ws_bytes < L2_BYTES else None
-    sampler = ClockSampler(local)
-    sampler.start()
-    ms = time_steps(step_fn, args.steps, stream, dist, flush=flush)
-    clocks = sampler.stop()
-    blk.check()
+    tb = timed_block(wl, mode, args, device, stream, dist, seed=args.seed + rank)
+    blk, graph, use_graph, ms, clocks, flush = (tb[k] for k in ("blk", "graph", "use_graph", "ms", "clocks",
+                                                                  "flush"))
 
     # the same steps again with every launch bracketed by events: per-kernel times
     cap = blk.launches_per_step * args.steps
@@ -661,6 +713,7 @@ def run_cola(args, wl):
     roofline, kinds = summarize_trace(records, peaks, ridge)
     roofline["traffic"] = traffic_from_profile(roofline["kernel"], wl.name,
                                                roofline["algorithmic_bytes_per_launch"])
+    trace_ms = sum(r[-1] for r in records) / args.steps
 
     flops = wl.flops
     value = whole_job_tflops(flops, world, ms)
@@ -675,19 +728,23 @@ def run_cola(args, wl):
                        "saved_activation_elems": sum(g[k].numel() for g in blk.groups for k in ("Z", "H")
                                                      if g.get(k) is not None),
                        "cuda_graph": use_graph,
-                       "l2": (f"flushed between steps (256 MB write): working set {ws_bytes / 1e6:.1f} MB < L2"
+                       "l2": (f"flushed between steps (256 MB write): working set {tb['ws_bytes'] / 1e6:.1f} MB < L2"
                               if flush is not None else
-                              f"no flush: working set {ws_bytes / 1e9:.2f} GB > 129 MB L2")},
+                              f"no flush: working set {tb['ws_bytes'] / 1e9:.2f} GB > 129 MB L2")},
             "tokens_per_s": round(wl.n * world / (ms / 1e3), 1),
             "pct_dense_bf16_peak": round(100.0 * value / world / peaks["bf16_tflops"], 2),
             "pct_dense_bf16_peak_sustained": round(100.0 * value / world / peaks["bf16_tflops_sustained"], 2),
             "roofline": roofline, "kernels": kinds,
+            # the per-kernel figures come from eager steps with events around
+            # every launch; their sum per step, beside the graph-timed step
+            "trace_ms_per_step": round(trace_ms, 4),
+            "kernels_how": "eager steps, CUDA events around each launch; shares are of trace_ms_per_step",
             "gpu_launches": blk.launches_per_step * args.steps, "clocks": clocks}
 
     if not args.no_extras:
         # end to end: each step's activations (and, training, upstream
-        # gradients) come from pinned host memory; the weight gradients (or,
-        # inference, the outputs) go back to pinned host memory
+        # gradients) come from pinned host memory; the step's results (see
+        # results_words) go back to pinned host memory
         def full_rows(t):   # the whole padded row-major buffer behind a view
             return torch.as_strided(t, (t.shape[0], t.stride(0)), (t.stride(0), 1))
 
@@ -762,32 +819,34 @@ def run_cola(args, wl):
         line["e2e"] = {"value": round(whole_job_tflops(flops, world, ms_e2e), 2), "unit": "TFLOP/s",
                        "ms_per_step": round(ms_e2e, 4), "steps": e2e_steps, "h2d_bytes_per_step": bi,
                        "d2h_bytes_per_step": bo,
-                       "inputs": "double-buffered, next step's copies overlap this step"}
-        del h_in, h_out
+                       "inputs": "double-buffered, next step's copies overlap this step",
+                       "results_to_host": blk.results_words()}
+        del h_in, h_out, sets_in, outs, run_set
+        if use_graph:
+            del g1
         if rank == 0 and world == 1:
             fr = full_rank_baseline(wl, device, max(3, args.steps // 2), 3, seed=args.seed, flush=flush)
             fr["speedup_cola_vs_full_rank"] = round(fr["ms_per_step"] / ms, 3)
             line["full_rank"] = fr
-            other = [m for m in wl.modes if m != mode]
-            if other:
-                # the same workload in the other mode: CoLA-M's time over CoLA's,
-                # the two modes timed alternately (3 rounds each, medians) so
-                # that both see the same clocks
-                ob = Block(wl, other[0], device, seed=args.seed + rank)
-                for _ in range(args.warmup):
-                    ob.step()
-                t_this, t_other = [], []
-                for _ in range(3):
-                    t_this.append(time_steps(blk.step, args.steps, stream))
-                    t_other.append(time_steps(ob.step, args.steps, stream))
-                ob.check()
-                blk.check()
-                ms_a, ms_o = statistics.median(t_this), statistics.median(t_other)
-                ms_m, ms_c = (ms_a, ms_o) if mode == "cola_m" else (ms_o, ms_a)
-                line["modes"] = {mode: round(ms_a, 4), other[0]: round(ms_o, 4),
-                                 "cola_m_over_cola": round(ms_m / ms_c, 4),
-                                 "how": "alternating, 3 rounds each, medians"}
-                del ob
+            mr = modes_ratio(wl, mode, blk, args, device, stream, seed=args.seed + rank)
+            if mr:
+                line["modes"] = mr
+            # the 1B block in the same run (its value and CoLA-M / CoLA ratio),
+            # after the main workload's tensors are released
+            if wl.name == "7b":
+                del blk, graph, tb
+                torch.cuda.synchronize()
+                torch.cuda.empty_cache()
+                w1 = WORKLOADS["1b"]
+                t1 = timed_block(w1, w1.modes[0], args, device, stream, None, seed=args.seed)
+                v1 = whole_job_tflops(w1.flops, 1, t1["ms"])
+                line["also"] = {"1b": {"workload": w1.desc, "mode": w1.modes[0], "value": round(v1, 2),
+                                       "unit": "TFLOP/s", "ms_per_step": round(t1["ms"], 4),
+                                       "pct_dense_bf16_peak": round(100.0 * v1 / peaks["bf16_tflops"], 2),
+                                       "cuda_graph": t1["use_graph"], "clocks": t1["clocks"],
+                                       "modes": modes_ratio(w1, w1.modes[0], t1["blk"], args, device, stream,
+                                                            seed=args.seed)}}
+                del t1
             line["cpu_baseline"] = cpu_baseline(wl)
     if rank == 0:
         print(json.dumps(line), flush=True)
@@ -804,7 +863,7 @@ def main(argv=None):
     ap.add_argument("--steps", type=int, default=20)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="cola", choices=["cola", "reference"])
-    ap.add_argument("--workload", default="60m", choices=sorted(WORKLOADS))
+    ap.add_argument("--workload", default="7b", choices=sorted(WORKLOADS))
     ap.add_argument("--mode", default=None, choices=["cola", "cola_m", "infer"])
     ap.add_argument("--graph", default="on", choices=["on", "off"],
                     help="replay each step as one CUDA graph (off: launch every kernel from the host)")

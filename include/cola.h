@@ -81,7 +81,7 @@ typedef enum {
 typedef enum {
     COLA_MODE_COLA = 0,          /* forward stores Z and H; backward reads both */
     COLA_MODE_COLA_M = 1,        /* forward stores Z only; backward recomputes H = sigma(Z) */
-    COLA_MODE_INFER = 2          /* forward only (inference, Table 10): nothing is saved, H lives
+    COLA_MODE_INFER = 2          /* forward only (inference, App. E.2): nothing is saved, H lives
                                     in the workspace; the backward entry points reject it */
 } cola_mode_t;
 
@@ -287,7 +287,12 @@ typedef struct {
     int32_t count;      /* GEMMs (or reductions) this one launch runs, 1..4 */
     int32_t mnk[4][3];  /* M, N, K of each (reductions: M, N, splits) */
     int32_t splits;     /* token splits (weight gradients), else 1 */
-    int32_t flags;      /* bit 0: the epilogue also wrote H (CoLA forward or CoLA-M backward) */
+    int32_t flags;      /* bit 0: the epilogue also wrote H (CoLA forward or CoLA-M backward);
+                           bit 1: a forward GEMM split over K into fp32 partials (the reduce
+                                  launch after it applies the epilogue);
+                           bit 2: the GEMM ran on CTA pairs (clusters of two CTAs, tcgen05
+                                  cta_group::2, 256-row tiles);
+                           bit 3: one CTA ran two 128-row sub-tiles sharing each B tile */
 } cola_trace_slot_t;
 
 cola_status_t cola_trace_attach(cola_trace_slot_t* slots, int32_t capacity, int32_t* count);

@@ -195,6 +195,25 @@ void oracle_bwd(long n, long d_in, long d_out, long r, int sigma, int mode, int 
     free(Hb);
 }
 
+/* ---- CoLA-M block-level recompute (Sec. 4.2, App. C) ----
+ * In the backward, CoLA-M rebuilds a layer output from the saved low-rank
+ * activation instead of keeping it: H = sigma(Z) elementwise, then
+ * Y[t,o] = sum_i H[t,i] B[o,i], the forward's second product. */
+void oracle_recompute_up(long n, long d_out, long r, int sigma, const double* Z, const double* B, double* Y)
+{
+    double* H = (double*)malloc(sizeof(double) * (size_t)(n * r));
+    for (long j = 0; j < n * r; ++j) H[j] = oracle_sigma(sigma, Z[j]);
+#pragma omp parallel for schedule(static)
+    for (long t = 0; t < n; ++t) {
+        for (long o = 0; o < d_out; ++o) {
+            double s = 0.0;
+            for (long i = 0; i < r; ++i) s += H[t * r + i] * B[o * r + i];
+            Y[t * d_out + o] = s;
+        }
+    }
+    free(H);
+}
+
 /* ---- sampled routines on bf16 inputs (large shapes) ----
  * X[t,k] at X[t*ld_x + k]; dY[t,o] at dY[t*ld_y + o]; A [r x d_in] and
  * B [d_out x r] dense.  Each routine computes only the requested outputs,

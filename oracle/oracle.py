@@ -64,6 +64,7 @@ def lib():
                                              _U16, _U16, _U16, _long, _long, _L, _L, _D]
         l.oracle_dB_entries_bf16.argtypes = [_long, _long, _long, _int, _int, _U16, _long, _U16,
                                              _U16, _long, _long, _L, _L, _D]
+        l.oracle_recompute_up.argtypes = [_long, _long, _long, _int, _D, _D, _D]
         l.oracle_num_threads.restype = _int
         _lib = l
     return _lib
@@ -167,12 +168,16 @@ def bwd(X, A, B, dY, Z, H=None, sigma="silu", mode="cola", round_store=False):
 
 def recompute_up(Z, B, sigma_kind="silu"):
     """CoLA-M's recompute of a layer output from its saved rank-r activation
-    (Sec. 4.2, App. C): Y = sigma(Z) B^T, sigma from the oracle's own fp64
-    routine, the product by numpy.  Returns Y [n x d_out]."""
-    Z, _ = _f64(Z)
-    B, _ = _f64(B)
-    assert Z.shape[1] == B.shape[1]
-    return sigma(sigma_kind, Z) @ B.T
+    (Sec. 4.2, App. C): H = sigma(Z), Y = H B^T, in the C loops.  Returns
+    Y [n x d_out]."""
+    Z, pz = _f64(Z)
+    B, pb = _f64(B)
+    n, r = Z.shape
+    d_out = B.shape[0]
+    assert B.shape == (d_out, r)
+    Y, py = _out((n, d_out))
+    lib().oracle_recompute_up(n, d_out, r, _sig(sigma_kind), pz, pb, py)
+    return Y
 
 
 def fwd_qkv(X, As, Bs, sigma="silu", round_store=False):

@@ -141,6 +141,18 @@ WgradPlan wgrad_plan(const cola_desc_t& d, int nproj, int sms)
     return plan_wgrad(M, N, nb + 1, d.n, sms);
 }
 
+// The split-tail schedule of the same group (bf16 gradients): the tile
+// configuration of wgrad_plan.  It runs when its cost is no higher than the
+// uniform token split's (tail_wins).
+TailPlan wgrad_tail_plan(const WgradPlan& w, int64_t ntok, int sms)
+{
+    GemmParams p[MAX_GROUP];
+    for (int j = 0; j < w.count; ++j) p[j] = base_params(w.p[j].M, w.p[j].N, ntok, w.bn, w.msub);
+    return plan_tail(p, w.count, w.bn, w.msub, sms);
+}
+
+bool tail_wins(const WgradPlan& w, const TailPlan& t) { return t.cost <= w.cost; }
+
 // fp32 partial elements the forward of `nproj` projections needs when its
 // GEMMs are small enough to be split over K (small_launch_splits)
 int64_t fwd_part_elems(const cola_desc_t& d, int nproj, int sms)
@@ -185,7 +197,11 @@ WsLayout ws_layout(const cola_desc_t& d, int nproj, int sms)
     size_t part = static_cast<size_t>(fwd_part_elems(d, nproj, sms)) * 4;
     if (d.mode != COLA_MODE_INFER) {
         const WgradPlan w = wgrad_plan(d, nproj, sms);
-        if (w.splits > 1 || d.wgrad_fp32) part = std::max(part, static_cast<size_t>(w.part_elems) * 4);
+        const TailPlan t = wgrad_tail_plan(w, d.n, sms);
+        if (!d.wgrad_fp32 && tail_wins(w, t))
+            part = std::max(part, static_cast<size_t>(t.part_elems) * 4);
+        else
+            part = std::max(part, static_cast<size_t>(w.part_elems) * 4);
     }
     off += align_up(part);
     L.total = off;
@@ -248,16 +264,30 @@ cudaError_t traced(int kind, int count, const int64_t (*mnk)[3], int splits, int
     return cudaSuccess;
 }
 
-// Launch a batch of `count` problems of one configuration, traced as one launch.
+// Launch a batch of `count` problems of one configuration, traced as one
+// launch; `tail` (EPI_TAIL only) is its split-tail schedule, with the
+// partial slots at tail_part.
 template <bool A_MN, bool B_MN, int EPI>
 cola_status_t run_batch(int kind, int bn, int msub, const GemmProblem* probs, const int64_t (*mnk)[3], int count,
-                        int flags, int sms, cudaStream_t st)
+                        int flags, int sms, cudaStream_t st, const TailPlan* tail = nullptr, float* tail_part = nullptr)
 {
     GemmBatch b;
     std::memset(&b, 0, sizeof b);
     b.count = count;
     for (int g = 0; g < count; ++g) b.prob[g] = probs[g];
-    return launched(traced(kind, count, mnk, probs[0].p.splits, flags, st,
+    int splits = probs[0].p.splits;
+    if (tail) {
+        b.tail_body = tail->body;
+        b.tail_tiles = tail->tail;
+        b.tail_pieces = tail->pieces;
+        b.tail_kps = tail->kps;
+        for (int g = 0; g < count; ++g) b.tile_begin[g] = tail->tile_begin[g];
+        b.tail_part = tail_part;
+        flags |= TRACE_TAIL;
+        splits = tail->pieces;
+    }
+    flags |= tile_flags<A_MN, EPI>(bn, msub);
+    return launched(traced(kind, count, mnk, splits, flags, st,
                            [&] { return dispatch<A_MN, B_MN, EPI>(bn, msub, b, sms, st); }));
 }
 
@@ -422,9 +452,11 @@ cola_status_t run_b1(const Shape& s, int sigma, int count, const void* const* dY
 
 // Weight gradients of one backward call, in one launch: D_j[M_j x N_j] =
 // sum_t P_j[t, m] Q_j[t, n] over the n tokens, both operands token-major
-// (MN-major).  Split over tokens into fp32 partial slabs (laid out one
-// gradient after another) reduced in a fixed order, or, unsplit, stored
-// directly as bf16.
+// (MN-major).  bf16 gradients run with a split tail (run_wgrad_tail) when
+// the planner's cost model prefers it; otherwise, and for fp32 gradients
+// accumulated into (D += ...), the token range of every tile is split
+// uniformly into fp32 partial slabs (laid out one gradient after another)
+// that the reduce adds, in a fixed order, into (onto) D.
 struct WgradJob {
     const void* P;
     int64_t ldp;
@@ -434,11 +466,15 @@ struct WgradJob {
     int64_t ldo;
 };
 
+cola_status_t run_wgrad_tail(const WgradPlan& w, int64_t ntok, const WgradJob* jobs, float* part, size_t part_bytes,
+                           unsigned int* status, int sms, cudaStream_t st);
+
 cola_status_t run_wgrad(const WgradPlan& w, int64_t ntok, const WgradJob* jobs, int accumulate_f32, float* part,
                         size_t part_bytes, unsigned int* status, int sms, cudaStream_t st)
 {
-    const bool direct = w.splits == 1 && !accumulate_f32;
-    if (!direct && static_cast<size_t>(w.part_elems) * 4 > part_bytes) return COLA_ERR_WORKSPACE;
+    if (!accumulate_f32 && tail_wins(w, wgrad_tail_plan(w, ntok, sms)))
+        return run_wgrad_tail(w, ntok, jobs, part, part_bytes, status, sms, st);
+    if (static_cast<size_t>(w.part_elems) * 4 > part_bytes) return COLA_ERR_WORKSPACE;
     GemmProblem pr[MAX_GROUP];
     int64_t mnk[MAX_GROUP][3];
     std::memset(pr, 0, sizeof pr);
@@ -451,32 +487,23 @@ cola_status_t run_wgrad(const WgradPlan& w, int64_t ntok, const WgradJob* jobs, 
         COLA_MAP(map_mnmajor(&pr[j].map_a, jobs[j].P, pj.M, ntok, jobs[j].ldp));
         COLA_MAP(map_mnmajor(&pr[j].map_b, jobs[j].Q, pj.N, ntok, jobs[j].ldq));
         pr[j].p.status = status;
-        if (direct) {
-            COLA_MAP(map_box32(&pr[j].map_d, jobs[j].out, pj.N, pj.M, jobs[j].ldo));
-            pr[j].p.d_ptr = static_cast<__nv_bfloat16*>(jobs[j].out);
-            pr[j].p.d_ld = jobs[j].ldo;
-        } else {
-            pr[j].map_d = pr[j].map_a;
-            pr[j].p.D = slab_base;
-            pr[j].p.ldd = static_cast<long long>(pj.n_tiles) * w.bn;
-            pr[j].p.part_stride = w.slab[j];
-            ReduceJob& rj = rb.job[j];
-            rj.part = slab_base;
-            rj.part_stride = w.slab[j];
-            rj.ldp = pj.n_tiles * w.bn;
-            rj.M = pj.M;
-            rj.N = pj.N;
-            rj.out = jobs[j].out;
-            rj.ldo = jobs[j].ldo;
-            slab_base += static_cast<int64_t>(pj.splits) * w.slab[j];
-        }
-        pr[j].map_d2 = pr[j].map_z = pr[j].map_d;
+        pr[j].map_d = pr[j].map_d2 = pr[j].map_z = pr[j].map_a;
+        pr[j].p.D = slab_base;
+        pr[j].p.ldd = static_cast<long long>(pj.n_tiles) * w.bn;
+        pr[j].p.part_stride = w.slab[j];
+        ReduceJob& rj = rb.job[j];
+        rj.part = slab_base;
+        rj.part_stride = w.slab[j];
+        rj.ldp = pj.n_tiles * w.bn;
+        rj.M = pj.M;
+        rj.N = pj.N;
+        rj.out = jobs[j].out;
+        rj.ldo = jobs[j].ldo;
+        slab_base += static_cast<int64_t>(pj.splits) * w.slab[j];
         mnk[j][0] = pj.M;
         mnk[j][1] = pj.N;
         mnk[j][2] = ntok;
     }
-    if (direct)
-        return run_batch<true, true, EPI_STORE>(COLA_KERNEL_WGRAD, w.bn, w.msub, pr, mnk, w.count, 0, sms, st);
     COLA_TRY((run_batch<true, true, EPI_F32>(COLA_KERNEL_WGRAD, w.bn, w.msub, pr, mnk, w.count, 0, sms, st)));
     rb.count = w.count;
     rb.splits = w.splits;
@@ -489,6 +516,50 @@ cola_status_t run_wgrad(const WgradPlan& w, int64_t ntok, const WgradJob* jobs, 
     }
     return launched(traced(COLA_KERNEL_REDUCE, w.count, rmnk, w.splits, 0, st,
                            [&] { return launch_splitk_reduce(rb, st); }));
+}
+
+// bf16 weight gradients with a split tail: the whole tiles are stored
+// straight from the GEMM epilogue; the pieces of the split tail tiles are
+// summed by the tail reduce (no reduce when the tail is not split).
+cola_status_t run_wgrad_tail(const WgradPlan& w, int64_t ntok, const WgradJob* jobs, float* part, size_t part_bytes,
+                           unsigned int* status, int sms, cudaStream_t st)
+{
+    const TailPlan tp = wgrad_tail_plan(w, ntok, sms);
+    if (static_cast<size_t>(tp.part_elems) * 4 > part_bytes) return COLA_ERR_WORKSPACE;
+    GemmProblem pr[MAX_GROUP];
+    int64_t mnk[MAX_GROUP][3];
+    std::memset(pr, 0, sizeof pr);
+    TailReduce rd;
+    std::memset(&rd, 0, sizeof rd);
+    for (int j = 0; j < w.count; ++j) {
+        pr[j].p = base_params(w.p[j].M, w.p[j].N, ntok, w.bn, w.msub);
+        const GemmParams& pj = pr[j].p;
+        COLA_MAP(map_mnmajor(&pr[j].map_a, jobs[j].P, pj.M, ntok, jobs[j].ldp));
+        COLA_MAP(map_mnmajor(&pr[j].map_b, jobs[j].Q, pj.N, ntok, jobs[j].ldq));
+        COLA_MAP(map_box32(&pr[j].map_d, jobs[j].out, pj.N, pj.M, jobs[j].ldo));
+        pr[j].map_d2 = pr[j].map_z = pr[j].map_d;
+        pr[j].p.d_ptr = static_cast<__nv_bfloat16*>(jobs[j].out);
+        pr[j].p.d_ld = jobs[j].ldo;
+        pr[j].p.status = status;
+        mnk[j][0] = pj.M;
+        mnk[j][1] = pj.N;
+        mnk[j][2] = ntok;
+        rd.out[j] = jobs[j].out;
+        rd.ldo[j] = jobs[j].ldo;
+        rd.M[j] = pj.M;
+        rd.N[j] = pj.N;
+    }
+    COLA_TRY((run_batch<true, true, EPI_TAIL>(COLA_KERNEL_WGRAD, w.bn, w.msub, pr, mnk, w.count, 0, sms, st, &tp,
+                                             part)));
+    if (tp.ntiles == 0) return COLA_OK;
+    rd.part = part;
+    rd.tile_rows = tile_rows(w.msub);
+    rd.tile_cols = w.bn;
+    rd.ntiles = tp.ntiles;
+    for (int t = 0; t < tp.ntiles; ++t) rd.tile[t] = tp.tile[t];
+    const int64_t rmnk[1][3] = {{static_cast<int64_t>(tp.ntiles) * rd.tile_rows, rd.tile_cols, tp.pieces}};
+    return launched(traced(COLA_KERNEL_REDUCE, 1, rmnk, tp.pieces, TRACE_TAIL, st,
+                           [&] { return launch_tail_reduce(rd, sms, st); }));
 }
 
 // B4: dX = dZ A  (dZ [n x K] pitch ldz, A [K x d_in] pitch ld_a; K = r or 3r)

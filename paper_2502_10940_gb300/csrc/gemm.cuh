@@ -37,8 +37,13 @@
 //   EPI_DSIGMA  dZ = bf16(acc * sigma'(Z_saved)); with CoLA-M also
 //               H = bf16(sigma(Z_saved)) for the weight gradient of B
 //   EPI_F32     fp32 split-K partial slab, reduced (in a fixed order) by the
-//               reduce kernel: the weight gradients, and the forward GEMMs of
-//               small launches
+//               reduce kernel: fp32-accumulated weight gradients, and the
+//               forward GEMMs of small launches
+//   EPI_TAIL      weight gradients (bf16 D) with a split tail: the tiles of
+//               the full waves run whole and store D = bf16(acc) as
+//               EPI_STORE; the tiles of the last, partial wave are split
+//               over K into pieces that store fp32 partials into slots, which
+//               the tail reduce sums in a fixed order
 //
 // Every mbarrier wait is bounded (WAIT_LIMIT_NS of global time).  On expiry
 // the waiting thread records where it gave up in the status word, raises a
@@ -68,7 +73,7 @@ enum : unsigned int {
     ST_TIMEOUT_DRAIN = 1u << 3,
 };
 
-enum Epi : int { EPI_STORE = 0, EPI_ZH = 1, EPI_DSIGMA = 2, EPI_F32 = 3 };
+enum Epi : int { EPI_STORE = 0, EPI_ZH = 1, EPI_DSIGMA = 2, EPI_F32 = 3, EPI_TAIL = 4 };
 enum Sigma : int { SIG_IDENTITY = 0, SIG_SILU = 1, SIG_GELU = 2 };
 
 struct GemmParams {
@@ -232,10 +237,22 @@ struct GemmProblem {
 // Up to MAX_GROUP independent GEMMs of one configuration (tile shape,
 // operand majors, epilogue) run by a single persistent launch; their work
 // units are numbered consecutively, problem after problem.
+//
+// EPI_TAIL (split tail): the problems share K; their output tiles, problem
+// after problem and row-major within one, are numbered batch-wide
+// (tile_begin[g] is the first tile of problem g).  Units [0, tail_body) are
+// the whole tiles 0 .. tail_body - 1 (the full waves), followed by the
+// tail_tiles tiles of the last wave in tail_pieces pieces each: unit tail_body + j is
+// piece j % tail_pieces of tile tail_body + j / tail_pieces, k-blocks
+// [piece * tail_kps, +tail_kps) clipped to K.  With tail_pieces > 1 piece j
+// stores its fp32 partial into slot j (TILE_M x BN fp32) of tail_part.
 struct GemmBatch {
     GemmProblem prob[MAX_GROUP];
     int count;
     int units;
+    int tail_body, tail_tiles, tail_pieces, tail_kps;
+    int tile_begin[MAX_GROUP];
+    float* tail_part;
 };
 
 struct Unit {
@@ -252,6 +269,60 @@ __device__ __forceinline__ Unit decode(const GemmBatch& b, int u)
     x.g = g;
     decode_unit(b.prob[g].p, u - b.prob[g].unit_begin, x.m_blk, x.n_blk, x.split, x.kb0, x.kb1);
     return x;
+}
+
+// This CTA's walk over its work: units u = first_unit, first_unit + step,
+// ...  The producer, MMA and epilogue roles walk the same sequence.
+struct WorkIter {
+    int u;   // next unit
+};
+
+template <int EPI>
+__device__ __forceinline__ void work_begin(const GemmBatch&, int first_unit, WorkIter& it)
+{
+    it.u = first_unit;
+}
+
+// The next unit of the walk; false once the walk is over.  EPI_TAIL: a unit
+// that covers its whole tile has split = -1, a piece of a split tail tile
+// has split = its partial slot.
+template <int EPI>
+__device__ __forceinline__ bool work_next(const GemmBatch& b, int unit_step, WorkIter& it, Unit& x)
+{
+    if (it.u >= b.units) return false;
+    const int u = it.u;
+    it.u += unit_step;
+    if constexpr (EPI == EPI_TAIL) {
+        int t, k0 = 0, split = -1;
+        int k1 = b.prob[0].p.k_blocks;
+        if (u < b.tail_body) {
+            t = u;
+        } else {
+            const int j = u - b.tail_body;
+            const int piece = j % b.tail_pieces;
+            t = b.tail_body + j / b.tail_pieces;
+            if (b.tail_pieces > 1) {
+                k0 = piece * b.tail_kps;
+                k1 = min(k1, k0 + b.tail_kps);
+                split = j;
+            }
+        }
+        int g = 0;
+#pragma unroll
+        for (int q = 1; q < MAX_GROUP; ++q)
+            if (q < b.count && t >= b.tile_begin[q]) g = q;
+        const int rem = t - b.tile_begin[g];
+        const int nt = b.prob[g].p.n_tiles;
+        x.g = g;
+        x.m_blk = rem / nt;
+        x.n_blk = rem - x.m_blk * nt;
+        x.split = split;
+        x.kb0 = k0;
+        x.kb1 = k1;
+    } else {
+        x = decode(b, u);
+    }
+    return true;
 }
 
 __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi)
@@ -369,8 +440,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             long long issued = 0;
             bool ok = true;
             const bool no_loads = batch.prob[0].p.selftest_no_loads != 0;
-            for (int u = first_unit; u < batch.units && ok && !no_loads; u += unit_step) {
-                const Unit x = decode(batch, u);
+            WorkIter it;
+            work_begin<EPI>(batch, first_unit, it);
+            Unit x;
+            while (ok && !no_loads && work_next<EPI>(batch, unit_step, it, x)) {
                 const CUtensorMap* map_a = &batch.prob[x.g].map_a;
                 const CUtensorMap* map_b = &batch.prob[x.g].map_b;
                 // this CTA's rows of A and columns of B
@@ -474,8 +547,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             uint32_t bphase = 0;
             bool ok = true;
             bool issued_any = false;
-            for (int u = first_unit; u < batch.units && ok; u += unit_step) {
-                const Unit x = decode(batch, u);
+            WorkIter it;
+            work_begin<EPI>(batch, first_unit, it);
+            Unit x;
+            while (ok && work_next<EPI>(batch, unit_step, it, x)) {
                 const int kb0 = x.kb0, kb1 = x.kb1;
                 if (!wait_bounded<PAIR>(&tempty_bar[buf], bphase ^ 1u, wc, ST_TIMEOUT_MMA)) {
                     ok = false;
@@ -564,11 +639,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         uint32_t bphase = 0;
         bool ok = true;
 
-        // 32-column chunks of unit u that hold output rows of this warp
-        auto chunk_count = [&](int u) {
-            const Unit x = decode(batch, u);
+        // 32-column chunks of unit x that hold output rows of this warp
+        auto chunk_count = [&](const Unit& x) {
             const GemmParams& pu = batch.prob[x.g].p;
-            if (EPI == EPI_F32) return BN / 32;
+            if (EPI == EPI_F32 || (EPI == EPI_TAIL && x.split >= 0)) return BN / 32;   // partial tiles: all of it
             if (x.m_blk * TILE_M + row_off + sub * BM + q * 32 >= pu.M) return 0;   // this warp's 32 rows are all past the end
             const int left = pu.N - x.n_blk * BN;
             return left >= BN ? BN / 32 : (left + 31) / 32;
@@ -600,7 +674,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         uint32_t zphase = 0;                    // bit b: parity of the next wait on zbar[b]
         int zload = 0, zuse = 0;
         auto z_advance = [&]() {                // move (zu, zc) to the next item that has a chunk
-            while (zu < batch.units && zc >= chunk_count(zu)) {
+            while (zu < batch.units && zc >= chunk_count(decode(batch, zu))) {
                 zu += unit_step;
                 zc = c_first;
             }
@@ -624,8 +698,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             z_issue();
         }
 
-        for (int u = first_unit; u < batch.units && ok; u += unit_step) {
-            const Unit x = decode(batch, u);
+        WorkIter it;
+        work_begin<EPI>(batch, first_unit, it);
+        Unit x;
+        while (ok && work_next<EPI>(batch, unit_step, it, x)) {
             const GemmParams& p = batch.prob[x.g].p;
             const CUtensorMap* map_d = &batch.prob[x.g].map_d;
             const CUtensorMap* map_d2 = &batch.prob[x.g].map_d2;
@@ -633,7 +709,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             cur_M = p.M;
             const int row0 = m_blk * TILE_M + row_off + sub * BM + q * 32;
             const int row = row0 + lane;
-            const int nch = chunk_count(u);
+            const int nch = chunk_count(x);
             if (!wait_bounded(&tfull_bar[buf], bphase, wc, ST_TIMEOUT_EPILOGUE)) break;
             tc_fence_after();
             const uint32_t tbase = tmem_base + (static_cast<uint32_t>(q * 32) << 16) +
@@ -645,10 +721,17 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                 uint32_t v[32];
                 tmem_ld_32x32b_x32(tbase + c * 32, v);
                 tmem_ld_wait();
-                if (EPI == EPI_F32) {
-                    if (row < p.M) {                // rows past the last one: the reduce never reads them
-                        float* dst = reinterpret_cast<float*>(p.D) + split * p.part_stride +
-                                     static_cast<long long>(m_blk * TILE_M + row_in_tile) * p.ldd + col0;
+                if (EPI == EPI_F32 || (EPI == EPI_TAIL && split >= 0)) {
+                    float* dst = nullptr;
+                    if (EPI == EPI_F32) {
+                        if (row < p.M)              // rows past the last one: the reduce never reads them
+                            dst = reinterpret_cast<float*>(p.D) + split * p.part_stride +
+                                  static_cast<long long>(m_blk * TILE_M + row_in_tile) * p.ldd + col0;
+                    } else {                        // the piece's partial slot: one whole TILE_M x BN tile
+                        dst = batch.tail_part + static_cast<long long>(split) * (TILE_M * BN) +
+                              static_cast<long long>(row_in_tile) * BN + c * 32;
+                    }
+                    if (dst) {
                         float4* d4 = reinterpret_cast<float4*>(dst);
 #pragma unroll
                         for (int j = 0; j < 8; ++j)
@@ -658,7 +741,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                     continue;
                 }
                 uint32_t w[16];
-                if (EPI == EPI_STORE) {
+                if (EPI == EPI_STORE || EPI == EPI_TAIL) {
 #pragma unroll
                     for (int j = 0; j < 16; ++j)
                         w[j] = pack_bf16x2(__uint_as_float(v[2 * j]), __uint_as_float(v[2 * j + 1]));

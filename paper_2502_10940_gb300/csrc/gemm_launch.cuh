@@ -43,6 +43,30 @@ struct ReduceBatch {
 
 cudaError_t launch_splitk_reduce(ReduceBatch& batch, cudaStream_t stream);
 
+// The tail reduce of an EPI_TAIL launch: each split tail tile is the sum of
+// its pieces' partial slots, added in piece order (so the result is
+// deterministic), stored as bf16 into its problem's output.
+constexpr int MAX_TAIL_TILES = 160;   // tail tiles are fewer than the CTA slots (<= 151 on GB300)
+
+struct TailTile {
+    int g;          // problem
+    int m0, n0;     // first row and column of the tile in the problem's output
+    int lo_slot;    // partial slot of its first piece; the others follow it
+    int count;      // pieces
+};
+
+struct TailReduce {
+    const float* part;              // partial slots of tile_rows x tile_cols fp32 each
+    int tile_rows, tile_cols;
+    void* out[MAX_GROUP];           // bf16 outputs of the launch's problems
+    long long ldo[MAX_GROUP];
+    int M[MAX_GROUP], N[MAX_GROUP];
+    int ntiles;
+    TailTile tile[MAX_TAIL_TILES];
+};
+
+cudaError_t launch_tail_reduce(const TailReduce& r, int sms, cudaStream_t stream);
+
 // H = bf16(sigma(Z)) elementwise over `elems` bf16 values (a multiple of 8;
 // both pointers 16-byte aligned).
 cudaError_t launch_sigma(const void* Z, void* H, long long elems, int sigma, int sms, cudaStream_t stream);

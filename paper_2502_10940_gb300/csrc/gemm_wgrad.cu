@@ -1,10 +1,12 @@
 // Weight-gradient GEMMs dB = dY^T H and dA = dZ^T X: the reduction runs over
-// the n tokens, both operands are token-major activations read MN-major, and
-// the token range is split across CTAs into fp32 partial slabs that
-// splitk_reduce_kernel sums in a fixed order (or, unsplit, the epilogue
-// stores the bf16 gradient directly).  The same reduce finishes the split-K
-// forward GEMMs of small launches (instantiated here too), applying the Z/H
-// epilogue for the Z GEMM.
+// the n tokens, and both operands are token-major activations read MN-major.
+// bf16 gradients either run their tiles whole in waves and split only the
+// tiles of the last, partial wave over the tokens (EPI_TAIL; tail_reduce_kernel
+// sums the pieces), or split every tile's token range uniformly into fp32
+// partial slabs that splitk_reduce_kernel sums in a fixed order; fp32
+// gradients accumulated into always take the uniform split.  The same
+// reduce finishes the split-K forward GEMMs of small launches (instantiated
+// here too), applying the Z/H epilogue for the Z GEMM.
 #define COLA_DEFINE_LAUNCHERS
 #include "gemm_launch.cuh"
 
@@ -88,6 +90,73 @@ __global__ void __launch_bounds__(RED_THREADS) splitk_reduce_kernel(const __grid
     }
 }
 
+// ------------------------------------------------ tail reduction
+// Every element of a split tail tile is the sum, in piece order, of its
+// pieces' partial slots: one thread per 4 consecutive columns of one row,
+// bf16 store of the columns inside the output.
+__global__ void __launch_bounds__(RED_THREADS) tail_reduce_kernel(const __grid_constant__ TailReduce r)
+{
+    grid_dependency_wait();            // the partials come from the GEMM launched just before
+    grid_launch_dependents();
+    const int groups_per_row = r.tile_cols / 4;
+    const long long per_tile = static_cast<long long>(r.tile_rows) * groups_per_row;
+    const long long total = per_tile * r.ntiles;
+    const long long slot_elems = static_cast<long long>(r.tile_rows) * r.tile_cols;
+    const long long stride = static_cast<long long>(gridDim.x) * RED_THREADS;
+    for (long long e = static_cast<long long>(blockIdx.x) * RED_THREADS + threadIdx.x; e < total; e += stride) {
+        const int k = static_cast<int>(e / per_tile);
+        const int local = static_cast<int>(e - static_cast<long long>(k) * per_tile);
+        const int i = local / groups_per_row;
+        const int j = (local - i * groups_per_row) * 4;
+        const TailTile& t = r.tile[k];
+        const int row = t.m0 + i, col = t.n0 + j;
+        if (row >= r.M[t.g] || col >= r.N[t.g]) continue;
+        const float* src = r.part + static_cast<long long>(i) * r.tile_cols + j;
+        float4 acc = __ldg(reinterpret_cast<const float4*>(src + t.lo_slot * slot_elems));
+        for (int q = 1; q < t.count; ++q) {
+            const float4 v = __ldg(reinterpret_cast<const float4*>(src + (t.lo_slot + q) * slot_elems));
+            acc.x += v.x;
+            acc.y += v.y;
+            acc.z += v.z;
+            acc.w += v.w;
+        }
+        const float v[4] = {acc.x, acc.y, acc.z, acc.w};
+        const int valid = min(4, r.N[t.g] - col);
+        __nv_bfloat16* o = reinterpret_cast<__nv_bfloat16*>(r.out[t.g]) + static_cast<long long>(row) * r.ldo[t.g] + col;
+        if (valid == 4 && ((reinterpret_cast<uintptr_t>(o) & 7) == 0)) {
+            *reinterpret_cast<uint2*>(o) = make_uint2(pack_bf16x2(v[0], v[1]), pack_bf16x2(v[2], v[3]));
+        } else {
+#pragma unroll
+            for (int e2 = 0; e2 < 4; ++e2)
+                if (e2 < valid) o[e2] = __float2bfloat16_rn(v[e2]);
+        }
+    }
+}
+
+cudaError_t launch_tail_reduce(const TailReduce& r, int sms, cudaStream_t stream)
+{
+    const long long groups = static_cast<long long>(r.ntiles) * r.tile_rows * (r.tile_cols / 4);
+    long long blocks = (groups + RED_THREADS - 1) / RED_THREADS;
+    if (blocks > 8LL * sms) blocks = 8LL * sms;
+    if (blocks < 1) blocks = 1;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(static_cast<unsigned>(blocks));
+    cfg.blockDim = dim3(RED_THREADS);
+    cfg.dynamicSmemBytes = 0;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, tail_reduce_kernel, r);
+}
+
+// bf16 weight gradients with a split tail (every tile configuration the planner picks)
+template cudaError_t launch_gemm<128, 1, true, true, EPI_TAIL>(const GemmBatch&, int, bool, cudaStream_t);
+template cudaError_t launch_gemm<256, 1, true, true, EPI_TAIL>(const GemmBatch&, int, bool, cudaStream_t);
+template cudaError_t launch_gemm<128, 2, true, true, EPI_TAIL>(const GemmBatch&, int, bool, cudaStream_t);
+template cudaError_t launch_gemm<256, 1, true, true, EPI_TAIL, true>(const GemmBatch&, int, bool, cudaStream_t);
 template cudaError_t launch_gemm<128, 1, true, true, EPI_STORE>(const GemmBatch&, int, bool, cudaStream_t);
 // split-K output GEMMs of small launches (both operands K-major)
 template cudaError_t launch_gemm<128, 1, false, false, EPI_F32>(const GemmBatch&, int, bool, cudaStream_t);

@@ -200,6 +200,7 @@ struct WgradPlan {
     GemmParams p[MAX_GROUP];
     int64_t slab[MAX_GROUP];       // fp32 elements per split slab of each GEMM
     int64_t part_elems;            // all slabs of all splits
+    double cost;                   // choose_splits' cost of the chosen split
 };
 
 WgradPlan plan_wgrad(const int64_t* M, const int64_t* N, int count, int64_t ntok, int sms)
@@ -230,7 +231,108 @@ WgradPlan plan_wgrad(const int64_t* M, const int64_t* N, int count, int64_t ntok
         w.part_elems += static_cast<int64_t>(w.p[i].splits) * w.slab[i];
     }
     w.splits = w.p[0].splits;
+    {
+        const int rows = tile_rows(w.msub);
+        const double c_part = 8.0 * w.bn * rows / (128.0 * (rows + w.bn)) + 2.0;
+        const int sl = unit_slots(w.msub, sms);
+        const long long units = static_cast<long long>(tiles) * w.splits;
+        const long long waves = (units + sl - 1) / sl;
+        w.cost = static_cast<double>(waves) * (w.p[0].kb_per_split + (w.splits > 1 ? c_part : 0.0));
+    }
     return w;
+}
+
+// Split-tail schedule of a weight-gradient launch with bf16 outputs
+// (EPI_TAIL).  The output tiles run whole in waves of `slots` CTAs (CTA
+// pairs); the CTAs of a wave walk the token range in step, so the operand
+// panels their tiles share are read from HBM about once.  The R < slots
+// tiles of the last, partial wave are split over the tokens into `pieces`
+// pieces each (R x pieces <= slots, >= 4 k-blocks per piece), so that the
+// last wave is as short as the others allow; the tail reduce sums their
+// partial slots.  Only the tail tiles write fp32 partials.  (Walking every
+// CTA's equal share of all tile-and-token steps instead, stream-K style, was
+// measured 1.4 to 1.6x slower at 60M to 7B: the CTAs drift apart in the token
+// range, and the shared panels are then read from HBM once per tile.)
+struct TailPlan {
+    int body;                  // whole tiles (full waves)
+    int tail;                  // tiles of the last wave
+    int ntiles;                // tail tiles the reduce finishes (tail when split, else 0)
+    int pieces, kps;           // pieces per tail tile, k-blocks per piece
+    int units;                 // body + ntiles x pieces
+    int kb;
+    int tile_begin[MAX_GROUP];
+    int64_t part_elems;        // ntiles x pieces x tile_rows x bn fp32 (0 when pieces == 1)
+    double cost;               // k-blocks of the busiest CTA, plus the partial round trip
+    TailTile tile[MAX_TAIL_TILES];
+};
+
+TailPlan plan_tail(const GemmParams* p, int count, int bn, int msub, int sms)
+{
+    TailPlan s;
+    std::memset(&s, 0, sizeof s);
+    int tiles = 0;
+    for (int g = 0; g < count; ++g) {
+        s.tile_begin[g] = tiles;
+        tiles += p[g].m_tiles * p[g].n_tiles;
+    }
+    s.kb = p[0].k_blocks;
+    const int slots = unit_slots(msub, sms);
+    const int waves = tiles / slots;
+    const int R = tiles - waves * slots;
+    s.body = waves * slots;
+    s.tail = R;
+    s.pieces = 1;
+    s.kps = s.kb;
+    if (R > 0 && R <= MAX_TAIL_TILES) {
+        const int most = s.kb / 4 > 1 ? s.kb / 4 : 1;
+        int St = slots / R < most ? slots / R : most;
+        if (St > 1) {
+            s.kps = (s.kb + St - 1) / St;
+            St = (s.kb + s.kps - 1) / s.kps;   // no empty piece
+        }
+        s.pieces = St > 1 ? St : 1;
+        if (s.pieces == 1) s.kps = s.kb;
+    }
+    s.units = s.body + R * s.pieces;
+    const int rows = tile_rows(msub);
+    const double c_part = 8.0 * bn * rows / (128.0 * (rows + bn)) + 2.0;   // as in choose_splits
+    s.cost = static_cast<double>(waves) * s.kb + (R > 0 ? s.kps + (s.pieces > 1 ? c_part : 0.0) : 0.0);
+    if (s.pieces > 1) {
+        s.part_elems = static_cast<int64_t>(R) * s.pieces * rows * bn;
+        s.ntiles = R;
+        for (int i = 0; i < R; ++i) {
+            const int t = s.body + i;
+            int g = 0;
+            for (int j = 1; j < count; ++j)
+                if (t >= s.tile_begin[j]) g = j;
+            const int rem = t - s.tile_begin[g];
+            TailTile& e = s.tile[i];
+            e.g = g;
+            e.m0 = rem / p[g].n_tiles * rows;
+            e.n0 = rem % p[g].n_tiles * bn;
+            e.lo_slot = i * s.pieces;
+            e.count = s.pieces;
+        }
+    }
+    return s;
+}
+
+// The tile configuration dispatch() launches for a planned (bn, msub): bit 2
+// set when the launch runs on CTA pairs (clusters of two, cta_group::2), bit
+// 3 when one CTA runs two 128-row sub-tiles.  These are the launch-trace
+// flag bits of the same meaning (include/cola.h).
+constexpr int TRACE_PAIR = 4;
+constexpr int TRACE_MSUB2 = 8;
+constexpr int TRACE_TAIL = 16;   // weight gradients with a split tail
+
+template <bool A_MN, int EPI>
+int tile_flags(int bn, int msub)
+{
+    constexpr bool small_only = EPI == EPI_F32 && !A_MN;   // split-K forward partials: 128-row tiles only
+    if (small_only) return 0;
+    if (msub == TILE_PAIR && bn == 256) return TRACE_PAIR;
+    if (msub == 2 && bn == 128) return TRACE_MSUB2;
+    return 0;
 }
 
 // Launch one batch (all problems of one configuration).  Programmatic
@@ -247,6 +349,7 @@ cudaError_t dispatch(int bn, int msub, GemmBatch& b, int sms, cudaStream_t s)
         units += b.prob[g].p.units;
         flops += 2.0 * b.prob[g].p.M * b.prob[g].p.N * (static_cast<double>(b.prob[g].p.k_blocks) * BK);
     }
+    if constexpr (EPI == EPI_TAIL) units = b.tail_body + b.tail_tiles * b.tail_pieces;
     b.units = units;
     const bool pdl = flops < 64e9;
     // the split-K forward GEMMs of small launches (K-major fp32 partials) run

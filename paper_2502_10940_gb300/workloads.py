@@ -100,7 +100,7 @@ WORKLOADS = {
                         "(128 x 256)", seqs=128),
     "1b-o": Workload("1b-o", 65536, (Layer("o", 2048, 2048, 512, "x_o"),), fused_qkv=False,
                      desc="single CoLA layer, LLaMA-1B o-proj shape, 65536 tokens, 2048->2048, r=512", seqs=256),
-    # inference at the pre-training shapes with 32 sequences of 256 tokens (Table 10)
+    # inference at the pre-training shapes with 32 sequences of 256 tokens (App. E.2)
     "1b-infer": Workload("1b-infer", 8192, llama_block(2048, 5461, 512), modes=("infer",), phase="infer", desc="LLaMA-1B-shaped CoLA block, forward only (inference), d=2048, "
                                           "d_ff=5461, r=512, 8192 tokens (32 x 256)", seqs=32),
     "7b-infer": Workload("7b-infer", 8192, llama_block(4096, 11008, 1024), modes=("infer",), phase="infer", desc="LLaMA-7B-shaped CoLA block, forward only (inference), d=4096, "
