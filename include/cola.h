@@ -220,6 +220,25 @@ cola_status_t cola_check_status(void* ws, void* stream, uint32_t* code_out);
  * CUDA context stays usable.  Async on `stream`. */
 cola_status_t cola_selftest_wait_timeout(void* ws, size_t ws_bytes, void* stream);
 
+/* The same self-test on a CTA pair (tcgen05 cta_group::2, the tile of the
+ * compute-heavy GEMMs): one 256 x 256 x 512 GEMM whose operands (zeros) and
+ * output lie in ws after its status header (ws_bytes >= 256 + 640 KB).
+ *   variant 1: neither CTA's TMA producer issues a load; the even CTA's MMA
+ *              issuer and the odd CTA's epilogue give up after 2 s.
+ *   variant 2: the odd CTA's producer issues its first k-block only, while
+ *              the even CTA's producer fills its whole ring; the MMA
+ *              issuer's second wait runs out with the even CTA's loads of
+ *              six more stages landed or in flight.  Before the pair exits,
+ *              the even CTA must see every load of both CTAs land (the abort
+ *              drain of a pair), or it records COLA_STATUS_DRAIN_TIMEOUT.
+ * The next cola_check_status on ws returns COLA_ERR_DEVICE_TIMEOUT with some
+ * of COLA_STATUS_PRODUCER_TIMEOUT, COLA_STATUS_MMA_TIMEOUT and
+ * COLA_STATUS_EPILOGUE_TIMEOUT set and, when the drain saw every load land,
+ * not COLA_STATUS_DRAIN_TIMEOUT.  Nothing is stored (ws beyond the status
+ * word is only read), and the CUDA context stays usable.  Async on `stream`;
+ * variant outside {1, 2}: COLA_ERR_INVALID. */
+cola_status_t cola_selftest_wait_timeout_pair(void* ws, size_t ws_bytes, int32_t variant, void* stream);
+
 /* ---- weight gradient without any workspace or allocation ----
  * The paper has no counterpart to this entry point.  It serves callers that
  * cannot allocate device memory: an operator or plugin interface that hands

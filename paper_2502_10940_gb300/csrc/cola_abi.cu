@@ -806,9 +806,35 @@ cola_status_t cola_selftest_wait_timeout(void* ws, size_t ws_bytes, void* stream
     pr.p.d_ptr = reinterpret_cast<__nv_bfloat16*>(base + 2 * tile_bytes);
     pr.p.d_ld = 128;
     pr.p.status = ws_status(ws);
-    pr.p.selftest_no_loads = 1;
+    pr.p.selftest = 1;
     const int64_t mnk[1][3] = {{128, 128, 64}};
     return run_batch<false, false, EPI_STORE>(COLA_KERNEL_FWD_Y, 128, 1, &pr, mnk, 1, 0, sms,
+                                              static_cast<cudaStream_t>(stream));
+}
+
+cola_status_t cola_selftest_wait_timeout_pair(void* ws, size_t ws_bytes, int32_t variant, void* stream)
+{
+    if (!ws || (variant != 1 && variant != 2)) return COLA_ERR_INVALID;
+    if (reinterpret_cast<uintptr_t>(ws) & (WS_ALIGN - 1)) return COLA_ERR_ALIGN;
+    constexpr int64_t M = 256, N = 256, K = 512;   // one 256 x 256 pair tile, 8 k-blocks
+    constexpr size_t a_bytes = M * K * 2, b_bytes = N * K * 2, d_bytes = M * N * 2;
+    if (ws_bytes < WS_HEADER + a_bytes + b_bytes + d_bytes) return COLA_ERR_WORKSPACE;
+    int sms = 0;
+    COLA_TRY(device_info(&sms));
+    uint8_t* base = wsb(ws) + WS_HEADER;
+    GemmProblem pr;
+    std::memset(&pr, 0, sizeof pr);
+    pr.p = base_params(M, N, K, 256, TILE_PAIR);
+    COLA_MAP(map_kmajor(&pr.map_a, base, K, M, K, a_box_rows(TILE_PAIR)));
+    COLA_MAP(map_kmajor(&pr.map_b, base + a_bytes, K, N, K, b_box_rows(256, TILE_PAIR)));
+    COLA_MAP(map_box32(&pr.map_d, base + a_bytes + b_bytes, N, M, N));
+    pr.map_d2 = pr.map_z = pr.map_d;
+    pr.p.d_ptr = reinterpret_cast<__nv_bfloat16*>(base + a_bytes + b_bytes);
+    pr.p.d_ld = N;
+    pr.p.status = ws_status(ws);
+    pr.p.selftest = variant;
+    const int64_t mnk[1][3] = {{M, N, K}};
+    return run_batch<false, false, EPI_STORE>(COLA_KERNEL_FWD_Y, 256, TILE_PAIR, &pr, mnk, 1, 0, sms,
                                               static_cast<cudaStream_t>(stream));
 }
 

@@ -50,6 +50,17 @@
 // CTA-wide abort flag that makes every other wait return, waits (bounded) for
 // its own copies and MMAs still in flight, and the CTA frees its TMEM and
 // exits.  No wait can spin forever.
+//
+// On a CTA pair the odd CTA's TMA loads complete on the even CTA's stage
+// barriers, so it cannot see them land itself.  At the end of the producer
+// role the odd producer reports how many k-blocks it issued (a store into
+// the even CTA's shared memory, published by a cluster-scope release arrive
+// on the even CTA's exchange barrier) and waits for the even CTA's relay.
+// The even producer, after an abort, reconciles the stage phases that the two
+// producers left unequal -- it arms the phases only the odd CTA issued (for
+// the odd CTA's bytes) and completes the odd CTA's share of the phases only
+// it issued -- waits for every phase still outstanding, so that every load of
+// either CTA has landed, and then arrives on the odd CTA's relay barrier.
 #pragma once
 #include <cuda_bf16.h>
 #include <cstdint>
@@ -95,7 +106,11 @@ struct GemmParams {
     long long d_ld;
     int sigma;
     unsigned int* status;
-    int selftest_no_loads;   // problem 0 only: the producer issues nothing, so the MMA's first wait runs out
+    // problem 0 only, for the failure-detection self-tests: 1 = the producers
+    // issue nothing, so the MMA's first wait runs out; 2 = the odd CTA of a
+    // pair issues its first k-block only, so the MMA's second wait runs out
+    // with the even CTA's loads of later stages in flight or landed
+    int selftest;
 };
 
 // Epilogue staging: per epilogue warp two 2 KB boxes of 32 rows x 32 bf16
@@ -124,7 +139,7 @@ struct GemmCfg {
     static constexpr int A_BYTES = CTA_ROWS * BK * 2;
     static constexpr int B_BYTES = B_ROWS * BK * 2;
     static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
-    static constexpr int BAR_BYTES = 512;        // 37 mbarriers, the TMEM address and the abort flag
+    static constexpr int BAR_BYTES = 512;        // 39 mbarriers, the TMEM address, the abort flag, a count
     static constexpr int SMEM_LIMIT = 232448;   // opt-in maximum per CTA
     static constexpr int STAGES_FIT = (SMEM_LIMIT - 1024 - BAR_BYTES - EPI_SMEM_BYTES) / STAGE_BYTES;
     static constexpr int STAGES = STAGES_FIT > 8 ? 8 : STAGES_FIT;
@@ -378,8 +393,11 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     uint64_t* tempty_bar = tfull_bar + 2;      // [2]
     uint64_t* drain_bar = tempty_bar + 2;      // [1]
     uint64_t* zfull_bar = drain_bar + 1;       // [NUM_EPI_WARPS][2]  Z boxes (EPI_DSIGMA)
-    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(zfull_bar + 2 * NUM_EPI_WARPS);
+    uint64_t* xchg_bar = zfull_bar + 2 * NUM_EPI_WARPS;   // [1] PAIR: the odd producer's report (even CTA)
+    uint64_t* relay_bar = xchg_bar + 1;        // [1] PAIR: the even CTA's drain is done (odd CTA)
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(relay_bar + 1);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+    volatile int* odd_issued = reinterpret_cast<volatile int*>(tmem_slot + 2);   // PAIR: written by the odd CTA
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
@@ -402,7 +420,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         }
         mbar_init(drain_bar, 1);
         for (int j = 0; j < 2 * NUM_EPI_WARPS; ++j) mbar_init(&zfull_bar[j], 1);
+        mbar_init(xchg_bar, 1);
+        mbar_init(relay_bar, 1);
         *abort_flag = 0;
+        *odd_issued = 0;
         fence_mbar_init();
         for (int g = 0; g < batch.count; ++g) {
             tma_prefetch_desc(&batch.prob[g].map_a);
@@ -439,17 +460,24 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             uint32_t phase = 0;
             long long issued = 0;
             bool ok = true;
-            const bool no_loads = batch.prob[0].p.selftest_no_loads != 0;
+            const int selftest = batch.prob[0].p.selftest;
+            const bool no_loads = selftest == 1;
+            const long long load_limit = (PAIR && !leader && selftest == 2) ? 1 : (1ll << 62);
+            bool stop = false;
             WorkIter it;
             work_begin<EPI>(batch, first_unit, it);
             Unit x;
-            while (ok && !no_loads && work_next<EPI>(batch, unit_step, it, x)) {
+            while (ok && !stop && !no_loads && work_next<EPI>(batch, unit_step, it, x)) {
                 const CUtensorMap* map_a = &batch.prob[x.g].map_a;
                 const CUtensorMap* map_b = &batch.prob[x.g].map_b;
                 // this CTA's rows of A and columns of B
                 const int m0 = x.m_blk * TILE_M + static_cast<int>(rank) * C::CTA_ROWS;
                 const int n0 = x.n_blk * BN + static_cast<int>(rank) * C::B_ROWS;
                 for (int kb = x.kb0; kb < x.kb1; ++kb) {
+                    if (issued >= load_limit) {
+                        stop = true;
+                        break;
+                    }
                     if (!wait_bounded(&empty_bar[stage], phase ^ 1u, wc, ST_TIMEOUT_PRODUCER)) {
                         ok = false;
                         break;
@@ -499,29 +527,29 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                     }
                 }
             }
-            if (ok && !*abort_flag) {
-                // tail: acquire every stage once more, i.e. wait until the MMA warp
-                // has released (its commits have arrived on) all of them
+            // normal: every k-block of the walk issued, and the MMA warp has
+            // released (its commits have arrived on) every stage since
+            bool normal = ok && !*abort_flag;
+            const int stage_end = stage;      // where the walk's last issue left the ring
+            const uint32_t phase_end = phase;
+            if (normal) {
+                // tail: acquire every stage once more
                 for (int j = 0; j < STAGES; ++j) {
-                    if (!wait_bounded(&empty_bar[stage], phase ^ 1u, wc, ST_TIMEOUT_PRODUCER)) break;
+                    if (!wait_bounded(&empty_bar[stage], phase ^ 1u, wc, ST_TIMEOUT_PRODUCER)) {
+                        normal = false;
+                        break;
+                    }
                     if (++stage == STAGES) {
                         stage = 0;
                         phase ^= 1u;
                     }
                 }
-            } else {
-                // drain: the last min(issued, STAGES) loads may still be landing.
-                // The odd CTA of a pair cannot observe its loads (they count on
-                // the even CTA's barriers): it gives them a fixed 50 us.
-                if (PAIR && !leader) {
-                    const uint64_t t0 = global_timer_ns();
-                    while (global_timer_ns() - t0 < 50000ull) {
-                    }
-                    issued = 0;
-                }
+            }
+            if (!normal && !PAIR) {
+                // drain: the last min(issued, STAGES) loads may still be landing
                 const int outstanding = issued < STAGES ? static_cast<int>(issued) : STAGES;
-                int s = stage;
-                uint32_t ph = phase;
+                int s = stage_end;
+                uint32_t ph = phase_end;
                 for (int j = 0; j < outstanding; ++j) {
                     if (--s < 0) {
                         s = STAGES - 1;
@@ -534,6 +562,51 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                             break;
                         }
                     }
+                }
+            }
+            if (PAIR) {
+                if (!leader) {
+                    // report the k-blocks issued to the even CTA, whose stage barriers
+                    // count them, and wait until it has seen every one of them land
+                    st_shared_cluster_u32(mapa_shared(smem_u32(const_cast<int*>(odd_issued)), 0),
+                                          static_cast<uint32_t>(issued));
+                    mbar_arrive_cluster(mapa_shared(smem_u32(xchg_bar), 0));
+                    const uint64_t t0 = global_timer_ns();
+                    while (!mbar_try_wait_cluster(relay_bar, 0)) {
+                        if (global_timer_ns() - t0 > 4 * WAIT_LIMIT_NS) {
+                            if (status) atomicOr(status, ST_TIMEOUT_DRAIN);
+                            break;
+                        }
+                    }
+                } else {
+                    bool got = true;
+                    const uint64_t t0 = global_timer_ns();
+                    while (!mbar_try_wait_cluster(xchg_bar, 0)) {
+                        if (global_timer_ns() - t0 > 2 * WAIT_LIMIT_NS) {
+                            if (status) atomicOr(status, ST_TIMEOUT_DRAIN);
+                            got = false;
+                            break;
+                        }
+                    }
+                    if (got && !normal) {
+                        // k-block q of the walk used stage q % STAGES in phase q / STAGES
+                        const long long L = issued, O = *odd_issued;
+                        const long long Q = L > O ? L : O;
+                        for (long long q = O; q < L; ++q)   // the odd CTA's share will not come
+                            mbar_complete_tx(&full_bar[q % STAGES], C::STAGE_BYTES);
+                        for (long long q = L; q < Q; ++q)   // only the odd CTA's share is coming
+                            mbar_arrive_expect_tx(&full_bar[q % STAGES], C::STAGE_BYTES);
+                        for (long long q = Q > STAGES ? Q - STAGES : 0; q < Q; ++q) {
+                            const uint64_t t1 = global_timer_ns();
+                            while (!mbar_try_wait(&full_bar[q % STAGES], static_cast<uint32_t>((q / STAGES) & 1))) {
+                                if (global_timer_ns() - t1 > WAIT_LIMIT_NS) {
+                                    if (status) atomicOr(status, ST_TIMEOUT_DRAIN);
+                                    break;
+                                }
+                            }
+                        }
+                    }
+                    mbar_arrive_cluster(mapa_shared(smem_u32(relay_bar), 1));
                 }
             }
         }

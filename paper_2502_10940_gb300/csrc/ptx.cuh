@@ -84,6 +84,21 @@ __device__ __forceinline__ void mbar_arrive_cluster(uint32_t cluster_addr)
     asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
 }
 
+// Count `bytes` transaction bytes as complete on `bar` without any copy:
+// stands in for a share of the expected bytes that will never arrive.
+__device__ __forceinline__ void mbar_complete_tx(uint64_t* bar, uint32_t bytes)
+{
+    asm volatile("mbarrier.complete_tx.relaxed.cta.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes)
+                 : "memory");
+}
+
+// Store a 32-bit value to the shared::cluster address `addr` (possibly in the
+// peer CTA); a following release arrive on the peer's barrier publishes it.
+__device__ __forceinline__ void st_shared_cluster_u32(uint32_t addr, uint32_t v)
+{
+    asm volatile("st.shared::cluster.u32 [%0], %1;" ::"r"(addr), "r"(v) : "memory");
+}
+
 // try_wait with cluster-scope acquire: for barriers that threads of the peer
 // CTA arrive on.
 __device__ __forceinline__ bool mbar_try_wait_cluster(uint64_t* bar, uint32_t parity)

@@ -172,6 +172,15 @@ def test_selftest_argument_errors(L):
     assert f(FAKE, 1024, None) == 4              # smaller than the status word plus three tiles
 
 
+def test_pair_selftest_argument_errors(L):
+    f = L.lib().cola_selftest_wait_timeout_pair
+    assert f(None, 1 << 20, 1, None) == 1
+    assert f(FAKE, 1 << 20, 0, None) == 1        # no such variant
+    assert f(FAKE, 1 << 20, 3, None) == 1
+    assert f(FAKE + 16, 1 << 20, 1, None) == 2   # not 256-byte aligned
+    assert f(FAKE, 4096, 2, None) == 4           # smaller than the status word plus the operands
+
+
 def test_workspace_init_and_check_reject_null(L):
     assert L.lib().cola_workspace_init(None, None) == 1
     assert L.lib().cola_workspace_init(FAKE + 16, None) == 2   # not 256-byte aligned
