@@ -214,6 +214,25 @@ void oracle_recompute_up(long n, long d_out, long r, int sigma, const double* Z,
     free(H);
 }
 
+/* ---- gated MLP (Fig. 4; Sec. 3.2; App. E) ----
+ * LLaMA's MLP multiplies its gate and up projections element-wise before the
+ * down projection; CoLA replaces both projections by auto-encoder layers and
+ * keeps the product (and no full-rank activation on the gate branch):
+ *   M = Y_gate (.) Y_up,   and for L = sum dM (.) M:
+ *   dY_gate = dM (.) Y_up,  dY_up = dM (.) Y_gate. */
+void oracle_gate_up_product(long m, const double* Yg, const double* Yu, double* M)
+{
+    for (long j = 0; j < m; ++j) M[j] = Yg[j] * Yu[j];
+}
+
+void oracle_gate_up_backward(long m, const double* dM, const double* Yg, const double* Yu, double* dYg, double* dYu)
+{
+    for (long j = 0; j < m; ++j) {
+        dYg[j] = dM[j] * Yu[j];
+        dYu[j] = dM[j] * Yg[j];
+    }
+}
+
 /* ---- sampled routines on bf16 inputs (large shapes) ----
  * X[t,k] at X[t*ld_x + k]; dY[t,o] at dY[t*ld_y + o]; A [r x d_in] and
  * B [d_out x r] dense.  Each routine computes only the requested outputs,

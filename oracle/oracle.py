@@ -13,6 +13,9 @@ Definitions followed (arXiv 2502.10940):
     they are three independent layers sharing X, and dX is their sum.
   * CoLA-M block recompute -- Sec. 4.2 / App. C: the up-projection B sigma(.)
     is recomputed in the backward from the saved Z: Y = sigma(Z) B^T.
+  * gated MLP -- Fig. 4, Sec. 3.2, App. E: the gate and up layers read one
+    x and their outputs are multiplied element-wise, M = Y_gate * Y_up (the
+    input of the down layer); backward dY_gate = dM * Y_up, dY_up = dM * Y_gate.
 
 Every function takes / returns numpy arrays.  Full routines take float64;
 the *_bf16 routines take bf16 bit patterns (uint16) and widen them exactly.
@@ -27,7 +30,7 @@ from .build import build as _build
 __all__ = [
     "SIGMA", "MODE", "lib", "sigma", "dsigma", "round_bf16", "widen_bf16",
     "fwd", "bwd", "fwd_qkv", "bwd_qkv", "recompute_up", "rows_bf16", "dA_entries_bf16",
-    "dB_entries_bf16", "num_threads",
+    "dB_entries_bf16", "num_threads", "gate_up_product", "gate_up_backward", "gated_fwd",
 ]
 
 SIGMA = {"identity": 0, "silu": 1, "gelu": 2}
@@ -65,6 +68,8 @@ def lib():
         l.oracle_dB_entries_bf16.argtypes = [_long, _long, _long, _int, _int, _U16, _long, _U16,
                                              _U16, _long, _long, _L, _L, _D]
         l.oracle_recompute_up.argtypes = [_long, _long, _long, _int, _D, _D, _D]
+        l.oracle_gate_up_product.argtypes = [_long, _D, _D, _D]
+        l.oracle_gate_up_backward.argtypes = [_long, _D, _D, _D, _D, _D]
         l.oracle_num_threads.restype = _int
         _lib = l
     return _lib
@@ -178,6 +183,36 @@ def recompute_up(Z, B, sigma_kind="silu"):
     Y, py = _out((n, d_out))
     lib().oracle_recompute_up(n, d_out, r, _sig(sigma_kind), pz, pb, py)
     return Y
+
+
+def gate_up_product(Yg, Yu):
+    """M = Y_gate * Y_up element-wise (the gated MLP's product, Fig. 4)."""
+    Yg, pg = _f64(Yg)
+    Yu, pu = _f64(Yu)
+    assert Yg.shape == Yu.shape
+    M, pm = _out(Yg.shape)
+    lib().oracle_gate_up_product(Yg.size, pg, pu, pm)
+    return M
+
+
+def gate_up_backward(dM, Yg, Yu):
+    """Gradients of the product: (dY_gate, dY_up) = (dM * Y_up, dM * Y_gate)."""
+    dM, pd = _f64(dM)
+    Yg, pg = _f64(Yg)
+    Yu, pu = _f64(Yu)
+    assert dM.shape == Yg.shape == Yu.shape
+    dYg, pdg = _out(dM.shape)
+    dYu, pdu = _out(dM.shape)
+    lib().oracle_gate_up_backward(dM.size, pd, pg, pu, pdg, pdu)
+    return dYg, dYu
+
+
+def gated_fwd(X, Ag, Bg, Au, Bu, sigma="silu", round_store=False):
+    """The gate and up layers on one X and their product.  Returns
+    (Z_gate, H_gate, Y_gate, Z_up, H_up, Y_up, M)."""
+    Zg, Hg, Yg = fwd(X, Ag, Bg, sigma, round_store)
+    Zu, Hu, Yu = fwd(X, Au, Bu, sigma, round_store)
+    return Zg, Hg, Yg, Zu, Hu, Yu, gate_up_product(Yg, Yu)
 
 
 def fwd_qkv(X, As, Bs, sigma="silu", round_store=False):

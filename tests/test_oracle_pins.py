@@ -345,3 +345,63 @@ def test_recompute_up_worked_example():
     s = 1.0 / (1.0 + math.exp(-1.0))
     Y = oracle.recompute_up(np.array([[0.0, 1.0]]), np.array([[1.0, 2.0], [-3.0, 0.5]]), "silu")
     np.testing.assert_allclose(Y, [[2.0 * s, 0.5 * s]], rtol=1e-15)
+
+
+# --- gated MLP: M = Y_gate * Y_up (Fig. 4, Sec. 3.2, App. E) ---
+
+def test_gate_up_closed_form_identity_sigma():
+    # sigma = identity and every row of B_up the same vector b: Y_up[t, o] =
+    # x_t . (A_up^T b) for every o, so M[t, o] = (X (B_g A_g)^T)[t, o] c_t with
+    # c = X A_up^T b -- computed here with the factors multiplied first
+    rng = np.random.default_rng(41)
+    n, d_in, d_ff, r = 7, 12, 10, 3
+    X = rng.standard_normal((n, d_in))
+    Ag = rng.standard_normal((r, d_in))
+    Bg = rng.standard_normal((d_ff, r))
+    Au = rng.standard_normal((r, d_in))
+    b = rng.standard_normal(r)
+    Bu = np.tile(b, (d_ff, 1))
+    *_, M = oracle.gated_fwd(X, Ag, Bg, Au, Bu, "identity")
+    c = X @ (Au.T @ b)
+    np.testing.assert_allclose(M, (X @ (Bg @ Ag).T) * c[:, None], rtol=1e-12, atol=1e-12)
+
+
+def test_gate_up_product_worked_example():
+    # two entries by hand: 2 x (-3) = -6 and 0.5 x 4 = 2; the backward swaps
+    # the factors: dY_gate = dM * Y_up, dY_up = dM * Y_gate
+    M = oracle.gate_up_product(np.array([[2.0, 0.5]]), np.array([[-3.0, 4.0]]))
+    np.testing.assert_array_equal(M, [[-6.0, 2.0]])
+    dYg, dYu = oracle.gate_up_backward(np.array([[1.0, -2.0]]), np.array([[2.0, 0.5]]), np.array([[-3.0, 4.0]]))
+    np.testing.assert_array_equal(dYg, [[-3.0, -8.0]])
+    np.testing.assert_array_equal(dYu, [[2.0, -1.0]])
+
+
+@pytest.mark.parametrize("kind", ["silu", "gelu"])
+def test_gated_mlp_central_differences(kind):
+    # the whole gated MLP of one block: M = gate(X) * up(X), out = down(M);
+    # L = sum(dOut * out).  Its gradients through the oracle's pieces (down
+    # backward -> dM -> product backward -> the two layers' backward, dX
+    # summed) against central differences of L w.r.t. X, A_gate, B_up, A_down
+    rng = np.random.default_rng(43)
+    n, d, d_ff, r = 4, 6, 8, 2
+    X = rng.standard_normal((n, d))
+    Ag, Au = (rng.standard_normal((r, d)) / math.sqrt(d) for _ in range(2))
+    Bg, Bu = (rng.standard_normal((d_ff, r)) / math.sqrt(r) for _ in range(2))
+    Ad = rng.standard_normal((r, d_ff)) / math.sqrt(d_ff)
+    Bd = rng.standard_normal((d, r)) / math.sqrt(r)
+    dOut = rng.standard_normal((n, d))
+
+    def loss():
+        *_, M = oracle.gated_fwd(X, Ag, Bg, Au, Bu, kind)
+        return float(np.sum(dOut * oracle.fwd(M, Ad, Bd, kind)[2]))
+
+    Zg, Hg, Yg, Zu, Hu, Yu, M = oracle.gated_fwd(X, Ag, Bg, Au, Bu, kind)
+    Zd, Hd, _ = oracle.fwd(M, Ad, Bd, kind)
+    dM, dAd, _, _ = oracle.bwd(M, Ad, Bd, dOut, Zd, Hd, kind, "cola")
+    dYg, dYu = oracle.gate_up_backward(dM, Yg, Yu)
+    dXg, dAg, _, _ = oracle.bwd(X, Ag, Bg, dYg, Zg, Hg, kind, "cola")
+    dXu, _, dBu, _ = oracle.bwd(X, Au, Bu, dYu, Zu, Hu, kind, "cola")
+    assert _rel(dXg + dXu, _fd_grad(loss, X)) < 1e-6
+    assert _rel(dAg, _fd_grad(loss, Ag)) < 1e-6
+    assert _rel(dBu, _fd_grad(loss, Bu)) < 1e-6
+    assert _rel(dAd, _fd_grad(loss, Ad)) < 1e-6
