@@ -57,7 +57,7 @@ def _peaks():
 class Block:
     """All tensors of one CoLA block workload, resident on the device."""
 
-    def __init__(self, wl, mode, device, seed=0, sigma="silu"):
+    def __init__(self, wl, mode, device, seed=0, sigma="silu", gated_unfused=False):
         import torch
 
         from paper_2502_10940_gb300 import cola
@@ -115,14 +115,46 @@ class Block:
                     g["dA"] = torch.empty((c * L.r, ldx), dtype=bf, device=device)[:, :L.d_in]
                 self.ws_bytes = max(self.ws_bytes, cola.cola_workspace_size(g["desc"], c))
                 self.groups.append(g)
+        # the gated MLP: the gate/up group's output GEMM forms M = Y_gate * Y_up
+        # straight into the down layer's input, and the down layer's backward
+        # forms dY_gate, dY_up straight into the gate/up upstream gradients
+        self.gated = bool(getattr(wl, "gated", False))
+        # gated_unfused (a comparison point, not the library's path): the same
+        # gated MLP with the product and its backward as torch element-wise
+        # ops between the library's calls (Y_gate, Y_up and dM stored)
+        self.gated_unfused = self.gated and gated_unfused
+        if self.gated:
+            gu = [g for g in self.groups if [m["L"].name for m in g["members"]] == ["gate", "up"]]
+            dn = [g for g in self.groups if [m["L"].name for m in g["members"]] == ["down"]]
+            if len(gu) != 1 or len(dn) != 1:
+                raise ValueError("a gated MLP needs one gate/up group and one down layer")
+            gu, dn = gu[0], dn[0]
+            gu["M_key"] = dn["members"][0]["L"].x
+            dn["gate_up"] = gu
+            if self.gated_unfused and self.train:
+                dn["dM"] = dn["dX"]
+            dn["dX"] = None
         self.ws = torch.empty(self.ws_bytes, dtype=torch.uint8, device=device)
         cola.cola_workspace_init(self.ws)
         self.launches_per_step = None
 
+    def _chained(self):
+        """Tensors a gated step forms itself: the down layer's input M and the
+        gate/up upstream gradients."""
+        if not self.gated:
+            return set()
+        dn = [g for g in self.groups if "gate_up" in g][0]
+        out = {id(self.X[dn["gate_up"]["M_key"]])}
+        if self.train:
+            out |= {id(m["dY"]) for m in dn["gate_up"]["members"]}
+        return out
+
     # inputs a step consumes from outside (activations, and upstream gradients
     # when training)
     def step_inputs(self):
-        return list(self.X.values()) + ([s["dY"] for s in self.layers] if self.train else [])
+        ins = list(self.X.values()) + ([s["dY"] for s in self.layers] if self.train else [])
+        chained = self._chained()
+        return [t for t in ins if id(t) not in chained]
 
     def add_input_set(self):
         """A second set of the step's input buffers (same shapes and pitches),
@@ -154,11 +186,15 @@ class Block:
     def step_results(self):
         if not self.train:
             return [s["Y"] for s in self.layers]
-        return [g["dA"] for g in self.groups] + [s["dB"] for s in self.layers] + [g["dX"] for g in self.groups]
+        return ([g["dA"] for g in self.groups] + [s["dB"] for s in self.layers] +
+                [g["dX"] for g in self.groups if g["dX"] is not None])
 
     def results_words(self):
         if not self.train:
             return "Y of every layer"
+        if self.gated:
+            return ("dA and dB of every layer and dX of the attention and gate/up input groups; Y, Z and H stay "
+                    "on the device (they feed the block's attention / MLP ops and the backward)")
         return ("dA and dB of every layer and dX of every input group; Y, Z and H stay on the device "
                 "(they feed the block's attention / MLP ops and the backward)")
 
@@ -166,7 +202,15 @@ class Block:
         c = self.cola
         for g in self.groups:
             m = g["members"]
-            if len(m) == 1:
+            if "M_key" in g and self.gated_unfused:
+                c.cola_fwd_shared_x(g["desc"], g["X"], g["A"], [s["B"] for s in m], [s["Y"] for s in m], g["Z"],
+                                    g["H"], self.ws)
+                self.torch.mul(m[0]["Y"], m[1]["Y"], out=self.X[g["M_key"]])
+            elif "M_key" in g:
+                Yg, Yu = (m[0]["Y"], m[1]["Y"]) if self.train else (None, None)
+                c.cola_fwd_gate_up(g["desc"], g["X"], g["A"], m[0]["B"], m[1]["B"], self.X[g["M_key"]], Yg, Yu,
+                                   g["Z"], g["H"], self.ws)
+            elif len(m) == 1:
                 s = m[0]
                 c.cola_fwd(g["desc"], g["X"], g["A"], s["B"], s["Y"], g["Z"], g["H"], self.ws)
             else:
@@ -177,7 +221,17 @@ class Block:
         c = self.cola
         for g in reversed(self.groups):
             m = g["members"]
-            if len(m) == 1:
+            if "gate_up" in g and self.gated_unfused:
+                s, gm = m[0], g["gate_up"]["members"]
+                c.cola_bwd(g["desc"], g["X"], g["A"], s["B"], s["dY"], g["Z"], g["H"], g["dM"], g["dA"], s["dB"],
+                           self.ws)
+                self.torch.mul(g["dM"], gm[1]["Y"], out=gm[0]["dY"])
+                self.torch.mul(g["dM"], gm[0]["Y"], out=gm[1]["dY"])
+            elif "gate_up" in g:
+                s, gm = m[0], g["gate_up"]["members"]
+                c.cola_bwd_down_gated(g["desc"], g["X"], g["A"], s["B"], s["dY"], g["Z"], g["H"], gm[0]["Y"],
+                                      gm[1]["Y"], gm[0]["dY"], gm[1]["dY"], g["dA"], s["dB"], self.ws)
+            elif len(m) == 1:
                 s = m[0]
                 c.cola_bwd(g["desc"], g["X"], g["A"], s["B"], s["dY"], g["Z"], g["H"], g["dX"], g["dA"], s["dB"],
                            self.ws)
@@ -229,7 +283,10 @@ def launch_cost(kind, shapes, splits, flags):
         elif kind == "wgrad":
             b = e * (k * m + k * n + m * n)
         elif kind == "bwd_dx":
-            b = e * (m * k + n * k + m * n)
+            # flag 32: the gated epilogue read Y_gate, Y_up and wrote dY_gate, dY_up
+            b = e * (m * k + n * k + m * n * (4 if flags & 32 else 1))
+        elif kind == "fwd_glu":
+            b = e * (m * k + n * k + m * n * (3 if flags & 1 else 1))   # M (+ Y_gate, Y_up)
         elif kind == "reduce":
             b = e * m * n * (2 if flags & 1 else 1)   # flag: the Z/H reduce writes Z and H
         elif kind == "sigma":
@@ -607,7 +664,7 @@ def full_rank_baseline(wl, device, steps, warmup, seed=0, flush=None):
             "impl": "torch.matmul (cuBLAS) bf16"}
 
 
-def timed_block(wl, mode, args, device, stream, dist=None, seed=0):
+def timed_block(wl, mode, args, device, stream, dist=None, seed=0, **block_kw):
     """Build the block, count its launches with the library trace, warm it
     up, capture its step as a CUDA graph (unless --graph off) and time K
     steps (clocks sampled meanwhile).  Returns a dict of what it built and
@@ -616,7 +673,7 @@ def timed_block(wl, mode, args, device, stream, dist=None, seed=0):
 
     from paper_2502_10940_gb300 import cola
 
-    blk = Block(wl, mode, device, seed=seed)
+    blk = Block(wl, mode, device, seed=seed, **block_kw)
     # launches per step, counted by the library's trace
     with cola.Trace(512) as tr:
         blk.step()
@@ -701,7 +758,8 @@ def run_cola(args, wl):
     if (mode == "infer") != (wl.phase == "infer"):
         raise SystemExit(f"mode {mode} does not fit the {wl.phase} workload {wl.name}")
     stream = torch.cuda.current_stream()
-    tb = timed_block(wl, mode, args, device, stream, dist, seed=args.seed + rank)
+    tb = timed_block(wl, mode, args, device, stream, dist, seed=args.seed + rank,
+                     **({"gated_unfused": True} if args.gated_unfused else {}))
     blk, graph, use_graph, ms, clocks, flush = (tb[k] for k in ("blk", "graph", "use_graph", "ms", "clocks",
                                                                   "flush"))
 
@@ -847,6 +905,22 @@ def run_cola(args, wl):
                                        "modes": modes_ratio(w1, w1.modes[0], t1["blk"], args, device, stream,
                                                             seed=args.seed)}}
                 del t1
+                # the same 7B block with the gated MLP chained through the library
+                torch.cuda.synchronize()
+                torch.cuda.empty_cache()
+                wg = WORKLOADS["7b-gated"]
+                tg = timed_block(wg, mode, args, device, stream, None, seed=args.seed)
+                vg = whole_job_tflops(wg.flops, 1, tg["ms"])
+                del tg["blk"], tg["graph"]
+                tu = timed_block(wg, mode, args, device, stream, None, seed=args.seed, gated_unfused=True)
+                line["also"]["7b_gated"] = {"workload": wg.desc, "mode": mode, "value": round(vg, 2),
+                                            "unit": "TFLOP/s", "ms_per_step": round(tg["ms"], 4),
+                                            "pct_dense_bf16_peak": round(100.0 * vg / peaks["bf16_tflops"], 2),
+                                            "cuda_graph": tg["use_graph"], "clocks": tg["clocks"],
+                                            "unfused_ms_per_step": round(tu["ms"], 4),
+                                            "unfused_how": "the library's GEMMs with the product and its "
+                                                           "backward as torch element-wise ops between them"}
+                del tg, tu
             line["cpu_baseline"] = cpu_baseline(wl)
     if rank == 0:
         print(json.dumps(line), flush=True)
@@ -869,6 +943,8 @@ def main(argv=None):
                     help="replay each step as one CUDA graph (off: launch every kernel from the host)")
     ap.add_argument("--seed", type=int, default=0)
     ap.add_argument("--no-extras", action="store_true", help="skip e2e, full-rank and CPU baselines")
+    ap.add_argument("--gated-unfused", action="store_true",
+                    help="gated workloads: the product and its backward as torch element-wise ops (comparison)")
     args = ap.parse_args(argv)
     args.warmup = max(3, args.warmup)   # at least 3 untimed warm-up steps, always
     args.steps = max(1, args.steps)

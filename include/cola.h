@@ -180,6 +180,45 @@ cola_status_t cola_bwd_qkv_fused(const cola_desc_t* desc, const void* X, const v
                                  const void* dY_v, const void* Z_qkv, const void* H_qkv, void* dX, void* dA_qkv,
                                  void* dB_q, void* dB_k, void* dB_v, void* ws, size_t ws_bytes, void* stream);
 
+/* ---- the gated MLP (Fig. 4; Sec. 3.2; App. E) ----
+ * LLaMA's MLP multiplies its gate and up projections element-wise and feeds
+ * the product to the down projection.  CoLA turns gate, up and down into
+ * auto-encoder layers and keeps the element-wise product (Sec. 3.2), with no
+ * full-rank activation on the gate branch (App. E, "Low-Rank sigma Only"):
+ *     M = Y_gate (.) Y_up,   Y_gate = B_gate sigma(A_gate x),  Y_up = B_up sigma(A_up x).
+ *
+ * Forward of gate and up and their product.  desc describes ONE of the two
+ * projections (d_in = model width, d_out = d_ff, r); both read X.
+ *   A_cat [2r x d_in] (ld_a) = [A_gate; A_up] stacked by rows: one GEMM with
+ *     N = 2r reads X once and writes Z_cat [n x 2r] = [Z_gate Z_up] and, under
+ *     COLA, H_cat [n x 2r], exactly as cola_fwd_shared_x with count 2.
+ *   B_gate, B_up [d_out x r]: one GEMM over both, each output tile's gate and
+ *     up halves in two accumulators of one CTA (CTA pair), whose epilogue
+ *     stores M [n x d_out] (ld_y) = bf16(Y_gate * Y_up), the product of the
+ *     bf16-rounded outputs (exact in fp32, rounded once), and, in the
+ *     training modes, Y_gate and Y_up [n x d_out] (ld_y) = bf16 outputs for
+ *     the backward.  Under COLA_MODE_INFER Y_gate, Y_up, Z_cat and H_cat must
+ *     be NULL (M alone is stored); otherwise Y_gate and Y_up are required.
+ * ws: cola_workspace_size(desc, 2).  The gate/up backward is
+ * cola_bwd_shared_x (count 2) with dY = {dY_gate, dY_up} from
+ * cola_bwd_down_gated. */
+cola_status_t cola_fwd_gate_up(const cola_desc_t* desc, const void* X, const void* A_cat, const void* B_gate,
+                               const void* B_up, void* M, void* Y_gate, void* Y_up, void* Z_cat, void* H_cat,
+                               void* ws, size_t ws_bytes, void* stream);
+
+/* Backward of the down projection whose input is M = Y_gate (.) Y_up: as
+ * cola_bwd with X = M (desc: the down layer, d_in = d_ff, ld_x = the pitch of
+ * M, Y_gate, Y_up, dY_gate, dY_up), except that its input gradient
+ * dM = dZ A is not stored: the epilogue of that GEMM reads Y_gate and Y_up
+ * and stores the gradients at the product's factors,
+ *     dY_gate = bf16(bf16(dM) * Y_up),   dY_up = bf16(bf16(dM) * Y_gate),
+ * which the gate/up backward (cola_bwd_shared_x, count 2) takes as its dY.
+ * dA, dB as in cola_bwd; H_save NULL under COLA_M; ws: cola_workspace_size(desc, 1). */
+cola_status_t cola_bwd_down_gated(const cola_desc_t* desc, const void* M, const void* A, const void* B,
+                                  const void* dY, const void* Z_save, const void* H_save, const void* Y_gate,
+                                  const void* Y_up, void* dY_gate, void* dY_up, void* dA, void* dB, void* ws,
+                                  size_t ws_bytes, void* stream);
+
 /* Block-level CoLA-M recompute of the up-projections (Sec. 4.2, App. C:
  * in the backward, CoLA-M recomputes B sigma(.) from the saved low-rank
  * activation instead of keeping the layer output):
@@ -296,7 +335,8 @@ typedef enum {
     COLA_KERNEL_WGRAD = 3,       /* dB = dY^T H and dA = dZ^T X, token split (M=d_out | r, N=r | d_in, K=n) */
     COLA_KERNEL_REDUCE = 4,      /* fixed-order sum of the partials       (M, N of the gradient, K=splits) */
     COLA_KERNEL_BWD_DX = 5,      /* dX = dZ A                             (M=n, N=d_in, K=r or 3r) */
-    COLA_KERNEL_SIGMA = 6        /* H = sigma(Z), elementwise             (M=n, N=count r, K=0) */
+    COLA_KERNEL_SIGMA = 6,       /* H = sigma(Z), elementwise             (M=n, N=count r, K=0) */
+    COLA_KERNEL_FWD_GLU = 7      /* M = (H_gate B_gate^T) * (H_up B_up^T) (M=n, N=d_ff, K=2r) */
 } cola_kernel_t;
 
 typedef struct {
@@ -311,7 +351,11 @@ typedef struct {
                                   launch after it applies the epilogue);
                            bit 2: the GEMM ran on CTA pairs (clusters of two CTAs, tcgen05
                                   cta_group::2, 256-row tiles);
-                           bit 3: one CTA ran two 128-row sub-tiles sharing each B tile */
+                           bit 3: one CTA ran two 128-row sub-tiles sharing each B tile;
+                           bit 4: weight gradients with a split tail (splits = pieces per
+                                  tail tile; a reduce launch follows when they are > 1);
+                           bit 5: the dX epilogue stored the gated-MLP gradients dY_gate,
+                                  dY_up instead of dX (cola_bwd_down_gated) */
 } cola_trace_slot_t;
 
 cola_status_t cola_trace_attach(cola_trace_slot_t* slots, int32_t capacity, int32_t* count);

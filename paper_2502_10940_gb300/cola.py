@@ -23,11 +23,11 @@ STATUS = {0: "COLA_OK", 1: "COLA_ERR_INVALID", 2: "COLA_ERR_ALIGN", 3: "COLA_ERR
 
 # the entry points include/cola.h declares
 SYMBOLS = ("cola_workspace_size", "cola_workspace_init", "cola_fwd", "cola_bwd", "cola_fwd_shared_x",
-           "cola_bwd_shared_x", "cola_recompute_up", "cola_fwd_qkv_fused", "cola_bwd_qkv_fused", "cola_check_status",
+           "cola_bwd_shared_x", "cola_fwd_gate_up", "cola_bwd_down_gated", "cola_recompute_up", "cola_fwd_qkv_fused", "cola_bwd_qkv_fused", "cola_check_status",
            "cola_wgrad_static_scratch", "cola_selftest_wait_timeout", "cola_selftest_wait_timeout_pair",
            "cola_trace_attach", "cola_trace_detach", "cola_status_string")
 STATIC_SCRATCH_BYTES = 64 * 1024 * 1024
-KERNELS = {0: "fwd_zh", 1: "fwd_y", 2: "bwd_dz", 3: "wgrad", 4: "reduce", 5: "bwd_dx", 6: "sigma"}
+KERNELS = {0: "fwd_zh", 1: "fwd_y", 2: "bwd_dz", 3: "wgrad", 4: "reduce", 5: "bwd_dx", 6: "sigma", 7: "fwd_glu"}
 
 
 class ColaError(RuntimeError):
@@ -76,6 +76,10 @@ def lib():
         l.cola_bwd_shared_x.argtypes = [D, ctypes.c_int32, _vp, _vp, PP, PP, _vp, _vp, _vp, _vp, PP, _vp,
                                         ctypes.c_size_t, _vp]
         l.cola_bwd_shared_x.restype = st
+        l.cola_fwd_gate_up.argtypes = [D] + [_vp] * 10 + [ctypes.c_size_t, _vp]
+        l.cola_fwd_gate_up.restype = st
+        l.cola_bwd_down_gated.argtypes = [D] + [_vp] * 13 + [ctypes.c_size_t, _vp]
+        l.cola_bwd_down_gated.restype = st
         l.cola_recompute_up.argtypes = [D, ctypes.c_int32, _vp, PP, PP, _vp, ctypes.c_size_t, _vp]
         l.cola_recompute_up.restype = st
         l.cola_fwd_qkv_fused.argtypes = [D] + [_vp] * 11 + [ctypes.c_size_t, _vp]
@@ -184,6 +188,18 @@ def cola_bwd_shared_x(d, X, A_cat, Bs, dYs, Z_cat, H_cat, dX, dA_cat, dBs, ws, s
     _check(lib().cola_bwd_shared_x(ctypes.byref(d), len(Bs), _ptr(X), _ptr(A_cat), _ptr_array(Bs), _ptr_array(dYs),
                                    _ptr(Z_cat), _ptr(H_cat), _ptr(dX), _ptr(dA_cat), _ptr_array(dBs), _ptr(ws),
                                    _nbytes(ws), _stream(stream)), "cola_bwd_shared_x")
+
+
+def cola_fwd_gate_up(d, X, A_cat, B_gate, B_up, M, Y_gate, Y_up, Z_cat, H_cat, ws, stream=None):
+    _check(lib().cola_fwd_gate_up(ctypes.byref(d), _ptr(X), _ptr(A_cat), _ptr(B_gate), _ptr(B_up), _ptr(M),
+                                  _ptr(Y_gate), _ptr(Y_up), _ptr(Z_cat), _ptr(H_cat), _ptr(ws), _nbytes(ws),
+                                  _stream(stream)), "cola_fwd_gate_up")
+
+
+def cola_bwd_down_gated(d, M, A, B, dY, Z_save, H_save, Y_gate, Y_up, dY_gate, dY_up, dA, dB, ws, stream=None):
+    _check(lib().cola_bwd_down_gated(ctypes.byref(d), _ptr(M), _ptr(A), _ptr(B), _ptr(dY), _ptr(Z_save),
+                                     _ptr(H_save), _ptr(Y_gate), _ptr(Y_up), _ptr(dY_gate), _ptr(dY_up), _ptr(dA),
+                                     _ptr(dB), _ptr(ws), _nbytes(ws), _stream(stream)), "cola_bwd_down_gated")
 
 
 def cola_recompute_up(d, Z_cat, Bs, Ys, ws, stream=None):

@@ -562,6 +562,69 @@ cola_status_t run_wgrad_tail(const WgradPlan& w, int64_t ntok, const WgradJob* j
                            [&] { return launch_tail_reduce(rd, sms, st); }));
 }
 
+// Gated MLP forward GEMM: per 128-column tile of M = Y_gate * Y_up (pitch
+// ld_y), one K walk over [H_gate H_up] (H_cat, pitch ldh) whose gate half
+// accumulates H_gate B_gate^T and whose up half H_up B_up^T, in two
+// accumulators; Y_gate, Y_up are stored too when not null (training).
+// Compute-heavy launches with r >= 512 run on CTA pairs.
+cola_status_t run_glu(const Shape& s, const void* H_cat, int64_t ldh, const void* Bg, const void* Bu, void* M,
+                      void* Yg, void* Yu, unsigned int* status, int sms, cudaStream_t st)
+{
+    const int64_t K2 = 2 * s.r;
+    const bool pair = heavy_gemm(s.n, s.d_out, K2) && s.r >= 512;
+    const int msub = pair ? TILE_PAIR : 1;
+    GemmBatch b;
+    std::memset(&b, 0, sizeof b);
+    b.count = 1;
+    GemmProblem& pr = b.prob[0];
+    pr.p = base_params(s.n, s.d_out, K2, 128, msub);
+    pr.p.glu_half = static_cast<int>(s.r / BK);
+    COLA_MAP(map_kmajor(&pr.map_a, H_cat, K2, s.n, ldh, a_box_rows(msub)));
+    COLA_MAP(map_kmajor(&pr.map_b, Bg, s.r, s.d_out, s.r, b_box_rows(128, msub)));
+    COLA_MAP(map_kmajor(&pr.map_b2, Bu, s.r, s.d_out, s.r, b_box_rows(128, msub)));
+    COLA_MAP(map_box32(&pr.map_d, M, s.d_out, s.n, s.ld_y));
+    pr.map_d2 = pr.map_d3 = pr.map_z = pr.map_d;
+    if (Yg) {
+        COLA_MAP(map_box32(&pr.map_d2, Yg, s.d_out, s.n, s.ld_y));
+        COLA_MAP(map_box32(&pr.map_d3, Yu, s.d_out, s.n, s.ld_y));
+    }
+    pr.p.has_d2 = Yg != nullptr;
+    pr.p.d_ptr = static_cast<__nv_bfloat16*>(M);
+    pr.p.d2_ptr = static_cast<__nv_bfloat16*>(Yg);
+    pr.p.d3_ptr = static_cast<__nv_bfloat16*>(Yu);
+    pr.p.d_ld = s.ld_y;
+    pr.p.status = status;
+    const int64_t mnk[1][3] = {{s.n, s.d_out, K2}};
+    const int flags = (Yg ? 1 : 0) | (pair ? TRACE_PAIR : 0);
+    return launched(traced(COLA_KERNEL_FWD_GLU, 1, mnk, 1, flags, st, [&] { return dispatch_glu(pair, b, sms, st); }));
+}
+
+// The down layer's input gradient when its input is M = Y_gate * Y_up: the
+// dX GEMM dM = dZ A (dZ [n x K] pitch ldz) whose epilogue stores
+// dY_gate = bf16(dM) * Y_up and dY_up = bf16(dM) * Y_gate (all pitch ld_x).
+cola_status_t run_b4_glu(const Shape& s, int64_t K, const void* dZ, int64_t ldz, const void* A, const void* Yg,
+                         const void* Yu, void* dYg, void* dYu, unsigned int* status, int sms, cudaStream_t st)
+{
+    const int bn = choose_bn_for(s.n, s.d_in, K);
+    const int ms = choose_msub(s.n, s.d_in, K, bn);
+    GemmProblem pr;
+    std::memset(&pr, 0, sizeof pr);
+    pr.p = base_params(s.n, s.d_in, K, bn, ms);
+    COLA_MAP(map_kmajor(&pr.map_a, dZ, K, s.n, ldz, a_box_rows(ms)));
+    COLA_MAP(map_mnmajor(&pr.map_b, A, s.d_in, K, s.ld_a));
+    COLA_MAP(map_box32(&pr.map_d, dYg, s.d_in, s.n, s.ld_x));
+    COLA_MAP(map_box32(&pr.map_d2, dYu, s.d_in, s.n, s.ld_x));
+    pr.map_z = pr.map_d3 = pr.map_b2 = pr.map_d;
+    pr.p.d_ptr = static_cast<__nv_bfloat16*>(dYg);
+    pr.p.d2_ptr = static_cast<__nv_bfloat16*>(dYu);
+    pr.p.d_ld = s.ld_x;
+    pr.p.yg_ptr = static_cast<const __nv_bfloat16*>(Yg);
+    pr.p.yu_ptr = static_cast<const __nv_bfloat16*>(Yu);
+    pr.p.status = status;
+    const int64_t mnk[1][3] = {{s.n, s.d_in, K}};
+    return run_batch<false, true, EPI_GLU_BWD>(COLA_KERNEL_BWD_DX, bn, ms, &pr, mnk, 1, TRACE_GLU, sms, st);
+}
+
 // B4: dX = dZ A  (dZ [n x K] pitch ldz, A [K x d_in] pitch ld_a; K = r or 3r)
 cola_status_t run_b4(const Shape& s, int64_t K, const void* dZ, int64_t ldz, const void* A, void* dX,
                      unsigned int* status, int sms, cudaStream_t st)
@@ -630,14 +693,31 @@ cola_status_t cola_fwd(const cola_desc_t* desc, const void* X, const void* A, co
     return run_f2(s, 1, Hs, s.r, Bs, Ys, part, part_bytes, status, sms, st);
 }
 
-cola_status_t cola_bwd(const cola_desc_t* desc, const void* X, const void* A, const void* B, const void* dY,
-                       const void* Z_save, const void* H_save, void* dX, void* dA, void* dB, void* ws,
-                       size_t ws_bytes, void* stream)
+}  // extern "C"
+
+namespace cola {
+namespace {
+
+// The gated-MLP ends of the down layer's backward (cola_bwd_down_gated).
+struct GluBwd {
+    const void* Yg;
+    const void* Yu;
+    void* dYg;
+    void* dYu;
+};
+
+cola_status_t bwd_single(const cola_desc_t* desc, const void* X, const void* A, const void* B, const void* dY,
+                         const void* Z_save, const void* H_save, void* dX, void* dA, void* dB, void* ws,
+                         size_t ws_bytes, void* stream, const GluBwd* glu)
 {
     Shape s;
     COLA_TRY(check_desc(desc, &s));
     if (desc->mode == COLA_MODE_INFER) return COLA_ERR_INVALID;
-    COLA_TRY(check_ptrs({X, A, B, dY, Z_save, dX, dA, dB}));
+    COLA_TRY(check_ptrs({X, A, B, dY, Z_save, dA, dB}));
+    if (glu)
+        COLA_TRY(check_ptrs({glu->Yg, glu->Yu, glu->dYg, glu->dYu}));
+    else
+        COLA_TRY(check_ptrs({dX}));
     const bool cola_m = desc->mode == COLA_MODE_COLA_M;
     if (cola_m ? H_save != nullptr : H_save == nullptr) return COLA_ERR_INVALID;
     if (H_save && !aligned16(H_save)) return COLA_ERR_ALIGN;
@@ -662,7 +742,54 @@ cola_status_t cola_bwd(const cola_desc_t* desc, const void* X, const void* A, co
     const WgradPlan w = wgrad_plan(*desc, 1, sms);
     const WgradJob jobs[2] = {{dY, s.ld_y, Hsrc, s.r, dB, s.r}, {dZ, s.r, X, s.ld_x, dA, s.ld_a}};
     COLA_TRY(run_wgrad(w, s.n, jobs, desc->wgrad_fp32, part, part_bytes, status, sms, st));
+    if (glu) return run_b4_glu(s, s.r, dZ, s.r, A, glu->Yg, glu->Yu, glu->dYg, glu->dYu, status, sms, st);
     return run_b4(s, s.r, dZ, s.r, A, dX, status, sms, st);
+}
+
+}  // namespace
+}  // namespace cola
+
+extern "C" {
+
+cola_status_t cola_bwd(const cola_desc_t* desc, const void* X, const void* A, const void* B, const void* dY,
+                       const void* Z_save, const void* H_save, void* dX, void* dA, void* dB, void* ws,
+                       size_t ws_bytes, void* stream)
+{
+    return bwd_single(desc, X, A, B, dY, Z_save, H_save, dX, dA, dB, ws, ws_bytes, stream, nullptr);
+}
+
+cola_status_t cola_bwd_down_gated(const cola_desc_t* desc, const void* M, const void* A, const void* B,
+                                  const void* dY, const void* Z_save, const void* H_save, const void* Y_gate,
+                                  const void* Y_up, void* dY_gate, void* dY_up, void* dA, void* dB, void* ws,
+                                  size_t ws_bytes, void* stream)
+{
+    const GluBwd glu{Y_gate, Y_up, dY_gate, dY_up};
+    return bwd_single(desc, M, A, B, dY, Z_save, H_save, nullptr, dA, dB, ws, ws_bytes, stream, &glu);
+}
+
+cola_status_t cola_fwd_gate_up(const cola_desc_t* desc, const void* X, const void* A_cat, const void* B_gate,
+                               const void* B_up, void* M, void* Y_gate, void* Y_up, void* Z_cat, void* H_cat,
+                               void* ws, size_t ws_bytes, void* stream)
+{
+    Shape s;
+    COLA_TRY(check_desc(desc, &s));
+    COLA_TRY(check_ptrs({X, A_cat, B_gate, B_up, M}));
+    COLA_TRY(check_saved(desc->mode, Z_cat, H_cat));
+    const bool train = desc->mode != COLA_MODE_INFER;
+    if ((Y_gate != nullptr) != train || (Y_up != nullptr) != train) return COLA_ERR_INVALID;
+    if ((Y_gate && !aligned16(Y_gate)) || (Y_up && !aligned16(Y_up))) return COLA_ERR_ALIGN;
+    int sms = 0;
+    COLA_TRY(device_info(&sms));
+    WsLayout L;
+    COLA_TRY(check_ws(*desc, 2, sms, ws, ws_bytes, &L));
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    unsigned int* status = ws_status(ws);
+    const int64_t R = 2 * s.r;
+    uint8_t* H = desc->mode != COLA_MODE_COLA ? wsb(ws) + L.h_off : static_cast<uint8_t*>(H_cat);
+    float* part = reinterpret_cast<float*>(wsb(ws) + L.part_off);
+    const size_t part_bytes = L.total - L.part_off;
+    COLA_TRY(run_f1(s, desc->sigma, R, X, A_cat, Z_cat, H, R, part, part_bytes, status, sms, st));
+    return run_glu(s, H, R, B_gate, B_up, M, Y_gate, Y_up, status, sms, st);
 }
 
 cola_status_t cola_fwd_shared_x(const cola_desc_t* desc, int32_t count, const void* X, const void* A_cat,

@@ -39,6 +39,14 @@
 //   EPI_F32     fp32 split-K partial slab, reduced (in a fixed order) by the
 //               reduce kernel: fp32-accumulated weight gradients, and the
 //               forward GEMMs of small launches
+//   EPI_GLU     gated MLP forward (Fig. 4): the K walk covers [H_gate H_up]
+//               (2r columns of H_cat); the gate half accumulates H_gate B_gate^T
+//               and the up half H_up B_up^T into a second accumulator of the
+//               same tile, and the epilogue stores M = bf16(Y_gate * Y_up) of
+//               the bf16-rounded outputs (and Y_gate, Y_up when training)
+//   EPI_GLU_BWD dX GEMM of the down layer whose input is that M: with
+//               dM = bf16(acc) it stores dY_gate = bf16(dM * Y_up) and
+//               dY_up = bf16(dM * Y_gate), reading Y_gate, Y_up per chunk
 //   EPI_TAIL      weight gradients (bf16 D) with a split tail: the tiles of
 //               the full waves run whole and store D = bf16(acc) as
 //               EPI_STORE; the tiles of the last, partial wave are split
@@ -84,7 +92,7 @@ enum : unsigned int {
     ST_TIMEOUT_DRAIN = 1u << 3,
 };
 
-enum Epi : int { EPI_STORE = 0, EPI_ZH = 1, EPI_DSIGMA = 2, EPI_F32 = 3, EPI_TAIL = 4 };
+enum Epi : int { EPI_STORE = 0, EPI_ZH = 1, EPI_DSIGMA = 2, EPI_F32 = 3, EPI_TAIL = 4, EPI_GLU = 5, EPI_GLU_BWD = 6 };
 enum Sigma : int { SIG_IDENTITY = 0, SIG_SILU = 1, SIG_GELU = 2 };
 
 struct GemmParams {
@@ -106,6 +114,14 @@ struct GemmParams {
     long long d_ld;
     int sigma;
     unsigned int* status;
+    // gated MLP (EPI_GLU, EPI_GLU_BWD): the outputs behind map_d2 and map_d3,
+    // for the masked stores of a ragged right edge (pitch d_ld), and the
+    // Y_gate, Y_up that the EPI_GLU_BWD epilogue reads (pitch d_ld)
+    int glu_half;                 // EPI_GLU: k-blocks of the gate half; the up half reads map_b2
+    __nv_bfloat16* d2_ptr;
+    __nv_bfloat16* d3_ptr;
+    const __nv_bfloat16* yg_ptr;
+    const __nv_bfloat16* yu_ptr;
     // problem 0 only, for the failure-detection self-tests: 1 = the producers
     // issue nothing, so the MMA's first wait runs out; 2 = the odd CTA of a
     // pair issues its first k-block only, so the MMA's second wait runs out
@@ -114,8 +130,8 @@ struct GemmParams {
 };
 
 // Epilogue staging: per epilogue warp two 2 KB boxes of 32 rows x 32 bf16
-// columns (64-byte rows, 64-byte TMA swizzle).  EPI_STORE / EPI_ZH use them as
-// a ring of output boxes.  EPI_DSIGMA uses them as a double buffer for the
+// columns (64-byte rows, 64-byte TMA swizzle).  EPI_STORE / EPI_ZH / EPI_GLU /
+// EPI_GLU_BWD use them as a ring of output boxes.  EPI_DSIGMA uses them as a double buffer for the
 // saved Z: the box of the warp's next chunk is TMA-loaded while the current
 // one is processed, and dZ is computed in place and TMA-stored from the box.
 constexpr int EPI_BOX_BYTES = 32 * 32 * 2;
@@ -125,8 +141,9 @@ constexpr int EPI_SMEM_BYTES = NUM_EPI_WARPS * EPI_WARP_BYTES;
 
 // A CTA tile is MSUB x 128 rows by BN columns: MSUB = 2 runs two M = 128
 // MMAs per k-step that share one B tile (halving the B-operand traffic per
-// output row), into two TMEM accumulators of BN columns each.
-template <int BN, int MSUB, bool PAIR = false>
+// output row), into two TMEM accumulators of BN columns each.  ACCS = 2: one
+// 128-row tile with two accumulators (the gate and up halves of EPI_GLU).
+template <int BN, int MSUB, bool PAIR = false, int ACCS = 1>
 struct GemmCfg {
     static_assert(BN % 64 == 0 && BN >= 64 && BN <= 256, "BN must be 64..256 in steps of 64");
     static_assert(MSUB == 1 || MSUB == 2, "one or two 128-row sub-tiles");
@@ -134,7 +151,7 @@ struct GemmCfg {
     static constexpr int TILE_M = PAIR ? 2 * BM : BM * MSUB;   // rows of one unit
     static constexpr int CTA_ROWS = PAIR ? BM : TILE_M;          // rows of A this CTA loads
     static constexpr int B_ROWS = PAIR ? BN / 2 : BN;           // columns of B this CTA loads
-    static constexpr int ACC_COLS = MSUB * BN;   // TMEM columns of one tile's accumulator
+    static constexpr int ACC_COLS = (MSUB > ACCS ? MSUB : ACCS) * BN;   // TMEM columns of one tile's accumulators
     static_assert(2 * ACC_COLS <= 512, "double-buffered accumulator must fit TMEM");
     static constexpr int A_BYTES = CTA_ROWS * BK * 2;
     static constexpr int B_BYTES = B_ROWS * BK * 2;
@@ -245,6 +262,7 @@ constexpr int MAX_GROUP = 4;
 // One GEMM of a batch: its operand / output tensor maps and parameters.
 struct GemmProblem {
     CUtensorMap map_a, map_b, map_d, map_d2, map_z;
+    CUtensorMap map_b2, map_d3;   // EPI_GLU: B_up, and the Y_up output
     GemmParams p;
     int unit_begin;   // first batch-wide unit index of this problem
 };
@@ -378,7 +396,7 @@ template <int BN, int MSUB, bool A_MN, bool B_MN, int EPI, bool PAIR = false>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
     gemm_kernel(const __grid_constant__ GemmBatch batch)
 {
-    using C = GemmCfg<BN, MSUB, PAIR>;
+    using C = GemmCfg<BN, MSUB, PAIR, EPI == EPI_GLU ? 2 : 1>;
     constexpr int STAGES = C::STAGES;
     constexpr int TILE_M = C::TILE_M;
     extern __shared__ uint8_t smem_raw[];
@@ -430,6 +448,11 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             tma_prefetch_desc(&batch.prob[g].map_b);
             if (EPI != EPI_F32) tma_prefetch_desc(&batch.prob[g].map_d);
             if (EPI == EPI_DSIGMA) tma_prefetch_desc(&batch.prob[g].map_z);
+            if (EPI == EPI_GLU) {
+                tma_prefetch_desc(&batch.prob[g].map_b2);
+                tma_prefetch_desc(&batch.prob[g].map_d2);
+                tma_prefetch_desc(&batch.prob[g].map_d3);
+            }
         }
     }
     if (warp == 1) {
@@ -485,6 +508,13 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                     uint8_t* sa = smem_a + stage * C::A_BYTES;
                     uint8_t* sb = smem_b + stage * C::B_BYTES;
                     const int k0 = kb * BK;
+                    // EPI_GLU: the up half of the walk reads B_up from its own k = 0
+                    int kB = k0;
+                    const CUtensorMap* mb = map_b;
+                    if (EPI == EPI_GLU && kb >= batch.prob[x.g].p.glu_half) {
+                        kB = k0 - batch.prob[x.g].p.glu_half * BK;
+                        mb = &batch.prob[x.g].map_b2;
+                    }
                     if (PAIR) {
                         // both CTAs' boxes count on the even CTA's stage barrier
                         const uint32_t fb = mapa_shared(smem_u32(&full_bar[stage]), 0);
@@ -499,9 +529,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                         if (B_MN) {
 #pragma unroll
                             for (int j = 0; j < C::B_ROWS / 64; ++j)
-                                tma_load_2d_pair(map_b, fb, sb + j * 64 * BK * 2, n0 + 64 * j, k0);
+                                tma_load_2d_pair(mb, fb, sb + j * 64 * BK * 2, n0 + 64 * j, kB);
                         } else {
-                            tma_load_2d_pair(map_b, fb, sb, k0, n0);
+                            tma_load_2d_pair(mb, fb, sb, kB, n0);
                         }
                     } else {
                         mbar_arrive_expect_tx(&full_bar[stage], C::STAGE_BYTES);
@@ -515,9 +545,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                         if (B_MN) {
 #pragma unroll
                             for (int j = 0; j < BN / 64; ++j)
-                                tma_load_2d(map_b, &full_bar[stage], sb + j * 64 * BK * 2, n0 + 64 * j, k0);
+                                tma_load_2d(mb, &full_bar[stage], sb + j * 64 * BK * 2, n0 + 64 * j, kB);
                         } else {
-                            tma_load_2d(map_b, &full_bar[stage], sb, k0, n0);
+                            tma_load_2d(mb, &full_bar[stage], sb, kB, n0);
                         }
                     }
                     ++issued;
@@ -631,6 +661,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                 }
                 tc_fence_after();
                 const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(buf * C::ACC_COLS);
+                // EPI_GLU: from k-block glu_half on, the up half accumulates into
+                // the tile's second accumulator, starting afresh
+                const int half = EPI == EPI_GLU ? batch.prob[x.g].p.glu_half : -1;
                 for (int kb = kb0; kb < kb1; ++kb) {
                     if (!wait_bounded(&full_bar[stage], phase, wc, ST_TIMEOUT_MMA)) {
                         ok = false;
@@ -651,10 +684,13 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                             const uint32_t sas = sa + sub * BM * BK * 2;
                             const uint64_t da = A_MN ? smem_desc_sw128(sas + ks * UMMA_K * 128, 64 * BK * 2, 1024)
                                                      : smem_desc_sw128(sas + ks * UMMA_K * 2, 16, 1024);
+                            const bool second = EPI == EPI_GLU && kb >= half;
+                            const uint32_t acc = (ks > 0 || (kb > kb0 && kb != half)) ? 1u : 0u;
+                            const uint32_t d_acc = d_tmem + (second ? BN : 0);
                             if (PAIR)
-                                umma_f16_pair(d_tmem, da, db, idesc, (kb > kb0 || ks > 0) ? 1u : 0u);
+                                umma_f16_pair(d_acc, da, db, idesc, acc);
                             else
-                                umma_f16(d_tmem + sub * BN, da, db, idesc, (kb > kb0 || ks > 0) ? 1u : 0u);
+                                umma_f16(d_acc + sub * BN, da, db, idesc, acc);
                         }
                     }
                     issued_any = true;
@@ -741,6 +777,24 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             store_box(map, box, x, y);
             if (++out_slot == EPI_OUT_BOXES) out_slot = 0;
         };
+        // store one 32-column chunk of a bf16 output (this thread's row) to the
+        // tensor behind `map` (base `ptr`, pitch d_ld): through the box ring,
+        // or, in the chunk that holds a ragged right edge, with masked direct
+        // stores that leave the row padding untouched
+        auto put = [&](const GemmParams& pp, const CUtensorMap* map, __nv_bfloat16* ptr, const uint32_t (&w)[16],
+                       int col0, int row0, int row) {
+            if ((pp.N & 7) != 0 && col0 + 32 > pp.N) {
+                if (row < pp.M) {
+                    uint16_t* d = reinterpret_cast<uint16_t*>(ptr + row * pp.d_ld + col0);
+                    const int valid = pp.N - col0;
+#pragma unroll
+                    for (int j = 0; j < 32; ++j)   // fully unrolled: w stays in registers
+                        if (j < valid) d[j] = static_cast<uint16_t>((j & 1) ? (w[j >> 1] >> 16) : (w[j >> 1] & 0xFFFFu));
+                }
+                return;
+            }
+            emit(map, w, col0, row0);
+        };
 
         // EPI_DSIGMA: Z boxes run one (tile, chunk) item ahead of their use
         int zu = first_unit, zc = c_first;      // next item whose Z box is to be loaded
@@ -791,8 +845,23 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             for (int c = c_first; c < nch; c += C_STEP) {
                 const int col0 = n_blk * BN + c * 32;
                 if (EPI == EPI_DSIGMA) z_issue();   // the next item's Z box, while this one is processed
+                // EPI_GLU_BWD: this row's Y_gate and Y_up chunk, loaded ahead of the accumulator
+                uint4 yg[4], yu[4];
+                if constexpr (EPI == EPI_GLU_BWD) {
+#pragma unroll
+                    for (int j = 0; j < 4; ++j) {
+                        yg[j] = yu[j] = make_uint4(0u, 0u, 0u, 0u);
+                        if (row < p.M && col0 + 8 * j < p.N) {   // 8-column vectors inside the padded row
+                            const long long off = static_cast<long long>(row) * p.d_ld + col0 + 8 * j;
+                            yg[j] = __ldg(reinterpret_cast<const uint4*>(p.yg_ptr + off));
+                            yu[j] = __ldg(reinterpret_cast<const uint4*>(p.yu_ptr + off));
+                        }
+                    }
+                }
                 uint32_t v[32];
+                uint32_t v2[32];   // EPI_GLU: the same chunk of the up accumulator
                 tmem_ld_32x32b_x32(tbase + c * 32, v);
+                if constexpr (EPI == EPI_GLU) tmem_ld_32x32b_x32(tbase + BN + c * 32, v2);
                 tmem_ld_wait();
                 if (EPI == EPI_F32 || (EPI == EPI_TAIL && split >= 0)) {
                     float* dst = nullptr;
@@ -818,19 +887,46 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 #pragma unroll
                     for (int j = 0; j < 16; ++j)
                         w[j] = pack_bf16x2(__uint_as_float(v[2 * j]), __uint_as_float(v[2 * j + 1]));
-                    if ((p.N & 7) != 0 && col0 + 32 > p.N) {
-                        // ragged right edge: masked per-element stores, padding untouched
-                        if (row < p.M) {
-                            uint16_t* d = reinterpret_cast<uint16_t*>(p.d_ptr + row * p.d_ld + col0);
-                            const int valid = p.N - col0;
+                    put(p, map_d, p.d_ptr, w, col0, row0, row);
+                } else if (EPI == EPI_GLU) {
+                    // Y_gate, Y_up rounded to bf16; M = bf16(Y_gate * Y_up) of the rounded
+                    // values (their product is exact in fp32)
+                    uint32_t wg[16], wu[16];
 #pragma unroll
-                            for (int j = 0; j < 32; ++j)   // fully unrolled: w stays in registers
-                                if (j < valid)
-                                    d[j] = static_cast<uint16_t>((j & 1) ? (w[j >> 1] >> 16) : (w[j >> 1] & 0xFFFFu));
-                        }
-                        continue;
+                    for (int j = 0; j < 16; ++j) {
+                        wg[j] = pack_bf16x2(__uint_as_float(v[2 * j]), __uint_as_float(v[2 * j + 1]));
+                        wu[j] = pack_bf16x2(__uint_as_float(v2[2 * j]), __uint_as_float(v2[2 * j + 1]));
+                        w[j] = pack_bf16x2(bf16_lo(wg[j]) * bf16_lo(wu[j]), bf16_hi(wg[j]) * bf16_hi(wu[j]));
                     }
-                    emit(map_d, w, col0, row0);
+                    put(p, map_d, p.d_ptr, w, col0, row0, row);
+                    if (p.has_d2) {                 // training: Y_gate and Y_up for the backward
+                        put(p, map_d2, p.d2_ptr, wg, col0, row0, row);
+                        put(p, &batch.prob[x.g].map_d3, p.d3_ptr, wu, col0, row0, row);
+                    }
+                } else if (EPI == EPI_GLU_BWD) {
+                    // dM rounded to bf16; dY_gate = bf16(dM * Y_up), dY_up = bf16(dM * Y_gate)
+                    uint32_t dm[16], gw[16], uw[16];
+#pragma unroll
+                    for (int j = 0; j < 4; ++j) {
+                        gw[4 * j] = yg[j].x;
+                        gw[4 * j + 1] = yg[j].y;
+                        gw[4 * j + 2] = yg[j].z;
+                        gw[4 * j + 3] = yg[j].w;
+                        uw[4 * j] = yu[j].x;
+                        uw[4 * j + 1] = yu[j].y;
+                        uw[4 * j + 2] = yu[j].z;
+                        uw[4 * j + 3] = yu[j].w;
+                    }
+#pragma unroll
+                    for (int j = 0; j < 16; ++j) {
+                        dm[j] = pack_bf16x2(__uint_as_float(v[2 * j]), __uint_as_float(v[2 * j + 1]));
+                        w[j] = pack_bf16x2(bf16_lo(dm[j]) * bf16_lo(uw[j]), bf16_hi(dm[j]) * bf16_hi(uw[j]));
+                    }
+                    put(p, map_d, p.d_ptr, w, col0, row0, row);      // dY_gate
+#pragma unroll
+                    for (int j = 0; j < 16; ++j)
+                        w[j] = pack_bf16x2(bf16_lo(dm[j]) * bf16_lo(gw[j]), bf16_hi(dm[j]) * bf16_hi(gw[j]));
+                    put(p, map_d2, p.d2_ptr, w, col0, row0, row);    // dY_up
                 } else if (EPI == EPI_ZH) {
 #pragma unroll
                     for (int j = 0; j < 16; ++j)

@@ -324,6 +324,7 @@ TailPlan plan_tail(const GemmParams* p, int count, int bn, int msub, int sms)
 constexpr int TRACE_PAIR = 4;
 constexpr int TRACE_MSUB2 = 8;
 constexpr int TRACE_TAIL = 16;   // weight gradients with a split tail
+constexpr int TRACE_GLU = 32;    // the dX epilogue stored the gated-MLP gradients dY_gate, dY_up
 
 template <bool A_MN, int EPI>
 int tile_flags(int bn, int msub)
@@ -368,6 +369,22 @@ cudaError_t dispatch(int bn, int msub, GemmBatch& b, int sms, cudaStream_t s)
         if (msub != 1) return launch_gemm<128, 2, A_MN, B_MN, EPI>(b, grid, pdl, s);
     }
     return launch_gemm<128, 1, A_MN, B_MN, EPI>(b, grid, pdl, s);
+}
+
+// The gated-MLP forward launch (EPI_GLU): 128-column tiles, whose two
+// double-buffered accumulators (gate and up) fill TMEM; on CTA pairs (256-row
+// tiles, 64 B columns per CTA) when `pair`.
+cudaError_t dispatch_glu(bool pair, GemmBatch& b, int sms, cudaStream_t s)
+{
+    b.prob[0].unit_begin = 0;
+    b.units = b.prob[0].p.units;
+    const GemmParams& p = b.prob[0].p;
+    const bool pdl = 2.0 * p.M * p.N * (static_cast<double>(p.k_blocks) * BK) < 64e9;
+    if (pair) {
+        const int pairs = b.units < sms / 2 ? b.units : sms / 2;
+        return launch_gemm<128, 1, false, false, EPI_GLU, true>(b, 2 * pairs, pdl, s);
+    }
+    return launch_gemm<128, 1, false, false, EPI_GLU>(b, b.units < sms ? b.units : sms, pdl, s);
 }
 
 }  // namespace

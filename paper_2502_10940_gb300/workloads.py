@@ -34,6 +34,11 @@ class Workload:
     seqs: int = 0
     seq_len: int = 256
     phase: str = "train"    # "train": forward + backward; "infer": forward only, nothing saved
+    # the MLP as LLaMA wires it (Fig. 4): the down layer reads M = Y_gate * Y_up,
+    # formed in the gate/up output GEMM, and its backward hands dY_gate, dY_up
+    # to the gate/up backward; otherwise the down input and the gate/up
+    # upstream gradients are independent synthetic tensors
+    gated: bool = False
 
     @property
     def flops(self) -> float:
@@ -100,11 +105,29 @@ WORKLOADS = {
                         "(128 x 256)", seqs=128),
     "1b-o": Workload("1b-o", 65536, (Layer("o", 2048, 2048, 512, "x_o"),), fused_qkv=False,
                      desc="single CoLA layer, LLaMA-1B o-proj shape, 65536 tokens, 2048->2048, r=512", seqs=256),
+    # the same blocks with the gated MLP chained through the library
+    "60m-gated": Workload("60m-gated", 65536, llama_block(512, 1376, 128), gated=True,
+                          desc="LLaMA-60M-shaped CoLA block with the gated MLP (M = Y_gate * Y_up fused), "
+                               "65536 tokens", seqs=256),
+    "1b-gated": Workload("1b-gated", 65536, llama_block(2048, 5461, 512), modes=("cola", "cola_m"), gated=True,
+                         desc="LLaMA-1B-shaped CoLA block with the gated MLP (M = Y_gate * Y_up fused), "
+                              "65536 tokens", seqs=256),
+    "7b-gated": Workload("7b-gated", 32768, llama_block(4096, 11008, 1024), modes=("cola_m", "cola"), gated=True,
+                         desc="LLaMA-7B-shaped CoLA block with the gated MLP (M = Y_gate * Y_up fused), "
+                              "32768 tokens", seqs=128),
     # inference at the pre-training shapes with 32 sequences of 256 tokens (App. E.2)
     "1b-infer": Workload("1b-infer", 8192, llama_block(2048, 5461, 512), modes=("infer",), phase="infer", desc="LLaMA-1B-shaped CoLA block, forward only (inference), d=2048, "
                                           "d_ff=5461, r=512, 8192 tokens (32 x 256)", seqs=32),
     "7b-infer": Workload("7b-infer", 8192, llama_block(4096, 11008, 1024), modes=("infer",), phase="infer", desc="LLaMA-7B-shaped CoLA block, forward only (inference), d=4096, "
                                           "d_ff=11008, r=1024, 8192 tokens (32 x 256)", seqs=32),
+    "1b-infer-gated": Workload("1b-infer-gated", 8192, llama_block(2048, 5461, 512), modes=("infer",),
+                               phase="infer", gated=True,
+                               desc="LLaMA-1B-shaped CoLA block with the gated MLP, forward only (inference), "
+                                    "8192 tokens (32 x 256)", seqs=32),
+    "7b-infer-gated": Workload("7b-infer-gated", 8192, llama_block(4096, 11008, 1024), modes=("infer",),
+                               phase="infer", gated=True,
+                               desc="LLaMA-7B-shaped CoLA block with the gated MLP, forward only (inference), "
+                                    "8192 tokens (32 x 256)", seqs=32),
     # one new token for each of 32 sequences: every GEMM has a few output tiles
     # (split over K across the SMs) and streams its weights
     "1b-decode": Workload("1b-decode", 32, llama_block(2048, 5461, 512), modes=("infer",), phase="infer", desc="LLaMA-1B-shaped CoLA block, forward only, 32 tokens (one per sequence)",
