@@ -270,6 +270,11 @@ def launch_cost(kind, shapes, splits, flags):
     the fp32 token-split partials of the weight gradients are implementation
     traffic and are not counted."""
     e = 2
+    if kind == "fwd_fused":
+        # X, A and B read, Z / H (as stored) and Y written; H stays on chip
+        (m, r, k1), (_, n_out, _) = shapes
+        nzh = (1 if flags & 1 else 0) + (1 if flags & 64 else 0)
+        return e * (m * k1 + r * k1 + m * r * nzh + n_out * r + m * n_out), 2.0 * m * r * (k1 + n_out)
     tb, tf = 0.0, 0.0
     for (m, n, k) in shapes:
         if kind in ("fwd_zh", "fwd_y") and flags & 2:
@@ -752,6 +757,7 @@ def run_cola(args, wl):
     from paper_2502_10940_gb300.workloads import WORKLOADS
 
     build.build()
+    cola.cola_set_fused_forward(args.fused_forward == "on")
     peaks = _peaks()
     ridge = peaks["bf16_tflops"] * 1e12 / (peaks["hbm_gbs"] * 1e9)
     mode = args.mode or wl.modes[0]
@@ -786,6 +792,7 @@ def run_cola(args, wl):
                        "saved_activation_elems": sum(g[k].numel() for g in blk.groups for k in ("Z", "H")
                                                      if g.get(k) is not None),
                        "cuda_graph": use_graph,
+                       "fused_forward": args.fused_forward == "on",
                        "l2": (f"flushed between steps (256 MB write): working set {tb['ws_bytes'] / 1e6:.1f} MB < L2"
                               if flush is not None else
                               f"no flush: working set {tb['ws_bytes'] / 1e9:.2f} GB > 129 MB L2")},
@@ -943,6 +950,8 @@ def main(argv=None):
                     help="replay each step as one CUDA graph (off: launch every kernel from the host)")
     ap.add_argument("--seed", type=int, default=0)
     ap.add_argument("--no-extras", action="store_true", help="skip e2e, full-rank and CPU baselines")
+    ap.add_argument("--fused-forward", default="on", choices=["on", "off"],
+                    help="single-layer forwards with r <= 128: one fused kernel (on) or two GEMMs (off)")
     ap.add_argument("--gated-unfused", action="store_true",
                     help="gated workloads: the product and its backward as torch element-wise ops (comparison)")
     args = ap.parse_args(argv)

@@ -120,7 +120,13 @@ cola_status_t cola_workspace_init(void* ws, void* stream);
  *                   NULL under COLA_MODE_INFER (Z is then never stored).
  *   H_save [n x r]: output under COLA_MODE_COLA; must be NULL under COLA_M
  *                   and INFER (H is then formed in the workspace and not kept).
- * Two tensor-core GEMMs: Z/H (sigma fused in the epilogue), then Y. */
+ * Two tensor-core GEMMs: Z/H (sigma fused in the epilogue), then Y.  For
+ * r = 64 or 128 when both products are HBM-bound (neither compute-heavy nor
+ * split over K) and n is at most 128 tokens per SM (19456 on GB300), one
+ * kernel instead: each CTA keeps the H of its 128-row tile in shared memory
+ * between the two products (H is an intermediate of Eq. (main-fwd), not an
+ * output), storing Z and H only as the mode saves them; the results are the
+ * same bit for bit (cola_set_fused_forward). */
 cola_status_t cola_fwd(const cola_desc_t* desc, const void* X, const void* A, const void* B, void* Y,
                        void* Z_save, void* H_save, void* ws, size_t ws_bytes, void* stream);
 
@@ -336,7 +342,9 @@ typedef enum {
     COLA_KERNEL_REDUCE = 4,      /* fixed-order sum of the partials       (M, N of the gradient, K=splits) */
     COLA_KERNEL_BWD_DX = 5,      /* dX = dZ A                             (M=n, N=d_in, K=r or 3r) */
     COLA_KERNEL_SIGMA = 6,       /* H = sigma(Z), elementwise             (M=n, N=count r, K=0) */
-    COLA_KERNEL_FWD_GLU = 7      /* M = (H_gate B_gate^T) * (H_up B_up^T) (M=n, N=d_ff, K=2r) */
+    COLA_KERNEL_FWD_GLU = 7,     /* M = (H_gate B_gate^T) * (H_up B_up^T) (M=n, N=d_ff, K=2r) */
+    COLA_KERNEL_FWD_FUSED = 8    /* Z, H = sigma(Z), Y = H B^T in one kernel, count 2:
+                                    (n, r, d_in) and (n, d_out, r) */
 } cola_kernel_t;
 
 typedef struct {
@@ -355,11 +363,18 @@ typedef struct {
                            bit 4: weight gradients with a split tail (splits = pieces per
                                   tail tile; a reduce launch follows when they are > 1);
                            bit 5: the dX epilogue stored the gated-MLP gradients dY_gate,
-                                  dY_up instead of dX (cola_bwd_down_gated) */
+                                  dY_up instead of dX (cola_bwd_down_gated);
+                           bit 6: the fused forward stored Z (bit 0: it stored H) */
 } cola_trace_slot_t;
 
 cola_status_t cola_trace_attach(cola_trace_slot_t* slots, int32_t capacity, int32_t* count);
 cola_status_t cola_trace_detach(void);
+
+/* Process-wide choice of cola_fwd's forward where the single-kernel form
+ * applies (see cola_fwd): 1 (default) runs it, 0 runs the two GEMMs instead,
+ * for comparisons; both give the same results bit for bit.  enable outside
+ * {0, 1}: COLA_ERR_INVALID.  Takes effect for calls made after it returns. */
+cola_status_t cola_set_fused_forward(int32_t enable);
 
 /* Static description of a status code. */
 const char* cola_status_string(cola_status_t status);

@@ -12,6 +12,7 @@
 #include <mutex>
 
 #include "cola.h"
+#include "fused_fwd.cuh"
 #include "gemm_launch.cuh"
 #include "host_plan.cuh"
 
@@ -350,6 +351,70 @@ cola_status_t run_f1(const Shape& s, int sigma, int64_t N, const void* X, const 
     return run_batch<false, false, EPI_ZH>(COLA_KERNEL_FWD_ZH, bn, ms, &pr, mnk, 1, Z && H, sms, st);
 }
 
+}  // namespace
+
+cudaError_t launch_fused_fwd(const FusedFwdParams& p, int r, int grid, bool pdl, cudaStream_t stream);
+
+namespace {
+
+// Whether cola_fwd runs a layer as one fused kernel (cola_set_fused_forward).
+std::atomic<int> g_fused_fwd{1};
+
+// The single-kernel forward applies to one layer with r = 64 or 128 whose
+// two GEMMs are HBM-bound (neither is compute-heavy), with at most one
+// 128-row tile per SM, and not split over K (small launches keep the
+// split-K forward).  Measured at 2048 tokens: -10 to -13 % against the two
+// GEMMs; at 65536 tokens it was 5-13 % slower, so larger launches keep them.
+bool fused_fwd_applies(const Shape& s, int sms)
+{
+    if (!g_fused_fwd.load(std::memory_order_relaxed) || (s.r != 64 && s.r != 128)) return false;
+    if ((s.n + BM - 1) / BM > sms) return false;
+    if (heavy_gemm(s.n, s.r, s.d_in) || heavy_gemm(s.n, s.d_out, s.r)) return false;
+    GemmParams p1 = base_params(s.n, s.r, s.d_in, choose_bn_for(s.n, s.r, s.d_in), 1);
+    if (small_launch_splits(p1.m_tiles * p1.n_tiles, p1.k_blocks, sms) > 1) return false;
+    GemmParams p2 = base_params(s.n, s.d_out, s.r, choose_bn_for(s.n, s.d_out, s.r), 1);
+    return small_launch_splits(p2.m_tiles * p2.n_tiles, p2.k_blocks, sms) == 1;
+}
+
+// F1 + F2 in one kernel: Z = X A^T, H = sigma(Z) kept on chip, Y = H B^T;
+// Z and H stored when not null.
+cola_status_t run_fused_fwd(const Shape& s, int sigma, const void* X, const void* A, const void* B, void* Y, void* Z,
+                            void* H, unsigned int* status, int sms, cudaStream_t st)
+{
+    FusedFwdParams p;
+    std::memset(&p, 0, sizeof p);
+    COLA_MAP(map_kmajor(&p.map_x, X, s.d_in, s.n, s.ld_x, BM));
+    COLA_MAP(map_kmajor(&p.map_a, A, s.d_in, s.r, s.ld_a, static_cast<int>(s.r)));
+    COLA_MAP(map_kmajor(&p.map_b, B, s.r, s.d_out, s.r, FBN));
+    COLA_MAP(map_box32(&p.map_y, Y, s.d_out, s.n, s.ld_y));
+    p.map_z = p.map_h = p.map_y;
+    if (Z) COLA_MAP(map_box32(&p.map_z, Z, s.r, s.n, s.r));
+    if (H) COLA_MAP(map_box32(&p.map_h, H, s.r, s.n, s.r));
+    p.n = static_cast<int>(s.n);
+    p.d_out = static_cast<int>(s.d_out);
+    p.kb1 = static_cast<int>((s.d_in + BK - 1) / BK);
+    p.m_tiles = static_cast<int>((s.n + BM - 1) / BM);
+    p.n_blocks = static_cast<int>((s.d_out + FBN - 1) / FBN);
+    // the Y blocks of a tile shared by up to sms / m_tiles work items
+    int groups = sms / (p.m_tiles > 0 ? p.m_tiles : 1);
+    groups = std::max(1, std::min(groups, p.n_blocks));
+    p.blocks_per_group = (p.n_blocks + groups - 1) / groups;
+    p.y_groups = (p.n_blocks + p.blocks_per_group - 1) / p.blocks_per_group;
+    p.store_z = Z != nullptr;
+    p.store_h = H != nullptr;
+    p.sigma = sigma;
+    p.y_ptr = static_cast<__nv_bfloat16*>(Y);
+    p.y_ld = s.ld_y;
+    p.status = status;
+    const int items = p.m_tiles * p.y_groups;
+    const int grid = items < sms ? items : sms;
+    const double flops = 2.0 * s.n * s.r * (s.d_in + s.d_out);
+    const int64_t mnk[2][3] = {{s.n, s.r, s.d_in}, {s.n, s.d_out, s.r}};
+    const int flags = (H ? 1 : 0) | (Z ? TRACE_Z : 0);
+    return launched(traced(COLA_KERNEL_FWD_FUSED, 2, mnk, 1, flags, st,
+                           [&] { return launch_fused_fwd(p, static_cast<int>(s.r), grid, flops < 64e9, st); }));
+}
+
 // F2: Y_j = H_j B_j^T for `count` projections of one shape (H_j [n x r] with
 // pitch ldh; Y_j pitch ld_y), one launch
 cola_status_t run_f2(const Shape& s, int count, const void* const* H, int64_t ldh, const void* const* B,
@@ -686,6 +751,8 @@ cola_status_t cola_fwd(const cola_desc_t* desc, const void* X, const void* A, co
     void* H = desc->mode != COLA_MODE_COLA ? static_cast<void*>(wsb(ws) + L.h_off) : H_save;
     float* part = reinterpret_cast<float*>(wsb(ws) + L.part_off);
     const size_t part_bytes = L.total - L.part_off;
+    if (fused_fwd_applies(s, sms))
+        return run_fused_fwd(s, desc->sigma, X, A, B, Y, Z_save, H_save, status, sms, st);
     COLA_TRY(run_f1(s, desc->sigma, s.r, X, A, Z_save, H, s.r, part, part_bytes, status, sms, st));
     const void* Hs[1] = {H};
     const void* Bs[1] = {B};
@@ -977,6 +1044,13 @@ cola_status_t cola_check_status(void* ws, void* stream, uint32_t* code_out)
         if (cudaMemset(ws, 0, sizeof code) != cudaSuccess) return COLA_ERR_LAUNCH;
         return COLA_ERR_DEVICE_TIMEOUT;
     }
+    return COLA_OK;
+}
+
+cola_status_t cola_set_fused_forward(int32_t enable)
+{
+    if (enable != 0 && enable != 1) return COLA_ERR_INVALID;
+    g_fused_fwd.store(enable, std::memory_order_relaxed);
     return COLA_OK;
 }
 

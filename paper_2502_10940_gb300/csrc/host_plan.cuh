@@ -325,6 +325,7 @@ constexpr int TRACE_PAIR = 4;
 constexpr int TRACE_MSUB2 = 8;
 constexpr int TRACE_TAIL = 16;   // weight gradients with a split tail
 constexpr int TRACE_GLU = 32;    // the dX epilogue stored the gated-MLP gradients dY_gate, dY_up
+constexpr int TRACE_Z = 64;      // the fused forward stored Z
 
 template <bool A_MN, int EPI>
 int tile_flags(int bn, int msub)

@@ -181,6 +181,12 @@ def test_pair_selftest_argument_errors(L):
     assert f(FAKE, 4096, 2, None) == 4           # smaller than the status word plus the operands
 
 
+def test_set_fused_forward_argument_errors(L):
+    f = L.lib().cola_set_fused_forward
+    assert f(2) == 1 and f(-1) == 1
+    assert f(1) == 0                             # the default, restored
+
+
 def test_workspace_init_and_check_reject_null(L):
     assert L.lib().cola_workspace_init(None, None) == 1
     assert L.lib().cola_workspace_init(FAKE + 16, None) == 2   # not 256-byte aligned
