@@ -148,7 +148,10 @@ WgradPlan wgrad_plan(const cola_desc_t& d, int nproj, int sms)
 TailPlan wgrad_tail_plan(const WgradPlan& w, int64_t ntok, int sms)
 {
     GemmParams p[MAX_GROUP];
-    for (int j = 0; j < w.count; ++j) p[j] = base_params(w.p[j].M, w.p[j].N, ntok, w.bn, w.msub);
+    for (int j = 0; j < w.count; ++j) {
+        p[j] = base_params(w.p[j].M, w.p[j].N, ntok, w.bn, w.msub);
+        p[j].n_major = w.p[j].n_major;
+    }
     return plan_tail(p, w.count, w.bn, w.msub, sms);
 }
 
@@ -598,6 +601,7 @@ cola_status_t run_wgrad_tail(const WgradPlan& w, int64_t ntok, const WgradJob* j
     std::memset(&rd, 0, sizeof rd);
     for (int j = 0; j < w.count; ++j) {
         pr[j].p = base_params(w.p[j].M, w.p[j].N, ntok, w.bn, w.msub);
+        pr[j].p.n_major = w.p[j].n_major;
         const GemmParams& pj = pr[j].p;
         COLA_MAP(map_mnmajor(&pr[j].map_a, jobs[j].P, pj.M, ntok, jobs[j].ldp));
         COLA_MAP(map_mnmajor(&pr[j].map_b, jobs[j].Q, pj.N, ntok, jobs[j].ldq));

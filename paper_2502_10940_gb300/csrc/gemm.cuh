@@ -106,6 +106,11 @@ struct GemmParams {
     long long part_stride; // EPI_F32: elements per split slab
     int has_d2;            // EPI_ZH / EPI_DSIGMA: also store H through map_d2
     int h_only;            // EPI_ZH: store H = sigma(bf16(acc)) through map_d and nothing else
+    // tile order within the problem: 0 = row-major (n_blk fastest), 1 =
+    // column-major (m_blk fastest).  A wave of CTAs walking the reduction in
+    // step reads each B-operand panel of its tiles once; column-major keeps a
+    // wave on few B panels, for problems whose B operand is the larger one.
+    int n_major;
     // The bf16 output behind map_d, for the one 32-column chunk per row block
     // that holds a ragged right edge (N % 8 != 0): a TMA store clips at
     // 16-byte granularity and would write the row padding past column N, so
@@ -245,14 +250,25 @@ __device__ __forceinline__ bool wait_bounded(uint64_t* bar, uint32_t parity, con
     }
 }
 
+// The (m_blk, n_blk) of tile `t` of a problem in its tile order.
+__host__ __device__ __forceinline__ void tile_coords(const GemmParams& p, int t, int& m_blk, int& n_blk)
+{
+    if (p.n_major) {
+        n_blk = t / p.m_tiles;
+        m_blk = t - n_blk * p.m_tiles;
+    } else {
+        m_blk = t / p.n_tiles;
+        n_blk = t - m_blk * p.n_tiles;
+    }
+}
+
 __device__ __forceinline__ void decode_unit(const GemmParams& p, int u, int& m_blk, int& n_blk, int& split,
                                             int& kb0, int& kb1)
 {
     const int tiles = p.m_tiles * p.n_tiles;
     split = u / tiles;
     const int rem = u - split * tiles;
-    m_blk = rem / p.n_tiles;
-    n_blk = rem - m_blk * p.n_tiles;
+    tile_coords(p, rem, m_blk, n_blk);
     kb0 = split * p.kb_per_split;
     kb1 = min(kb0 + p.kb_per_split, p.k_blocks);
 }
@@ -344,11 +360,8 @@ __device__ __forceinline__ bool work_next(const GemmBatch& b, int unit_step, Wor
 #pragma unroll
         for (int q = 1; q < MAX_GROUP; ++q)
             if (q < b.count && t >= b.tile_begin[q]) g = q;
-        const int rem = t - b.tile_begin[g];
-        const int nt = b.prob[g].p.n_tiles;
         x.g = g;
-        x.m_blk = rem / nt;
-        x.n_blk = rem - x.m_blk * nt;
+        tile_coords(b.prob[g].p, t - b.tile_begin[g], x.m_blk, x.n_blk);
         x.split = split;
         x.kb0 = k0;
         x.kb1 = k1;

@@ -221,6 +221,9 @@ WgradPlan plan_wgrad(const int64_t* M, const int64_t* N, int count, int64_t ntok
     int tiles = 0;
     for (int i = 0; i < count; ++i) {
         w.p[i] = base_params(M[i], N[i], ntok, w.bn, w.msub);
+        // the token-major operands are read along the whole reduction: walk
+        // the tiles so that a wave shares the panels of the larger one
+        w.p[i].n_major = N[i] > M[i] ? 1 : 0;
         tiles += w.p[i].m_tiles * w.p[i].n_tiles;
     }
     const int S = choose_splits(tiles, w.p[0].k_blocks, w.bn, w.msub, sms);
@@ -305,11 +308,12 @@ TailPlan plan_tail(const GemmParams* p, int count, int bn, int msub, int sms)
             int g = 0;
             for (int j = 1; j < count; ++j)
                 if (t >= s.tile_begin[j]) g = j;
-            const int rem = t - s.tile_begin[g];
+            int mb = 0, nb = 0;
+            tile_coords(p[g], t - s.tile_begin[g], mb, nb);
             TailTile& e = s.tile[i];
             e.g = g;
-            e.m0 = rem / p[g].n_tiles * rows;
-            e.n0 = rem % p[g].n_tiles * bn;
+            e.m0 = mb * rows;
+            e.n0 = nb * bn;
             e.lo_slot = i * s.pieces;
             e.count = s.pieces;
         }

@@ -103,6 +103,11 @@ WORKLOADS = {
     "7b": Workload("7b", 32768, llama_block(4096, 11008, 1024), modes=("cola_m", "cola"),
                    desc="LLaMA-7B-shaped CoLA block, d=4096, d_ff=11008, r=1024, 32768 tokens "
                         "(128 x 256)", seqs=128),
+    # the 7B block at a quarter of its tokens: small enough for ncu captures
+    # with many metrics, large enough that every GEMM keeps its tile
+    # configuration (CTA pairs)
+    "7b-8k": Workload("7b-8k", 8192, llama_block(4096, 11008, 1024), modes=("cola_m", "cola"),
+                      desc="LLaMA-7B-shaped CoLA block, 8192 tokens (32 x 256), for profiling", seqs=32),
     "1b-o": Workload("1b-o", 65536, (Layer("o", 2048, 2048, 512, "x_o"),), fused_qkv=False,
                      desc="single CoLA layer, LLaMA-1B o-proj shape, 65536 tokens, 2048->2048, r=512", seqs=256),
     # the same blocks with the gated MLP chained through the library
