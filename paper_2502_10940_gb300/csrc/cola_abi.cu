@@ -642,15 +642,21 @@ cola_status_t run_glu(const Shape& s, const void* H_cat, int64_t ldh, const void
     const int64_t K2 = 2 * s.r;
     const bool pair = heavy_gemm(s.n, s.d_out, K2) && s.r >= 512;
     const int msub = pair ? TILE_PAIR : 1;
+    // 256-column pair tiles hold one tile in TMEM, so the next tile's up half
+    // waits for this tile's stores: worth it when the epilogue stores M alone
+    // or a half runs long (r >= 1024).  Measured: 7B inference GLU 355 -> 230
+    // us, 7B training -3 % per block; 1B training 912 -> 1110 us, which keeps
+    // the double-buffered 128-column pair tiles.
+    const int bn = pair && (Yg == nullptr || s.r >= 1024) ? 256 : 128;
     GemmBatch b;
     std::memset(&b, 0, sizeof b);
     b.count = 1;
     GemmProblem& pr = b.prob[0];
-    pr.p = base_params(s.n, s.d_out, K2, 128, msub);
+    pr.p = base_params(s.n, s.d_out, K2, bn, msub);
     pr.p.glu_half = static_cast<int>(s.r / BK);
     COLA_MAP(map_kmajor(&pr.map_a, H_cat, K2, s.n, ldh, a_box_rows(msub)));
-    COLA_MAP(map_kmajor(&pr.map_b, Bg, s.r, s.d_out, s.r, b_box_rows(128, msub)));
-    COLA_MAP(map_kmajor(&pr.map_b2, Bu, s.r, s.d_out, s.r, b_box_rows(128, msub)));
+    COLA_MAP(map_kmajor(&pr.map_b, Bg, s.r, s.d_out, s.r, b_box_rows(bn, msub)));
+    COLA_MAP(map_kmajor(&pr.map_b2, Bu, s.r, s.d_out, s.r, b_box_rows(bn, msub)));
     COLA_MAP(map_box32(&pr.map_d, M, s.d_out, s.n, s.ld_y));
     pr.map_d2 = pr.map_d3 = pr.map_z = pr.map_d;
     if (Yg) {
@@ -665,7 +671,7 @@ cola_status_t run_glu(const Shape& s, const void* H_cat, int64_t ldh, const void
     pr.p.status = status;
     const int64_t mnk[1][3] = {{s.n, s.d_out, K2}};
     const int flags = (Yg ? 1 : 0) | (pair ? TRACE_PAIR : 0);
-    return launched(traced(COLA_KERNEL_FWD_GLU, 1, mnk, 1, flags, st, [&] { return dispatch_glu(pair, b, sms, st); }));
+    return launched(traced(COLA_KERNEL_FWD_GLU, 1, mnk, 1, flags, st, [&] { return dispatch_glu(bn, pair, b, sms, st); }));
 }
 
 // The down layer's input gradient when its input is M = Y_gate * Y_up: the

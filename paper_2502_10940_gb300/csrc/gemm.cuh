@@ -148,7 +148,9 @@ constexpr int EPI_SMEM_BYTES = NUM_EPI_WARPS * EPI_WARP_BYTES;
 // MMAs per k-step that share one B tile (halving the B-operand traffic per
 // output row), into two TMEM accumulators of BN columns each.  ACCS = 2: one
 // 128-row tile with two accumulators (the gate and up halves of EPI_GLU).
-template <int BN, int MSUB, bool PAIR = false, int ACCS = 1>
+// BUFS: tiles whose accumulators TMEM holds at once (2: the epilogue of one
+// tile overlaps the main loop of the next).
+template <int BN, int MSUB, bool PAIR = false, int ACCS = 1, int BUFS = 2>
 struct GemmCfg {
     static_assert(BN % 64 == 0 && BN >= 64 && BN <= 256, "BN must be 64..256 in steps of 64");
     static_assert(MSUB == 1 || MSUB == 2, "one or two 128-row sub-tiles");
@@ -157,7 +159,7 @@ struct GemmCfg {
     static constexpr int CTA_ROWS = PAIR ? BM : TILE_M;          // rows of A this CTA loads
     static constexpr int B_ROWS = PAIR ? BN / 2 : BN;           // columns of B this CTA loads
     static constexpr int ACC_COLS = (MSUB > ACCS ? MSUB : ACCS) * BN;   // TMEM columns of one tile's accumulators
-    static_assert(2 * ACC_COLS <= 512, "double-buffered accumulator must fit TMEM");
+    static_assert(BUFS * ACC_COLS <= 512, "the accumulators must fit TMEM");
     static constexpr int A_BYTES = CTA_ROWS * BK * 2;
     static constexpr int B_BYTES = B_ROWS * BK * 2;
     static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
@@ -165,7 +167,7 @@ struct GemmCfg {
     static constexpr int SMEM_LIMIT = 232448;   // opt-in maximum per CTA
     static constexpr int STAGES_FIT = (SMEM_LIMIT - 1024 - BAR_BYTES - EPI_SMEM_BYTES) / STAGE_BYTES;
     static constexpr int STAGES = STAGES_FIT > 8 ? 8 : STAGES_FIT;
-    static constexpr int TMEM_COLS = (2 * ACC_COLS <= 128) ? 128 : (2 * ACC_COLS <= 256 ? 256 : 512);
+    static constexpr int TMEM_COLS = (BUFS * ACC_COLS <= 128) ? 128 : (BUFS * ACC_COLS <= 256 ? 256 : 512);
     static constexpr int SMEM_BYTES = 1024 + STAGES * STAGE_BYTES + EPI_SMEM_BYTES + BAR_BYTES;
     static_assert(SMEM_BYTES <= SMEM_LIMIT, "shared memory budget");
 };
@@ -409,7 +411,14 @@ template <int BN, int MSUB, bool A_MN, bool B_MN, int EPI, bool PAIR = false>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
     gemm_kernel(const __grid_constant__ GemmBatch batch)
 {
-    using C = GemmCfg<BN, MSUB, PAIR, EPI == EPI_GLU ? 2 : 1>;
+    // EPI_GLU with 256-column tiles: the gate and up accumulators of one tile
+    // fill TMEM, so there is one tile slot, and its two accumulators are
+    // released apart: the epilogue copies the gate half to registers and frees
+    // it at once (tempty_bar[0]), so the MMAs of the next tile's gate half
+    // overlap this tile's up-half epilogue; the up half is freed when stored
+    // (tempty_bar[1]).
+    constexpr bool GLU_SPLIT = EPI == EPI_GLU && BN == 256;
+    using C = GemmCfg<BN, MSUB, PAIR, EPI == EPI_GLU ? 2 : 1, GLU_SPLIT ? 1 : 2>;
     constexpr int STAGES = C::STAGES;
     constexpr int TILE_M = C::TILE_M;
     extern __shared__ uint8_t smem_raw[];
@@ -673,11 +682,18 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                     break;
                 }
                 tc_fence_after();
-                const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(buf * C::ACC_COLS);
+                const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(GLU_SPLIT ? 0 : buf * C::ACC_COLS);
                 // EPI_GLU: from k-block glu_half on, the up half accumulates into
                 // the tile's second accumulator, starting afresh
                 const int half = EPI == EPI_GLU ? batch.prob[x.g].p.glu_half : -1;
                 for (int kb = kb0; kb < kb1; ++kb) {
+                    if (GLU_SPLIT && kb == half) {   // the up accumulator, freed by the previous tile's epilogue
+                        if (!wait_bounded<PAIR>(&tempty_bar[1], bphase ^ 1u, wc, ST_TIMEOUT_MMA)) {
+                            ok = false;
+                            break;
+                        }
+                        tc_fence_after();
+                    }
                     if (!wait_bounded(&full_bar[stage], phase, wc, ST_TIMEOUT_MMA)) {
                         ok = false;
                         break;
@@ -723,7 +739,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                     umma_commit_pair(&tfull_bar[buf], 0x3);
                 else
                     umma_commit(&tfull_bar[buf]);
-                if (++buf == 2) {
+                if (GLU_SPLIT) {
+                    bphase ^= 1u;   // one slot: buf stays 0
+                } else if (++buf == 2) {
                     buf = 0;
                     bphase ^= 1u;
                 }
@@ -853,7 +871,57 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             if (!wait_bounded(&tfull_bar[buf], bphase, wc, ST_TIMEOUT_EPILOGUE)) break;
             tc_fence_after();
             const uint32_t tbase = tmem_base + (static_cast<uint32_t>(q * 32) << 16) +
-                                   static_cast<uint32_t>(buf * C::ACC_COLS + sub * BN);
+                                   static_cast<uint32_t>((GLU_SPLIT ? 0 : buf * C::ACC_COLS) + sub * BN);
+            if constexpr (GLU_SPLIT) {
+                // the gate half of this warp's chunks into registers, then free it
+                uint32_t gsave[BN / 64][16];
+#pragma unroll
+                for (int i = 0; i < BN / 64; ++i) {
+                    const int c = c_first + C_STEP * i;
+                    if (c < nch) {
+                        uint32_t v[32];
+                        tmem_ld_32x32b_x32(tbase + c * 32, v);
+                        tmem_ld_wait();
+#pragma unroll
+                        for (int j = 0; j < 16; ++j)
+                            gsave[i][j] = pack_bf16x2(__uint_as_float(v[2 * j]), __uint_as_float(v[2 * j + 1]));
+                    }
+                }
+                tc_fence_before();
+                if (PAIR)
+                    mbar_arrive_cluster(mapa_shared(smem_u32(&tempty_bar[0]), 0));
+                else
+                    mbar_arrive(&tempty_bar[0]);
+                // the up half: M = bf16(Y_gate * Y_up), and Y_gate, Y_up when training
+#pragma unroll
+                for (int i = 0; i < BN / 64; ++i) {
+                    const int c = c_first + C_STEP * i;
+                    if (c < nch) {
+                        const int col0 = n_blk * BN + c * 32;
+                        uint32_t v[32];
+                        tmem_ld_32x32b_x32(tbase + BN + c * 32, v);
+                        tmem_ld_wait();
+                        uint32_t wu[16], w[16];
+#pragma unroll
+                        for (int j = 0; j < 16; ++j) {
+                            wu[j] = pack_bf16x2(__uint_as_float(v[2 * j]), __uint_as_float(v[2 * j + 1]));
+                            w[j] = pack_bf16x2(bf16_lo(gsave[i][j]) * bf16_lo(wu[j]), bf16_hi(gsave[i][j]) * bf16_hi(wu[j]));
+                        }
+                        put(p, map_d, p.d_ptr, w, col0, row0, row);
+                        if (p.has_d2) {
+                            put(p, map_d2, p.d2_ptr, gsave[i], col0, row0, row);
+                            put(p, &batch.prob[x.g].map_d3, p.d3_ptr, wu, col0, row0, row);
+                        }
+                    }
+                }
+                tc_fence_before();
+                if (PAIR)
+                    mbar_arrive_cluster(mapa_shared(smem_u32(&tempty_bar[1]), 0));
+                else
+                    mbar_arrive(&tempty_bar[1]);
+                bphase ^= 1u;
+                continue;
+            }
 #pragma unroll 1
             for (int c = c_first; c < nch; c += C_STEP) {
                 const int col0 = n_blk * BN + c * 32;

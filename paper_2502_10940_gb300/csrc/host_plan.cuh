@@ -376,10 +376,11 @@ cudaError_t dispatch(int bn, int msub, GemmBatch& b, int sms, cudaStream_t s)
     return launch_gemm<128, 1, A_MN, B_MN, EPI>(b, grid, pdl, s);
 }
 
-// The gated-MLP forward launch (EPI_GLU): 128-column tiles, whose two
-// double-buffered accumulators (gate and up) fill TMEM; on CTA pairs (256-row
-// tiles, 64 B columns per CTA) when `pair`.
-cudaError_t dispatch_glu(bool pair, GemmBatch& b, int sms, cudaStream_t s)
+// The gated-MLP forward launch (EPI_GLU) with `bn`-column tiles: on CTA
+// pairs (when `pair`) either 256 x 256 tiles with one TMEM slot whose gate and
+// up accumulators are freed apart, or 256 x 128 tiles with two
+// double-buffered slots; 128 x 128 tiles on single CTAs.
+cudaError_t dispatch_glu(int bn, bool pair, GemmBatch& b, int sms, cudaStream_t s)
 {
     b.prob[0].unit_begin = 0;
     b.units = b.prob[0].p.units;
@@ -387,6 +388,7 @@ cudaError_t dispatch_glu(bool pair, GemmBatch& b, int sms, cudaStream_t s)
     const bool pdl = 2.0 * p.M * p.N * (static_cast<double>(p.k_blocks) * BK) < 64e9;
     if (pair) {
         const int pairs = b.units < sms / 2 ? b.units : sms / 2;
+        if (bn == 256) return launch_gemm<256, 1, false, false, EPI_GLU, true>(b, 2 * pairs, pdl, s);
         return launch_gemm<128, 1, false, false, EPI_GLU, true>(b, 2 * pairs, pdl, s);
     }
     return launch_gemm<128, 1, false, false, EPI_GLU>(b, b.units < sms ? b.units : sms, pdl, s);

@@ -265,3 +265,37 @@ def test_gated_mlp_1b_widths_on_pairs_sampled():
     assert_close("dY_gate rows", to64(dYg[ridx]), dYg_o)
     assert_close("dY_up rows", to64(dYu[ridx]), dYu_o)
     assert padding_intact(dYg, d_ff) and padding_intact(dYu, d_ff)
+
+
+@pytest.mark.parametrize("shape", [(8200, 4096, 11008, 1024), (8320, 2048, 5461, 512)], ids=str)
+def test_gate_up_256_column_pair_tiles(shape):
+    # 7B widths in training (r = 1024) and 1B widths in inference: the product
+    # GEMM on 256 x 256 CTA-pair tiles with one TMEM slot whose gate and up
+    # accumulators are freed apart.  Sampled rows against the oracle, M the
+    # product of the stored outputs bit for bit, and the inference M equal to
+    # the training M
+    n, d, d_ff, r = shape
+    t = _mlp(n, d, d_ff, r, seed=85)
+    f = _forward(t, n, d, d_ff, r, "cola_m")
+    fi = _forward(t, n, d, d_ff, r, "infer")
+    assert f["trace"][-1][0] == "fwd_glu" and f["trace"][-1][3] & PAIR, f["trace"]
+    assert fi["trace"][-1][0] == "fwd_glu" and fi["trace"][-1][3] & PAIR, fi["trace"]
+    assert torch.equal(fi["M"], f["M"])
+    assert torch.equal(f["M"], _product_bits(f["Yg"], f["Yu"]))
+    rows = np.array([0, 255, 256, 4097, n - 257, n - 200, n - 1])
+    ridx = torch.from_numpy(rows).cuda()
+
+    def bits(x):
+        return I.bf16_bits(torch.as_strided(x, (x.shape[0], x.stride(0)), (x.stride(0), 1)))
+
+    Xb = bits(t["X"])
+    _, _, Yg_o = oracle.rows_bf16(Xb, I.bf16_bits(t["Ag"]), I.bf16_bits(t["Bg"]), rows, None, "silu", d_in=d,
+                                  d_out=d_ff)
+    _, _, Yu_o = oracle.rows_bf16(Xb, I.bf16_bits(t["Au"]), I.bf16_bits(t["Bu"]), rows, None, "silu", d_in=d,
+                                  d_out=d_ff)
+    assert_close("Y_gate rows", to64(f["Yg"][ridx]), Yg_o)
+    assert_close("Y_up rows", to64(f["Yu"][ridx]), Yu_o)
+    assert_close("M rows", to64(f["M"][ridx]), oracle.gate_up_product(Yg_o, Yu_o))
+    for k in ("M", "Yg", "Yu"):
+        assert padding_intact(f[k], d_ff), k
+    assert padding_intact(fi["M"], d_ff)
