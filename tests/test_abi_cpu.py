@@ -165,6 +165,28 @@ def test_infer_mode_argument_errors(L):
     assert f(ctypes.byref(dc), FAKE, FAKE, FAKE, FAKE, None, None, FAKE, 1 << 20, None) == 1
 
 
+def test_gated_mlp_argument_errors(L):
+    # cola_fwd_gate_up(desc, X, A_cat, B_gate, B_up, M, Y_gate, Y_up, Z_cat, H_cat, ws, ws_bytes, stream)
+    f = L.lib().cola_fwd_gate_up
+    d = L.desc(256, 128, 344, 64, mode="cola")
+    assert f(ctypes.byref(d), FAKE, FAKE, FAKE, FAKE, None, FAKE, FAKE, FAKE, FAKE, FAKE, 1 << 20, None) == 1  # no M
+    assert f(ctypes.byref(d), FAKE, FAKE, FAKE, FAKE, FAKE, None, FAKE, FAKE, FAKE, FAKE, 1 << 20, None) == 1  # training needs Y_gate
+    assert f(ctypes.byref(d), FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE + 2, FAKE, FAKE, FAKE, 1 << 20, None) == 2
+    assert f(ctypes.byref(d), FAKE, FAKE, FAKE + 8, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, 1 << 20, None) == 2
+    assert f(ctypes.byref(d), FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, None, FAKE, 1 << 20, None) == 1  # CoLA saves H
+    di = L.desc(256, 128, 344, 64, mode="infer")
+    assert f(ctypes.byref(di), FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, None, None, FAKE, 1 << 20, None) == 1  # inference: no Y_gate
+    assert f(ctypes.byref(L.desc(256, 128, 344, 100)), *([FAKE] * 10), 1 << 20, None) == 3   # r % 64
+    # cola_bwd_down_gated(desc, M, A, B, dY, Z, H, Y_gate, Y_up, dY_gate, dY_up, dA, dB, ws, ws_bytes, stream)
+    g = L.lib().cola_bwd_down_gated
+    dd = L.desc(256, 344, 128, 64, ld_x=352, mode="cola_m")
+    assert g(ctypes.byref(dd), *([FAKE] * 5), FAKE, *([FAKE] * 7), 1 << 20, None) == 1                # H under CoLA-M
+    assert g(ctypes.byref(dd), *([FAKE] * 5), None, FAKE, None, *([FAKE] * 5), 1 << 20, None) == 1    # no Y_up
+    assert g(ctypes.byref(dd), *([FAKE] * 5), None, FAKE, FAKE, FAKE + 4, *([FAKE] * 4), 1 << 20, None) == 2
+    assert g(ctypes.byref(L.desc(256, 344, 128, 64, mode="infer")), *([FAKE] * 5), None, *([FAKE] * 7), 1 << 20,
+             None) == 1                                                                               # no backward in inference
+
+
 def test_selftest_argument_errors(L):
     f = L.lib().cola_selftest_wait_timeout
     assert f(None, 1 << 20, None) == 1
