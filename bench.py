@@ -156,41 +156,54 @@ class Block:
         chained = self._chained()
         return [t for t in ins if id(t) not in chained]
 
-    def add_input_set(self):
-        """A second set of the step's input buffers (same shapes and pitches),
-        so that the next step's inputs can be copied in while this step runs;
-        bind(i) selects the set the next step reads."""
+    def add_io_set(self):
+        """A second set of the step's input and result buffers (same shapes
+        and pitches), so that the next step's inputs can be copied in, and the
+        last step's results copied out, while this step runs; bind(i) selects
+        the set the next step reads and writes."""
         torch = self.torch
 
         def twin(t):
             full = torch.as_strided(t, (t.shape[0], t.stride(0)), (t.stride(0), 1))
             return full.clone()[:, :t.shape[1]]
 
-        if not hasattr(self, "input_sets"):
-            self.input_sets = [(dict(self.X), [s["dY"] for s in self.layers])]
-        X2 = {k: twin(v) for k, v in self.X.items()}
-        dY2 = [twin(s["dY"]) if s["dY"] is not None else None for s in self.layers]
-        self.input_sets.append((X2, dY2))
+        if not hasattr(self, "io_sets"):
+            self.io_sets = [(dict(self.X), [s["dY"] for s in self.layers], self.step_results())]
+        X0, dY0, R0 = self.io_sets[0]
+        X2 = {k: twin(v) for k, v in X0.items()}
+        dY2 = [twin(d) if d is not None else None for d in dY0]
+        R2 = [twin(t) for t in R0]
+        self.io_sets.append((X2, dY2, R2))
 
     def bind(self, i):
-        X, dY = self.input_sets[i]
+        X, dY, R = self.io_sets[i]
         self.X = dict(X)
         for s, d in zip(self.layers, dY):
             s["X"] = X[s["L"].x]
             s["dY"] = d
         for g in self.groups:
             g["X"] = X[g["members"][0]["L"].x]
+        for (obj, key), t in zip(self._result_slots(), R):
+            obj[key] = t
 
     # what a step hands back: the weight gradients and the block's input
     # gradients (training), or the outputs (inference)
-    def step_results(self):
+    def _result_slots(self):
         if not self.train:
-            return [s["Y"] for s in self.layers]
-        return ([g["dA"] for g in self.groups] + [s["dB"] for s in self.layers] +
-                [g["dX"] for g in self.groups if g["dX"] is not None])
+            # a gated MLP's gate and up outputs are consumed inside the kernel
+            # that forms M = Y_gate * Y_up: not results
+            inner = {id(m) for g in self.groups if "M_key" in g and not self.gated_unfused for m in g["members"]}
+            return [(s, "Y") for s in self.layers if id(s) not in inner]
+        return ([(g, "dA") for g in self.groups] + [(s, "dB") for s in self.layers] +
+                [(g, "dX") for g in self.groups if g["dX"] is not None])
+
+    def step_results(self):
+        return [obj[key] for obj, key in self._result_slots()]
 
     def results_words(self):
         if not self.train:
+            if self.gated and not self.gated_unfused:
+                return "Y of every layer but gate and up (M = Y_gate * Y_up feeds the down layer on the device)"
             return "Y of every layer"
         if self.gated:
             return ("dA and dB of every layer and dX of the attention and gate/up input groups; Y, Z and H stay "
@@ -397,6 +410,7 @@ class ClockSampler:
         self._nvml = None
         self._h = None
         self._smi = None
+        self._opened = False
 
     def _open_nvml(self):
         import ctypes
@@ -429,12 +443,21 @@ class ClockSampler:
         self._nvml.nvmlDeviceGetPowerUsage(self._h, ctypes.byref(pw))
         self.samples.append((float(c.value), int(r.value), pw.value / 1000.0))
 
-    def start(self):
-        import threading
+    def open(self):
+        """Load NVML (this can take a while on a cold start).  Called before
+        the warm-up, so that the GPU does not idle between the warm-up and
+        the timed region."""
+        if self._opened:
+            return
+        self._opened = True
         try:
             self._open_nvml()
         except Exception:  # noqa: BLE001 -- no NVML: use nvidia-smi instead
             self._nvml = None
+
+    def start(self):
+        import threading
+        self.open()
         if self._nvml is None:
             try:
                 self._smi = subprocess.Popen(
@@ -567,6 +590,34 @@ def run_reference(args, wl):
     return 0
 
 
+# untimed steps after the warm-up until the GPU has run this long, so that the
+# timed steps see the clocks and power state of sustained load (a GPU coming
+# out of idle ramps its clocks up; a 1.4 kW part under a tensor-bound load
+# reaches its power cap within a few hundred milliseconds)
+SETTLE_S = 0.5
+
+
+def settle_steps(fn, seconds, max_steps=20000):
+    """Run fn() until `seconds` of wall time have passed with the device kept
+    busy (synchronising after each batch of calls); returns the steps run and
+    the seconds taken."""
+    import torch
+
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    n, batch = 0, 1
+    while n < max_steps:
+        for _ in range(batch):
+            fn()
+        n += batch
+        torch.cuda.synchronize()
+        dt = time.perf_counter() - t0
+        if dt >= seconds:
+            break
+        batch = min(2 * batch, max(1, max_steps - n))
+    return {"steps": n, "s": round(time.perf_counter() - t0, 3)}
+
+
 def time_steps(fn, steps, stream, dist=None, flush=None):
     """Mean device time of one fn() over `steps` back-to-back calls.  With
     `flush` (a buffer larger than L2), each call is timed alone and the
@@ -618,7 +669,7 @@ def whole_job_tflops(flops_per_rank_step, world, ms_per_step):
     return flops_per_rank_step * world / (ms_per_step / 1e3) / 1e12
 
 
-def full_rank_baseline(wl, device, steps, warmup, seed=0, flush=None):
+def full_rank_baseline(wl, device, steps, warmup, seed=0, flush=None, settle=0.0):
     """Same-shape full-rank layers (fwd Y = X W^T, bwd dX = dY W, dW = dY^T X;
     forward only for an inference workload) with torch.matmul (cuBLAS);
     layers reading one input (q/k/v, gate/up) are fused into one GEMM with
@@ -663,10 +714,11 @@ def full_rank_baseline(wl, device, steps, warmup, seed=0, flush=None):
 
     for _ in range(warmup):
         step()
+    st = settle_steps(step, settle)
     ms = time_steps(step, steps, torch.cuda.current_stream(), flush=flush)
     del bufs
     return {"ms_per_step": round(ms, 4), "tflops": round(flops / (ms / 1e3) / 1e12, 1), "flops": flops,
-            "impl": "torch.matmul (cuBLAS) bf16"}
+            "impl": "torch.matmul (cuBLAS) bf16", "settle": st}
 
 
 def timed_block(wl, mode, args, device, stream, dist=None, seed=0, **block_kw):
@@ -678,6 +730,8 @@ def timed_block(wl, mode, args, device, stream, dist=None, seed=0, **block_kw):
 
     from paper_2502_10940_gb300 import cola
 
+    sampler = ClockSampler(torch.cuda.current_device())
+    sampler.open()
     blk = Block(wl, mode, device, seed=seed, **block_kw)
     # launches per step, counted by the library's trace
     with cola.Trace(512) as tr:
@@ -707,13 +761,13 @@ def timed_block(wl, mode, args, device, stream, dist=None, seed=0, **block_kw):
     # between steps
     ws_bytes = blk.working_set_bytes()
     flush = torch.empty(256 << 20, dtype=torch.uint8, device=device) if ws_bytes < L2_BYTES else None
-    sampler = ClockSampler(torch.cuda.current_device())
+    settle = settle_steps(step_fn, args.settle)
     sampler.start()
     ms = time_steps(step_fn, args.steps, stream, dist, flush=flush)
     clocks = sampler.stop()
     blk.check()
     return dict(blk=blk, graph=graph, step_fn=step_fn, use_graph=use_graph, ms=ms, clocks=clocks,
-                flush=flush, ws_bytes=ws_bytes)
+                flush=flush, ws_bytes=ws_bytes, settle=settle)
 
 
 def modes_ratio(wl, mode, blk, args, device, stream, seed=0):
@@ -804,7 +858,9 @@ def run_cola(args, wl):
             # every launch; their sum per step, beside the graph-timed step
             "trace_ms_per_step": round(trace_ms, 4),
             "kernels_how": "eager steps, CUDA events around each launch; shares are of trace_ms_per_step",
-            "gpu_launches": blk.launches_per_step * args.steps, "clocks": clocks}
+            "gpu_launches": blk.launches_per_step * args.steps, "clocks": clocks,
+            "settle": {**tb["settle"], "how": "untimed steps after the warm-up, device kept busy, "
+                                              "before the timed region and the clock samples"}}
 
     if not args.no_extras:
         # end to end: each step's activations (and, training, upstream
@@ -813,17 +869,18 @@ def run_cola(args, wl):
         def full_rows(t):   # the whole padded row-major buffer behind a view
             return torch.as_strided(t, (t.shape[0], t.stride(0)), (t.stride(0), 1))
 
-        outs = [full_rows(t) for t in blk.step_results()]
-        h_out = [torch.empty(t.shape, dtype=t.dtype, pin_memory=True) for t in outs]
-        # The inputs are double-buffered: step k+1's inputs are copied on a
-        # second stream while step k runs (it waits for them before it starts,
-        # and the copy into a buffer waits for the step that last read it).
-        # With graphs, one graph per buffer set.
-        blk.add_input_set()
-        sets_in = []
+        # The inputs and results are double-buffered: step k+1's inputs are
+        # copied in on one stream and step k-1's results copied out on another
+        # while step k runs.  A step waits for its inputs and for the copy-out
+        # of the results its buffer set last held; a copy into an input buffer
+        # waits for the step that last read it.  With graphs, one graph per
+        # buffer set.
+        blk.add_io_set()
+        sets_in, sets_out = [], []
         for i in range(2):
             blk.bind(i)
             sets_in.append([full_rows(t) for t in blk.step_inputs()])
+            sets_out.append([full_rows(t) for t in blk.step_results()])
         run_set = [blk.step, blk.step]
         if use_graph:
             g1 = torch.cuda.CUDAGraph()
@@ -833,9 +890,10 @@ def run_cola(args, wl):
             run_set = [graph.replay, g1.replay]
         blk.bind(0)
         h_in = [torch.empty(t.shape, dtype=t.dtype, pin_memory=True) for t in sets_in[0]]
+        h_out = [[torch.empty(t.shape, dtype=t.dtype, pin_memory=True) for t in sets_out[0]] for _ in range(2)]
         for h, t in zip(h_in, sets_in[0]):
             h.copy_(t)
-        copy_stream = torch.cuda.Stream()
+        copy_stream, out_stream = torch.cuda.Stream(), torch.cuda.Stream()
 
         def copy_in(dst):
             for h, t in zip(h_in, dst):
@@ -845,11 +903,13 @@ def run_cola(args, wl):
             e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
             ev_in = [torch.cuda.Event(), torch.cuda.Event()]
             ev_done = [torch.cuda.Event(), torch.cuda.Event()]
+            ev_out = [torch.cuda.Event(), torch.cuda.Event()]
             if dist:
                 dist.barrier()
             torch.cuda.synchronize()
             e0.record(stream)
             copy_stream.wait_event(e0)
+            out_stream.wait_event(e0)
             with torch.cuda.stream(copy_stream):
                 copy_in(sets_in[0])
             ev_in[0].record(copy_stream)
@@ -862,12 +922,18 @@ def run_cola(args, wl):
                         copy_in(sets_in[nxt])
                     ev_in[nxt].record(copy_stream)
                 stream.wait_event(ev_in[cur])
+                if k >= 2:
+                    stream.wait_event(ev_out[cur])
                 if not use_graph:
                     blk.bind(cur)
                 run_set[cur]()
                 ev_done[cur].record(stream)
-                for h, t in zip(h_out, outs):
-                    h.copy_(t, non_blocking=True)
+                out_stream.wait_event(ev_done[cur])
+                with torch.cuda.stream(out_stream):
+                    for h, t in zip(h_out[cur], sets_out[cur]):
+                        h.copy_(t, non_blocking=True)
+                ev_out[cur].record(out_stream)
+            stream.wait_stream(out_stream)
             e1.record(stream)
             torch.cuda.synchronize()
             if dist:
@@ -880,17 +946,19 @@ def run_cola(args, wl):
         blk.bind(0)
         blk.check()
         bi = sum(t.numel() * t.element_size() for t in sets_in[0])
-        bo = sum(t.numel() * t.element_size() for t in outs)
+        bo = sum(t.numel() * t.element_size() for t in sets_out[0])
         line["e2e"] = {"value": round(whole_job_tflops(flops, world, ms_e2e), 2), "unit": "TFLOP/s",
                        "ms_per_step": round(ms_e2e, 4), "steps": e2e_steps, "h2d_bytes_per_step": bi,
                        "d2h_bytes_per_step": bo,
                        "inputs": "double-buffered, next step's copies overlap this step",
+                       "results": "double-buffered, last step's copies overlap this step",
                        "results_to_host": blk.results_words()}
-        del h_in, h_out, sets_in, outs, run_set
+        del h_in, h_out, sets_in, sets_out, run_set
         if use_graph:
             del g1
         if rank == 0 and world == 1:
-            fr = full_rank_baseline(wl, device, max(3, args.steps // 2), 3, seed=args.seed, flush=flush)
+            fr = full_rank_baseline(wl, device, max(3, args.steps // 2), 3, seed=args.seed, flush=flush,
+                                    settle=args.settle)
             fr["speedup_cola_vs_full_rank"] = round(fr["ms_per_step"] / ms, 3)
             line["full_rank"] = fr
             mr = modes_ratio(wl, mode, blk, args, device, stream, seed=args.seed + rank)
@@ -909,6 +977,7 @@ def run_cola(args, wl):
                                        "unit": "TFLOP/s", "ms_per_step": round(t1["ms"], 4),
                                        "pct_dense_bf16_peak": round(100.0 * v1 / peaks["bf16_tflops"], 2),
                                        "cuda_graph": t1["use_graph"], "clocks": t1["clocks"],
+                                       "settle": t1["settle"],
                                        "modes": modes_ratio(w1, w1.modes[0], t1["blk"], args, device, stream,
                                                             seed=args.seed)}}
                 del t1
@@ -924,6 +993,7 @@ def run_cola(args, wl):
                                             "unit": "TFLOP/s", "ms_per_step": round(tg["ms"], 4),
                                             "pct_dense_bf16_peak": round(100.0 * vg / peaks["bf16_tflops"], 2),
                                             "cuda_graph": tg["use_graph"], "clocks": tg["clocks"],
+                                            "settle": tg["settle"],
                                             "unfused_ms_per_step": round(tu["ms"], 4),
                                             "unfused_how": "the library's GEMMs with the product and its "
                                                            "backward as torch element-wise ops between them"}
@@ -949,6 +1019,8 @@ def main(argv=None):
     ap.add_argument("--graph", default="on", choices=["on", "off"],
                     help="replay each step as one CUDA graph (off: launch every kernel from the host)")
     ap.add_argument("--seed", type=int, default=0)
+    ap.add_argument("--settle", type=float, default=SETTLE_S,
+                    help="seconds of untimed steps after the warm-up, before the timed region")
     ap.add_argument("--no-extras", action="store_true", help="skip e2e, full-rank and CPU baselines")
     ap.add_argument("--fused-forward", default="on", choices=["on", "off"],
                     help="single-layer forwards with r <= 128: one fused kernel (on) or two GEMMs (off)")
