@@ -288,6 +288,11 @@ def launch_cost(kind, shapes, splits, flags):
         (m, r, k1), (_, n_out, _) = shapes
         nzh = (1 if flags & 1 else 0) + (1 if flags & 64 else 0)
         return e * (m * k1 + r * k1 + m * r * nzh + n_out * r + m * n_out), 2.0 * m * r * (k1 + n_out)
+    if kind == "bwd_fused":
+        # dY, B, the saved Z and A read; dZ (and, flag 1, H) and dX written; dZ stays on chip in between
+        (m, r, k1), (_, n_out, _) = shapes
+        nzh = 2 + (1 if flags & 1 else 0)
+        return e * (m * k1 + k1 * r + m * r * nzh + r * n_out + m * n_out), 2.0 * m * r * (k1 + n_out)
     tb, tf = 0.0, 0.0
     for (m, n, k) in shapes:
         if kind in ("fwd_zh", "fwd_y") and flags & 2:

@@ -138,7 +138,15 @@ cola_status_t cola_fwd(const cola_desc_t* desc, const void* X, const void* A, co
  * Inputs X, A, B, dY [n x d_out] (ld_y), Z_save; H_save under COLA (must be
  * NULL under COLA_M, where H = sigma(Z_save) is recomputed into the
  * workspace).  Outputs dX (bf16), dA and dB (bf16, or fp32 accumulated when
- * desc->wgrad_fp32).  The result does not depend on the mode, bit for bit. */
+ * desc->wgrad_fp32).  The result does not depend on the mode, bit for bit.
+ * Launches: the dZ GEMM (sigma' fused in its epilogue), the weight-gradient
+ * GEMMs (and their token-split reduce), the dX GEMM.  For r = 64 or 128 when
+ * neither the dZ nor the dX GEMM is compute-heavy and n is at most 128
+ * tokens per SM, dZ and dX run as one kernel instead: each CTA keeps the dZ
+ * of its 128-row tile in shared memory between the two products (loading the
+ * tile's Z there and overwriting it with dZ), storing dZ (and, under COLA_M,
+ * H) to the workspace for the weight gradients; the results are the same
+ * bit for bit (cola_set_fused_backward). */
 cola_status_t cola_bwd(const cola_desc_t* desc, const void* X, const void* A, const void* B, const void* dY,
                        const void* Z_save, const void* H_save, void* dX, void* dA, void* dB, void* ws,
                        size_t ws_bytes, void* stream);
@@ -343,8 +351,10 @@ typedef enum {
     COLA_KERNEL_BWD_DX = 5,      /* dX = dZ A                             (M=n, N=d_in, K=r or 3r) */
     COLA_KERNEL_SIGMA = 6,       /* H = sigma(Z), elementwise             (M=n, N=count r, K=0) */
     COLA_KERNEL_FWD_GLU = 7,     /* M = (H_gate B_gate^T) * (H_up B_up^T) (M=n, N=d_ff, K=2r) */
-    COLA_KERNEL_FWD_FUSED = 8    /* Z, H = sigma(Z), Y = H B^T in one kernel, count 2:
+    COLA_KERNEL_FWD_FUSED = 8,   /* Z, H = sigma(Z), Y = H B^T in one kernel, count 2:
                                     (n, r, d_in) and (n, d_out, r) */
+    COLA_KERNEL_BWD_FUSED = 9    /* dZ = (dY B) * sigma'(Z), dX = dZ A in one kernel, count 2:
+                                    (n, r, d_out) and (n, d_in, r) */
 } cola_kernel_t;
 
 typedef struct {
@@ -364,7 +374,8 @@ typedef struct {
                                   tail tile; a reduce launch follows when they are > 1);
                            bit 5: the dX epilogue stored the gated-MLP gradients dY_gate,
                                   dY_up instead of dX (cola_bwd_down_gated);
-                           bit 6: the fused forward stored Z (bit 0: it stored H) */
+                           bit 6: the fused forward stored Z (bit 0: it stored H; in the
+                                  fused backward bit 0 means H recomputed under CoLA-M) */
 } cola_trace_slot_t;
 
 cola_status_t cola_trace_attach(cola_trace_slot_t* slots, int32_t capacity, int32_t* count);
@@ -375,6 +386,11 @@ cola_status_t cola_trace_detach(void);
  * for comparisons; both give the same results bit for bit.  enable outside
  * {0, 1}: COLA_ERR_INVALID.  Takes effect for calls made after it returns. */
 cola_status_t cola_set_fused_forward(int32_t enable);
+
+/* The same choice for cola_bwd's dZ and dX GEMMs (see cola_bwd): 1 (default)
+ * runs them as one kernel where that form applies, 0 as two GEMMs; both give
+ * the same results bit for bit.  enable outside {0, 1}: COLA_ERR_INVALID. */
+cola_status_t cola_set_fused_backward(int32_t enable);
 
 /* Static description of a status code. */
 const char* cola_status_string(cola_status_t status);

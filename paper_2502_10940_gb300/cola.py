@@ -25,9 +25,11 @@ STATUS = {0: "COLA_OK", 1: "COLA_ERR_INVALID", 2: "COLA_ERR_ALIGN", 3: "COLA_ERR
 SYMBOLS = ("cola_workspace_size", "cola_workspace_init", "cola_fwd", "cola_bwd", "cola_fwd_shared_x",
            "cola_bwd_shared_x", "cola_fwd_gate_up", "cola_bwd_down_gated", "cola_recompute_up", "cola_fwd_qkv_fused", "cola_bwd_qkv_fused", "cola_check_status",
            "cola_wgrad_static_scratch", "cola_selftest_wait_timeout", "cola_selftest_wait_timeout_pair",
-           "cola_trace_attach", "cola_trace_detach", "cola_set_fused_forward", "cola_status_string")
+           "cola_trace_attach", "cola_trace_detach", "cola_set_fused_forward", "cola_set_fused_backward",
+           "cola_status_string")
 STATIC_SCRATCH_BYTES = 64 * 1024 * 1024
-KERNELS = {0: "fwd_zh", 1: "fwd_y", 2: "bwd_dz", 3: "wgrad", 4: "reduce", 5: "bwd_dx", 6: "sigma", 7: "fwd_glu", 8: "fwd_fused"}
+KERNELS = {0: "fwd_zh", 1: "fwd_y", 2: "bwd_dz", 3: "wgrad", 4: "reduce", 5: "bwd_dx", 6: "sigma", 7: "fwd_glu", 8: "fwd_fused",
+           9: "bwd_fused"}
 
 
 class ColaError(RuntimeError):
@@ -102,6 +104,8 @@ def lib():
         l.cola_trace_detach.restype = st
         l.cola_set_fused_forward.argtypes = [ctypes.c_int32]
         l.cola_set_fused_forward.restype = st
+        l.cola_set_fused_backward.argtypes = [ctypes.c_int32]
+        l.cola_set_fused_backward.restype = st
         l.cola_status_string.argtypes = [ctypes.c_int]
         l.cola_status_string.restype = ctypes.c_char_p
         _lib = l
@@ -243,6 +247,12 @@ def cola_set_fused_forward(enable: bool):
     """cola_fwd's single-kernel forward where it applies (default on) or the
     two GEMMs (off), process-wide; the results are the same bit for bit."""
     _check(lib().cola_set_fused_forward(int(bool(enable))), "cola_set_fused_forward")
+
+
+def cola_set_fused_backward(enable: bool):
+    """cola_bwd's single-kernel dZ + dX where it applies (default on) or the
+    two GEMMs (off), process-wide; the results are the same bit for bit."""
+    _check(lib().cola_set_fused_backward(int(bool(enable))), "cola_set_fused_backward")
 
 
 def cola_status_string(status: int) -> str:

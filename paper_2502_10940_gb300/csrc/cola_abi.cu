@@ -12,7 +12,7 @@
 #include <mutex>
 
 #include "cola.h"
-#include "fused_fwd.cuh"
+#include "fused_layer.cuh"
 #include "gemm_launch.cuh"
 #include "host_plan.cuh"
 
@@ -356,12 +356,14 @@ cola_status_t run_f1(const Shape& s, int sigma, int64_t N, const void* X, const 
 
 }  // namespace
 
-cudaError_t launch_fused_fwd(const FusedFwdParams& p, int r, int grid, bool pdl, cudaStream_t stream);
+cudaError_t launch_fused_layer(const FusedParams& p, int r, bool bwd, int grid, bool pdl, cudaStream_t stream);
 
 namespace {
 
-// Whether cola_fwd runs a layer as one fused kernel (cola_set_fused_forward).
+// Whether cola_fwd / cola_bwd run a layer's two products as one fused kernel
+// where that form applies (cola_set_fused_forward / cola_set_fused_backward).
 std::atomic<int> g_fused_fwd{1};
+std::atomic<int> g_fused_bwd{1};
 
 // The single-kernel forward applies to one layer with r = 64 or 128 whose
 // two GEMMs are HBM-bound (neither is compute-heavy), with at most one
@@ -379,43 +381,96 @@ bool fused_fwd_applies(const Shape& s, int sms)
     return small_launch_splits(p2.m_tiles * p2.n_tiles, p2.k_blocks, sms) == 1;
 }
 
+// The single-kernel dZ + dX applies on the same terms: r = 64 or 128, at
+// most one 128-row tile per SM, neither GEMM compute-heavy (the backward's
+// GEMMs are never split over K).
+bool fused_bwd_applies(const Shape& s, int sms)
+{
+    if (!g_fused_bwd.load(std::memory_order_relaxed) || (s.r != 64 && s.r != 128)) return false;
+    if ((s.n + BM - 1) / BM > sms) return false;
+    return !heavy_gemm(s.n, s.r, s.d_out) && !heavy_gemm(s.n, s.d_in, s.r);
+}
+
+// Work items of a fused pass: the output blocks of a tile shared by up to
+// sms / m_tiles items, so that the launch fills the SMs.
+void fused_items(FusedParams& p, int sms)
+{
+    int groups = sms / (p.m_tiles > 0 ? p.m_tiles : 1);
+    groups = std::max(1, std::min(groups, p.n_blocks));
+    p.blocks_per_group = (p.n_blocks + groups - 1) / groups;
+    p.out_groups = (p.n_blocks + p.blocks_per_group - 1) / p.blocks_per_group;
+}
+
 // F1 + F2 in one kernel: Z = X A^T, H = sigma(Z) kept on chip, Y = H B^T;
 // Z and H stored when not null.
 cola_status_t run_fused_fwd(const Shape& s, int sigma, const void* X, const void* A, const void* B, void* Y, void* Z,
                             void* H, unsigned int* status, int sms, cudaStream_t st)
 {
-    FusedFwdParams p;
+    FusedParams p;
     std::memset(&p, 0, sizeof p);
-    COLA_MAP(map_kmajor(&p.map_x, X, s.d_in, s.n, s.ld_x, BM));
-    COLA_MAP(map_kmajor(&p.map_a, A, s.d_in, s.r, s.ld_a, static_cast<int>(s.r)));
-    COLA_MAP(map_kmajor(&p.map_b, B, s.r, s.d_out, s.r, FBN));
-    COLA_MAP(map_box32(&p.map_y, Y, s.d_out, s.n, s.ld_y));
-    p.map_z = p.map_h = p.map_y;
-    if (Z) COLA_MAP(map_box32(&p.map_z, Z, s.r, s.n, s.r));
-    if (H) COLA_MAP(map_box32(&p.map_h, H, s.r, s.n, s.r));
+    COLA_MAP(map_kmajor(&p.map_in, X, s.d_in, s.n, s.ld_x, BM));
+    COLA_MAP(map_kmajor(&p.map_w1, A, s.d_in, s.r, s.ld_a, static_cast<int>(s.r)));
+    COLA_MAP(map_kmajor(&p.map_w2, B, s.r, s.d_out, s.r, FBN));
+    COLA_MAP(map_box32(&p.map_out, Y, s.d_out, s.n, s.ld_y));
+    p.map_zin = p.map_s1 = p.map_s2 = p.map_out;
+    if (Z) COLA_MAP(map_box32(&p.map_s1, Z, s.r, s.n, s.r));
+    if (H) COLA_MAP(map_box32(&p.map_s2, H, s.r, s.n, s.r));
     p.n = static_cast<int>(s.n);
-    p.d_out = static_cast<int>(s.d_out);
+    p.n_out = static_cast<int>(s.d_out);
     p.kb1 = static_cast<int>((s.d_in + BK - 1) / BK);
     p.m_tiles = static_cast<int>((s.n + BM - 1) / BM);
     p.n_blocks = static_cast<int>((s.d_out + FBN - 1) / FBN);
-    // the Y blocks of a tile shared by up to sms / m_tiles work items
-    int groups = sms / (p.m_tiles > 0 ? p.m_tiles : 1);
-    groups = std::max(1, std::min(groups, p.n_blocks));
-    p.blocks_per_group = (p.n_blocks + groups - 1) / groups;
-    p.y_groups = (p.n_blocks + p.blocks_per_group - 1) / p.blocks_per_group;
-    p.store_z = Z != nullptr;
-    p.store_h = H != nullptr;
+    fused_items(p, sms);
+    p.store_s1 = Z != nullptr;
+    p.store_s2 = H != nullptr;
     p.sigma = sigma;
-    p.y_ptr = static_cast<__nv_bfloat16*>(Y);
-    p.y_ld = s.ld_y;
+    p.out_ptr = static_cast<__nv_bfloat16*>(Y);
+    p.out_ld = s.ld_y;
     p.status = status;
-    const int items = p.m_tiles * p.y_groups;
+    const int items = p.m_tiles * p.out_groups;
     const int grid = items < sms ? items : sms;
     const double flops = 2.0 * s.n * s.r * (s.d_in + s.d_out);
     const int64_t mnk[2][3] = {{s.n, s.r, s.d_in}, {s.n, s.d_out, s.r}};
     const int flags = (H ? 1 : 0) | (Z ? TRACE_Z : 0);
     return launched(traced(COLA_KERNEL_FWD_FUSED, 2, mnk, 1, flags, st,
-                           [&] { return launch_fused_fwd(p, static_cast<int>(s.r), grid, flops < 64e9, st); }));
+                           [&] { return launch_fused_layer(p, static_cast<int>(s.r), false, grid, flops < 64e9, st); }));
+}
+
+// B1 + B4 in one kernel: dZ = (dY B) * sigma'(Z) kept on chip (and stored
+// to dZ, pitch r), dX = dZ A; under CoLA-M H = sigma(Z) stored to Hrec
+// (pitch r) for the weight gradient of B.
+cola_status_t run_fused_bwd(const Shape& s, int sigma, const void* dY, const void* B, const void* Z, const void* A,
+                            void* dX, void* dZ, void* Hrec, unsigned int* status, int sms, cudaStream_t st)
+{
+    FusedParams p;
+    std::memset(&p, 0, sizeof p);
+    COLA_MAP(map_kmajor(&p.map_in, dY, s.d_out, s.n, s.ld_y, BM));
+    COLA_MAP(map_mnmajor(&p.map_w1, B, s.r, s.d_out, s.r));
+    COLA_MAP(map_mnmajor(&p.map_w2, A, s.d_in, s.r, s.ld_a));
+    COLA_MAP(map_kmajor(&p.map_zin, Z, s.r, s.n, s.r, BM));
+    COLA_MAP(map_box32(&p.map_s1, dZ, s.r, s.n, s.r));
+    p.map_s2 = p.map_s1;
+    if (Hrec) COLA_MAP(map_box32(&p.map_s2, Hrec, s.r, s.n, s.r));
+    COLA_MAP(map_box32(&p.map_out, dX, s.d_in, s.n, s.ld_x));
+    p.n = static_cast<int>(s.n);
+    p.n_out = static_cast<int>(s.d_in);
+    p.kb1 = static_cast<int>((s.d_out + BK - 1) / BK);
+    p.m_tiles = static_cast<int>((s.n + BM - 1) / BM);
+    p.n_blocks = static_cast<int>((s.d_in + FBN - 1) / FBN);
+    fused_items(p, sms);
+    p.store_s1 = 1;
+    p.store_s2 = Hrec != nullptr;
+    p.sigma = sigma;
+    p.out_ptr = static_cast<__nv_bfloat16*>(dX);
+    p.out_ld = s.ld_x;
+    p.status = status;
+    const int items = p.m_tiles * p.out_groups;
+    const int grid = items < sms ? items : sms;
+    const double flops = 2.0 * s.n * s.r * (s.d_out + s.d_in);
+    const int64_t mnk[2][3] = {{s.n, s.r, s.d_out}, {s.n, s.d_in, s.r}};
+    const int flags = Hrec ? 1 : 0;
+    return launched(traced(COLA_KERNEL_BWD_FUSED, 2, mnk, 1, flags, st,
+                           [&] { return launch_fused_layer(p, static_cast<int>(s.r), true, grid, flops < 64e9, st); }));
 }
 
 // F2: Y_j = H_j B_j^T for `count` projections of one shape (H_j [n x r] with
@@ -814,10 +869,15 @@ cola_status_t bwd_single(const cola_desc_t* desc, const void* X, const void* A, 
     const void* Zs[1] = {Z_save};
     void* dZs[1] = {dZ};
     void* Hs[1] = {Hrec};
-    COLA_TRY(run_b1(s, desc->sigma, 1, dYs, Bs, Zs, s.r, dZs, cola_m ? Hs : nullptr, status, sms, st));
     const void* Hsrc = cola_m ? Hrec : H_save;
     const WgradPlan w = wgrad_plan(*desc, 1, sms);
     const WgradJob jobs[2] = {{dY, s.ld_y, Hsrc, s.r, dB, s.r}, {dZ, s.r, X, s.ld_x, dA, s.ld_a}};
+    if (!glu && fused_bwd_applies(s, sms)) {
+        // dZ (and H) with dX in one kernel, then the weight gradients
+        COLA_TRY(run_fused_bwd(s, desc->sigma, dY, B, Z_save, A, dX, dZ, Hrec, status, sms, st));
+        return run_wgrad(w, s.n, jobs, desc->wgrad_fp32, part, part_bytes, status, sms, st);
+    }
+    COLA_TRY(run_b1(s, desc->sigma, 1, dYs, Bs, Zs, s.r, dZs, cola_m ? Hs : nullptr, status, sms, st));
     COLA_TRY(run_wgrad(w, s.n, jobs, desc->wgrad_fp32, part, part_bytes, status, sms, st));
     if (glu) return run_b4_glu(s, s.r, dZ, s.r, A, glu->Yg, glu->Yu, glu->dYg, glu->dYu, status, sms, st);
     return run_b4(s, s.r, dZ, s.r, A, dX, status, sms, st);
@@ -1061,6 +1121,13 @@ cola_status_t cola_set_fused_forward(int32_t enable)
 {
     if (enable != 0 && enable != 1) return COLA_ERR_INVALID;
     g_fused_fwd.store(enable, std::memory_order_relaxed);
+    return COLA_OK;
+}
+
+cola_status_t cola_set_fused_backward(int32_t enable)
+{
+    if (enable != 0 && enable != 1) return COLA_ERR_INVALID;
+    g_fused_bwd.store(enable, std::memory_order_relaxed);
     return COLA_OK;
 }
 

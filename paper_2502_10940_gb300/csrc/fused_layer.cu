@@ -1,18 +1,19 @@
-// The single-kernel forward of a CoLA layer with r <= 128 (fused_fwd.cuh):
-// its launcher, instantiated for r = 64 and r = 128.
+// The single-kernel forward and backward passes of a CoLA layer with
+// r <= 128 (fused_layer.cuh): their launcher, instantiated for r = 64 and
+// r = 128 in both directions.
 #include <cuda_runtime.h>
 
 #include <atomic>
 
-#include "fused_fwd.cuh"
+#include "fused_layer.cuh"
 
 namespace cola {
 
-template <int R>
-static cudaError_t launch_fused_fwd_r(const FusedFwdParams& p, int grid, bool pdl, cudaStream_t stream)
+template <int R, bool BWD>
+static cudaError_t launch_fused_layer_r(const FusedParams& p, int grid, bool pdl, cudaStream_t stream)
 {
     constexpr int smem = FusedCfg<R>::SMEM_BYTES;
-    auto kern = fused_fwd_kernel<R>;
+    auto kern = fused_layer_kernel<R, BWD>;
     static std::atomic<unsigned long long> configured{0};   // bit d: attribute set on device d
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
@@ -35,10 +36,12 @@ static cudaError_t launch_fused_fwd_r(const FusedFwdParams& p, int grid, bool pd
     return cudaLaunchKernelEx(&cfg, kern, p);
 }
 
-cudaError_t launch_fused_fwd(const FusedFwdParams& p, int r, int grid, bool pdl, cudaStream_t stream)
+cudaError_t launch_fused_layer(const FusedParams& p, int r, bool bwd, int grid, bool pdl, cudaStream_t stream)
 {
-    if (r == 64) return launch_fused_fwd_r<64>(p, grid, pdl, stream);
-    if (r == 128) return launch_fused_fwd_r<128>(p, grid, pdl, stream);
+    if (r == 64) return bwd ? launch_fused_layer_r<64, true>(p, grid, pdl, stream)
+                            : launch_fused_layer_r<64, false>(p, grid, pdl, stream);
+    if (r == 128) return bwd ? launch_fused_layer_r<128, true>(p, grid, pdl, stream)
+                             : launch_fused_layer_r<128, false>(p, grid, pdl, stream);
     return cudaErrorInvalidValue;
 }
 

@@ -203,8 +203,9 @@ def test_pair_selftest_argument_errors(L):
     assert f(FAKE, 4096, 2, None) == 4           # smaller than the status word plus the operands
 
 
-def test_set_fused_forward_argument_errors(L):
-    f = L.lib().cola_set_fused_forward
+@pytest.mark.parametrize("name", ["cola_set_fused_forward", "cola_set_fused_backward"])
+def test_set_fused_argument_errors(L, name):
+    f = getattr(L.lib(), name)
     assert f(2) == 1 and f(-1) == 1
     assert f(1) == 0                             # the default, restored
 
