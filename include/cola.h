@@ -375,7 +375,10 @@ typedef struct {
                            bit 5: the dX epilogue stored the gated-MLP gradients dY_gate,
                                   dY_up instead of dX (cola_bwd_down_gated);
                            bit 6: the fused forward stored Z (bit 0: it stored H; in the
-                                  fused backward bit 0 means H recomputed under CoLA-M) */
+                                  fused backward bit 0 means H recomputed under CoLA-M);
+                           bit 7: the GEMM's K range split `splits` ways inside thread-block
+                                  clusters of that size, the partial tiles reduced on chip and
+                                  the epilogue applied in the same launch (no reduce launch) */
 } cola_trace_slot_t;
 
 cola_status_t cola_trace_attach(cola_trace_slot_t* slots, int32_t capacity, int32_t* count);
@@ -391,6 +394,17 @@ cola_status_t cola_set_fused_forward(int32_t enable);
  * runs them as one kernel where that form applies, 0 as two GEMMs; both give
  * the same results bit for bit.  enable outside {0, 1}: COLA_ERR_INVALID. */
 cola_status_t cola_set_fused_backward(int32_t enable);
+
+/* Weight-gradient launches with few output tiles and a short token walk (a
+ * few thousand tokens) split their tokens to fill the SMs.  1 (default): the
+ * splits of a 128 x 128 gradient tile run as one thread-block cluster of up
+ * to 8 CTAs that adds the partial tiles on chip, in a fixed order, and
+ * stores (or accumulates) in the same launch; 0: the planned split with fp32
+ * partials in the workspace and a reduce launch.  The two add the same
+ * partials in the same order only when they split alike, so results may
+ * differ in the last bits between the settings (each is deterministic run
+ * to run).  enable outside {0, 1}: COLA_ERR_INVALID. */
+cola_status_t cola_set_cluster_splitk(int32_t enable);
 
 /* Static description of a status code. */
 const char* cola_status_string(cola_status_t status);

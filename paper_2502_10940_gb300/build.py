@@ -14,8 +14,8 @@ INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libcola.so")
 
-SOURCES = ["cola_abi.cu", "gemm_fwd.cu", "gemm_bwd.cu", "gemm_wgrad.cu", "gemm_glu.cu", "fused_layer.cu", "cola_noalloc.cu"]
-HEADERS = ["ptx.cuh", "gemm.cuh", "gemm_launch.cuh", "host_plan.cuh", "fused_layer.cuh"]
+SOURCES = ["cola_abi.cu", "gemm_fwd.cu", "gemm_bwd.cu", "gemm_wgrad.cu", "gemm_glu.cu", "fused_layer.cu", "gemm_cluster.cu", "cola_noalloc.cu"]
+HEADERS = ["ptx.cuh", "gemm.cuh", "gemm_launch.cuh", "host_plan.cuh", "fused_layer.cuh", "splitk_cluster.cuh"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

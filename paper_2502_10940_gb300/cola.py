@@ -26,6 +26,7 @@ SYMBOLS = ("cola_workspace_size", "cola_workspace_init", "cola_fwd", "cola_bwd",
            "cola_bwd_shared_x", "cola_fwd_gate_up", "cola_bwd_down_gated", "cola_recompute_up", "cola_fwd_qkv_fused", "cola_bwd_qkv_fused", "cola_check_status",
            "cola_wgrad_static_scratch", "cola_selftest_wait_timeout", "cola_selftest_wait_timeout_pair",
            "cola_trace_attach", "cola_trace_detach", "cola_set_fused_forward", "cola_set_fused_backward",
+           "cola_set_cluster_splitk",
            "cola_status_string")
 STATIC_SCRATCH_BYTES = 64 * 1024 * 1024
 KERNELS = {0: "fwd_zh", 1: "fwd_y", 2: "bwd_dz", 3: "wgrad", 4: "reduce", 5: "bwd_dx", 6: "sigma", 7: "fwd_glu", 8: "fwd_fused",
@@ -106,6 +107,8 @@ def lib():
         l.cola_set_fused_forward.restype = st
         l.cola_set_fused_backward.argtypes = [ctypes.c_int32]
         l.cola_set_fused_backward.restype = st
+        l.cola_set_cluster_splitk.argtypes = [ctypes.c_int32]
+        l.cola_set_cluster_splitk.restype = st
         l.cola_status_string.argtypes = [ctypes.c_int]
         l.cola_status_string.restype = ctypes.c_char_p
         _lib = l
@@ -253,6 +256,13 @@ def cola_set_fused_backward(enable: bool):
     """cola_bwd's single-kernel dZ + dX where it applies (default on) or the
     two GEMMs (off), process-wide; the results are the same bit for bit."""
     _check(lib().cola_set_fused_backward(int(bool(enable))), "cola_set_fused_backward")
+
+
+def cola_set_cluster_splitk(enable: bool):
+    """Weight gradients of few tiles split their tokens inside thread-block
+    clusters reduced on chip (default on), or into fp32 slabs with a reduce
+    launch (off), process-wide."""
+    _check(lib().cola_set_cluster_splitk(int(bool(enable))), "cola_set_cluster_splitk")
 
 
 def cola_status_string(status: int) -> str:

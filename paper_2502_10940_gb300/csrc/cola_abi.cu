@@ -296,6 +296,99 @@ cola_status_t run_batch(int kind, int bn, int msub, const GemmProblem* probs, co
 }
 
 // ------------------------------------------------------------ passes
+}  // namespace
+
+cudaError_t launch_splitk_cluster(const CredBatch& b, bool pdl, cudaStream_t stream);
+
+namespace {
+
+// Whether weight-gradient launches of few tiles split the tokens inside
+// thread-block clusters (cola_set_cluster_splitk); off: the planned split
+// with its reduce launch.
+std::atomic<int> g_cluster_splitk{1};
+
+// One gradient of a cluster-reduced launch: D [M x N] = sum over the tokens
+// of P[t, m] Q[t, n], both token-major (pitches ldp, ldq), D with pitch ldo.
+struct CredJob {
+    const void* P;
+    int64_t ldp;
+    const void* Q;
+    int64_t ldq;
+    int64_t M, N;
+    void* out;
+    int64_t ldo;
+};
+
+// `count` weight gradients over the same ntok tokens in one launch, each
+// 128 x 128 tile on a cluster of S CTAs that split its tokens and reduce the
+// partials on chip (splitk_cluster.cuh); bf16 store or fp32 accumulate.
+cola_status_t run_cluster_wgrad(int count, const CredJob* jobs, int64_t ntok, int S, bool accumulate_f32,
+                                unsigned int* status, cudaStream_t st)
+{
+    CredBatch b;
+    std::memset(&b, 0, sizeof b);
+    const int kb = static_cast<int>((ntok + BK - 1) / BK);
+    b.count = count;
+    b.S = S;
+    b.kps = (kb + S - 1) / S;
+    b.op = accumulate_f32 ? CRED_ACC : CRED_STORE;
+    b.status = status;
+    int64_t mnk[MAX_GROUP][3];
+    double flops = 0.0;
+    int tiles = 0;
+    for (int j = 0; j < count; ++j) {
+        const CredJob& J = jobs[j];
+        CredProblem& P = b.prob[j];
+        COLA_MAP(map_mnmajor(&P.map_a, J.P, J.M, ntok, J.ldp));
+        COLA_MAP(map_mnmajor(&P.map_b, J.Q, J.N, ntok, J.ldq));
+        P.M = static_cast<int>(J.M);
+        P.N = static_cast<int>(J.N);
+        P.k_blocks = kb;
+        P.m_tiles = static_cast<int>((J.M + BM - 1) / BM);
+        P.n_tiles = static_cast<int>((J.N + CBN - 1) / CBN);
+        P.tile_begin = tiles;
+        tiles += P.m_tiles * P.n_tiles;
+        P.out = J.out;
+        P.ldo = J.ldo;
+        mnk[j][0] = J.M;
+        mnk[j][1] = J.N;
+        mnk[j][2] = ntok;
+        flops += 2.0 * J.M * J.N * ntok;
+    }
+    b.tiles = tiles;
+    return launched(traced(COLA_KERNEL_WGRAD, count, mnk, S, TRACE_CLUSTER, st,
+                           [&] { return launch_splitk_cluster(b, flops < 64e9, st); }));
+}
+
+// A reduce launch after a split weight-gradient launch, in k-block steps of
+// the busiest CTA (a few microseconds), for the comparison below.
+constexpr double REDUCE_LAUNCH_KB = 16.0;
+
+// The cluster split of a weight-gradient group (128 x 128 tiles, at most 8
+// splits, one wave of clusters): > 1 when it applies -- each CTA walks at
+// most CLUSTER_MAX_KPS k-blocks -- and its k-blocks per CTA undercut the
+// planned schedule with its reduce launch.  Its 4-stage, one-tile-per-CTA
+// form is made for short token walks: at 65536 tokens (the LLaMA-60M block,
+// 128-171 k-blocks per CTA) it ran the weight gradients 60 -> 93 us.
+constexpr int CLUSTER_MAX_KPS = 16;
+
+int wgrad_cluster_splits(const WgradPlan& w, int64_t ntok, int accumulate_f32, int sms)
+{
+    if (!g_cluster_splitk.load(std::memory_order_relaxed)) return 1;
+    int tiles = 0;
+    for (int j = 0; j < w.count; ++j)
+        tiles += static_cast<int>(((w.p[j].M + BM - 1) / BM) * ((w.p[j].N + CBN - 1) / CBN));
+    const int kb = static_cast<int>((ntok + BK - 1) / BK);
+    const int S = cluster_splits(tiles, kb, sms);
+    if (S < 2 || (kb + S - 1) / S > CLUSTER_MAX_KPS) return 1;
+    double planned = w.cost + REDUCE_LAUNCH_KB;
+    if (!accumulate_f32) {
+        const TailPlan tp = wgrad_tail_plan(w, ntok, sms);
+        if (tail_wins(w, tp)) planned = tp.cost + (tp.pieces > 1 ? REDUCE_LAUNCH_KB : 0.0);
+    }
+    return (kb + S - 1) / S <= planned ? S : 1;
+}
+
 // F1: Z = X A^T, H = sigma(Z)  (N = r, or 3r for the fused q/k/v factors;
 // Z / H pitch ldz)
 cola_status_t run_f1(const Shape& s, int sigma, int64_t N, const void* X, const void* A, void* Z, void* H,
@@ -595,6 +688,18 @@ cola_status_t run_wgrad_tail(const WgradPlan& w, int64_t ntok, const WgradJob* j
 cola_status_t run_wgrad(const WgradPlan& w, int64_t ntok, const WgradJob* jobs, int accumulate_f32, float* part,
                         size_t part_bytes, unsigned int* status, int sms, cudaStream_t st)
 {
+    {
+        // a small launch: the token splits reduced inside clusters, when one
+        // wave of clusters costs less than the planned schedule with its
+        // reduce launch (counted as REDUCE_LAUNCH_KB k-block steps)
+        const int Sc = wgrad_cluster_splits(w, ntok, accumulate_f32, sms);
+        if (Sc > 1) {
+            CredJob J[MAX_GROUP];
+            for (int j = 0; j < w.count; ++j)
+                J[j] = CredJob{jobs[j].P, jobs[j].ldp, jobs[j].Q, jobs[j].ldq, w.p[j].M, w.p[j].N, jobs[j].out, jobs[j].ldo};
+            return run_cluster_wgrad(w.count, J, ntok, Sc, accumulate_f32 != 0, status, st);
+        }
+    }
     if (!accumulate_f32 && tail_wins(w, wgrad_tail_plan(w, ntok, sms)))
         return run_wgrad_tail(w, ntok, jobs, part, part_bytes, status, sms, st);
     if (static_cast<size_t>(w.part_elems) * 4 > part_bytes) return COLA_ERR_WORKSPACE;
@@ -1128,6 +1233,13 @@ cola_status_t cola_set_fused_backward(int32_t enable)
 {
     if (enable != 0 && enable != 1) return COLA_ERR_INVALID;
     g_fused_bwd.store(enable, std::memory_order_relaxed);
+    return COLA_OK;
+}
+
+cola_status_t cola_set_cluster_splitk(int32_t enable)
+{
+    if (enable != 0 && enable != 1) return COLA_ERR_INVALID;
+    g_cluster_splitk.store(enable, std::memory_order_relaxed);
     return COLA_OK;
 }
 

@@ -10,6 +10,7 @@
 #include <mutex>
 
 #include "gemm_launch.cuh"
+#include "splitk_cluster.cuh"
 
 namespace cola {
 namespace {
@@ -188,6 +189,19 @@ int small_launch_splits(int tiles, int k_blocks, int sms)
     return s < k_blocks / 4 ? s : k_blocks / 4;
 }
 
+// K splits of a small launch reduced inside thread-block clusters
+// (splitk_cluster.cuh, 128 x 128 tiles): with fewer tiles than half the SMs,
+// the largest S <= 8 that keeps tiles * S within the SMs and >= 4 k-blocks
+// per split.  1 = no split.
+int cluster_splits(int tiles, int k_blocks, int sms)
+{
+    if (tiles < 1 || 2 * tiles >= sms) return 1;
+    int s = sms / tiles;
+    if (s > MAX_CLUSTER) s = MAX_CLUSTER;
+    if (s > k_blocks / 4) s = k_blocks / 4;
+    return s < 1 ? 1 : s;
+}
+
 int64_t partial_elems(const GemmParams& p, int bn, int msub)
 {
     return static_cast<int64_t>(p.m_tiles) * tile_rows(msub) * p.n_tiles * bn;
@@ -330,6 +344,7 @@ constexpr int TRACE_MSUB2 = 8;
 constexpr int TRACE_TAIL = 16;   // weight gradients with a split tail
 constexpr int TRACE_GLU = 32;    // the dX epilogue stored the gated-MLP gradients dY_gate, dY_up
 constexpr int TRACE_Z = 64;      // the fused forward stored Z
+constexpr int TRACE_CLUSTER = 128;   // K splits reduced inside thread-block clusters (no reduce launch)
 
 template <bool A_MN, int EPI>
 int tile_flags(int bn, int msub)

@@ -203,7 +203,7 @@ def test_pair_selftest_argument_errors(L):
     assert f(FAKE, 4096, 2, None) == 4           # smaller than the status word plus the operands
 
 
-@pytest.mark.parametrize("name", ["cola_set_fused_forward", "cola_set_fused_backward"])
+@pytest.mark.parametrize("name", ["cola_set_fused_forward", "cola_set_fused_backward", "cola_set_cluster_splitk"])
 def test_set_fused_argument_errors(L, name):
     f = getattr(L.lib(), name)
     assert f(2) == 1 and f(-1) == 1
