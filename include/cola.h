@@ -292,6 +292,19 @@ cola_status_t cola_selftest_wait_timeout(void* ws, size_t ws_bytes, void* stream
  * variant outside {1, 2}: COLA_ERR_INVALID. */
 cola_status_t cola_selftest_wait_timeout_pair(void* ws, size_t ws_bytes, int32_t variant, void* stream);
 
+/* The same self-test on a cluster-reduced weight gradient (cola_set_cluster_splitk):
+ * one 128 x 128 gradient tile over 512 tokens split over a cluster of two
+ * CTAs, operands in ws after its status header (ws_bytes >= 256 + 256 KB).
+ * CTA 1 issues no loads: its MMA issuer gives up after 2 s, and it still
+ * sends its (zero) partial band so that CTA 0 completes; CTA 0 then stores its
+ * band (64 rows of bf16) over the start of the first operand, CTA 1 stores
+ * nothing.  The next cola_check_status on ws returns COLA_ERR_DEVICE_TIMEOUT
+ * with some of COLA_STATUS_PRODUCER_TIMEOUT, COLA_STATUS_MMA_TIMEOUT and
+ * COLA_STATUS_EPILOGUE_TIMEOUT set and not COLA_STATUS_DRAIN_TIMEOUT (the
+ * exchange between the two CTAs completed), and the CUDA context stays
+ * usable.  Async on `stream`. */
+cola_status_t cola_selftest_wait_timeout_cluster(void* ws, size_t ws_bytes, void* stream);
+
 /* ---- weight gradient without any workspace or allocation ----
  * The paper has no counterpart to this entry point.  It serves callers that
  * cannot allocate device memory: an operator or plugin interface that hands

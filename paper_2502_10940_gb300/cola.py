@@ -25,6 +25,7 @@ STATUS = {0: "COLA_OK", 1: "COLA_ERR_INVALID", 2: "COLA_ERR_ALIGN", 3: "COLA_ERR
 SYMBOLS = ("cola_workspace_size", "cola_workspace_init", "cola_fwd", "cola_bwd", "cola_fwd_shared_x",
            "cola_bwd_shared_x", "cola_fwd_gate_up", "cola_bwd_down_gated", "cola_recompute_up", "cola_fwd_qkv_fused", "cola_bwd_qkv_fused", "cola_check_status",
            "cola_wgrad_static_scratch", "cola_selftest_wait_timeout", "cola_selftest_wait_timeout_pair",
+           "cola_selftest_wait_timeout_cluster",
            "cola_trace_attach", "cola_trace_detach", "cola_set_fused_forward", "cola_set_fused_backward",
            "cola_set_cluster_splitk",
            "cola_status_string")
@@ -93,6 +94,8 @@ def lib():
         l.cola_selftest_wait_timeout.restype = st
         l.cola_selftest_wait_timeout_pair.argtypes = [_vp, ctypes.c_size_t, ctypes.c_int32, _vp]
         l.cola_selftest_wait_timeout_pair.restype = st
+        l.cola_selftest_wait_timeout_cluster.argtypes = [_vp, ctypes.c_size_t, _vp]
+        l.cola_selftest_wait_timeout_cluster.restype = st
         l.cola_check_status.argtypes = [_vp, _vp, ctypes.POINTER(ctypes.c_uint32)]
         l.cola_check_status.restype = st
         i64 = ctypes.c_int64
@@ -223,6 +226,11 @@ def cola_selftest_wait_timeout(ws, stream=None):
 def cola_selftest_wait_timeout_pair(ws, variant, stream=None):
     _check(lib().cola_selftest_wait_timeout_pair(_ptr(ws), _nbytes(ws), int(variant), _stream(stream)),
            "cola_selftest_wait_timeout_pair")
+
+
+def cola_selftest_wait_timeout_cluster(ws, stream=None):
+    _check(lib().cola_selftest_wait_timeout_cluster(_ptr(ws), _nbytes(ws), _stream(stream)),
+           "cola_selftest_wait_timeout_cluster")
 
 
 def cola_fwd_qkv_fused(d, X, A_qkv, B_q, B_k, B_v, Y_q, Y_k, Y_v, Z_qkv, H_qkv, ws, stream=None):

@@ -1207,6 +1207,39 @@ cola_status_t cola_selftest_wait_timeout_pair(void* ws, size_t ws_bytes, int32_t
                                               static_cast<cudaStream_t>(stream));
 }
 
+cola_status_t cola_selftest_wait_timeout_cluster(void* ws, size_t ws_bytes, void* stream)
+{
+    if (!ws) return COLA_ERR_INVALID;
+    if (reinterpret_cast<uintptr_t>(ws) & (WS_ALIGN - 1)) return COLA_ERR_ALIGN;
+    constexpr int64_t M = 128, N = 128, T = 512;   // one 128 x 128 gradient tile over 512 tokens
+    constexpr size_t p_bytes = T * M * 2, q_bytes = T * N * 2;
+    if (ws_bytes < WS_HEADER + p_bytes + q_bytes) return COLA_ERR_WORKSPACE;
+    uint8_t* base = wsb(ws) + WS_HEADER;
+    CredBatch b;
+    std::memset(&b, 0, sizeof b);
+    b.count = 1;
+    b.tiles = 1;
+    b.S = 2;
+    b.kps = 4;
+    b.op = CRED_STORE;
+    b.status = ws_status(ws);
+    b.selftest = 1;
+    CredProblem& P = b.prob[0];
+    COLA_MAP(map_mnmajor(&P.map_a, base, M, T, M));
+    COLA_MAP(map_mnmajor(&P.map_b, base + p_bytes, N, T, N));
+    P.M = static_cast<int>(M);
+    P.N = static_cast<int>(N);
+    P.k_blocks = static_cast<int>(T / BK);
+    P.m_tiles = P.n_tiles = 1;
+    // the owner that completes normally stores its band over the operand P
+    // (already read by then); the CTA that gave up stores nothing
+    P.out = base;
+    P.ldo = N;
+    const int64_t mnk[1][3] = {{M, N, T}};
+    return launched(traced(COLA_KERNEL_WGRAD, 1, mnk, 2, TRACE_CLUSTER, static_cast<cudaStream_t>(stream),
+                           [&] { return launch_splitk_cluster(b, false, static_cast<cudaStream_t>(stream)); }));
+}
+
 cola_status_t cola_check_status(void* ws, void* stream, uint32_t* code_out)
 {
     if (!ws) return COLA_ERR_INVALID;

@@ -41,7 +41,10 @@
 // (an arrive on its `done` barrier), and a CTA exits only once all S have.
 // All waits are bounded, as in gemm.cuh; a CTA whose own wait ran out still
 // sends its bands (zeros where its accumulator is unusable), so that no other
-// CTA of the cluster waits for rows that never come.
+// CTA of the cluster waits for rows that never come, and the exchange's own
+// waits outlast the main loop's (4 s for the bands, 6 s for the exit signal,
+// against 2 s), so that the bands of a CTA that gave up still land before
+// anyone exits.
 //
 // Warp roles as in gemm.cuh (320 threads, one CTA per SM): warp 0 TMA
 // producer, warp 1 MMA issuer (allocates TMEM), warps 2..9 the exchange and
@@ -68,6 +71,26 @@ __device__ __forceinline__ void bulk_copy_to_cluster(uint32_t dst, uint32_t src,
 __device__ __forceinline__ void mbar_arrive_cluster_relaxed(uint32_t cluster_addr)
 {
     asm volatile("mbarrier.arrive.relaxed.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
+}
+
+// A wait of the exchange between the CTAs of a cluster.  It does not return
+// early on this CTA's abort flag, since copies of other CTAs may still be on
+// their way into this CTA's shared memory; its bound (`limit` ns) exceeds
+// the bounds of every earlier phase of the other CTAs, so that a CTA that
+// gave up on its own main loop (after WAIT_LIMIT_NS) still delivers its
+// bands and signals before its peers stop waiting for them.  On expiry it
+// records ST_TIMEOUT_DRAIN and returns false.
+__device__ __forceinline__ bool exchange_wait(uint64_t* bar, uint64_t limit, unsigned int* status)
+{
+    if (mbar_try_wait_cluster(bar, 0)) return true;
+    const uint64_t t0 = global_timer_ns();
+    while (!mbar_try_wait_cluster(bar, 0)) {
+        if (global_timer_ns() - t0 > limit) {
+            if (status) atomicOr(status, ST_TIMEOUT_DRAIN);
+            return false;
+        }
+    }
+    return true;
 }
 
 // Named barrier of the eight exchange warps.
@@ -98,6 +121,10 @@ struct CredBatch {
     int kps;    // k-blocks per split (the last split may have fewer, or none)
     int op;     // CredOp
     unsigned int* status;
+    // failure-detection self-test: 1 = CTA rank 1 of the first cluster issues
+    // no loads, so its MMA issuer's first wait runs out while the other CTAs
+    // of the cluster complete normally
+    int selftest;
 };
 
 struct CredCfg {
@@ -192,7 +219,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) splitk_cluster_kernel(const __
             long long issued = 0;
             bool ok = true;
             const int m0 = m_blk * BM, n0 = n_blk * CBN;
-            for (int kb = kb0; kb < kb1; ++kb) {
+            const bool no_loads = b.selftest == 1 && tile == 0 && rank == 1;
+            for (int kb = kb0; kb < kb1 && !no_loads; ++kb) {
                 if (!wait_bounded(&empty_bar[stage], phase ^ 1u, wc, ST_TIMEOUT_PRODUCER)) {
                     ok = false;
                     break;
@@ -297,7 +325,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) splitk_cluster_kernel(const __
         // stage this row's partial in the ring: row-major fp32, 16-byte chunk j
         // of the row at (j xor (row mod 8))
         const uint32_t stg = smem_u32(smem) + static_cast<uint32_t>(row * CBN * 4);
-        const bool use_acc = __all_sync(0xffffffffu, acc_ok && has_k);   // tcgen05.ld is warp-wide
+        // an accumulator this CTA gave up on sends zeros (tcgen05.ld is warp-wide)
+        const bool use_acc = __all_sync(0xffffffffu, acc_ok && has_k && !*abort_flag);
 #pragma unroll
         for (int i = 0; i < CBN / 64; ++i) {
             const int c = half + 2 * i;
@@ -326,7 +355,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) splitk_cluster_kernel(const __
                                  mapa_shared(smem_u32(data), static_cast<uint32_t>(tid)));
         }
         // this CTA's band from every CTA, summed in CTA order
-        const bool dok = wait_bounded<true>(data, 0, wc, ST_TIMEOUT_EPILOGUE);
+        const bool dok = exchange_wait(data, 2 * WAIT_LIMIT_NS, status);
         // every copy into this CTA has landed: tell each sender that its band
         // here has been read
         if (tid < S) mbar_arrive_cluster_relaxed(mapa_shared(smem_u32(done), static_cast<uint32_t>(tid)));
@@ -372,7 +401,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) splitk_cluster_kernel(const __
         }
         // the bands this CTA sent have been read by their owners: its staging
         // may go away with it
-        if (threadIdx.x == 64) wait_bounded<true>(done, 0, wc, ST_TIMEOUT_DRAIN);
+        if (threadIdx.x == 64) exchange_wait(done, 3 * WAIT_LIMIT_NS, status);
     }
 
     tc_fence_before();

@@ -203,6 +203,13 @@ def test_pair_selftest_argument_errors(L):
     assert f(FAKE, 4096, 2, None) == 4           # smaller than the status word plus the operands
 
 
+def test_cluster_selftest_argument_errors(L):
+    f = L.lib().cola_selftest_wait_timeout_cluster
+    assert f(None, 1 << 20, None) == 1
+    assert f(FAKE + 16, 1 << 20, None) == 2      # not 256-byte aligned
+    assert f(FAKE, 4096, None) == 4              # smaller than the status word plus the operands
+
+
 @pytest.mark.parametrize("name", ["cola_set_fused_forward", "cola_set_fused_backward", "cola_set_cluster_splitk"])
 def test_set_fused_argument_errors(L, name):
     f = getattr(L.lib(), name)

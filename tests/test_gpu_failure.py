@@ -5,7 +5,10 @@ COLA_ERR_DEVICE_TIMEOUT, and the context keeps working.  The same on a CTA
 pair, where the odd CTA's loads complete on the even CTA's barriers: with no
 loads at all, and with the odd CTA stopping after one k-block while the even
 CTA's loads of later stages land, in which case the pair's abort drain must
-see every load of both CTAs land (no drain-timeout bit) before it exits."""
+see every load of both CTAs land (no drain-timeout bit) before it exits.  And
+on a cluster-reduced weight gradient, where one CTA of the cluster gives up on
+its main loop: it still sends its (zero) partial band, the other CTA
+completes, and the exchange between them ends without a drain timeout."""
 import time
 
 import pytest
@@ -17,6 +20,7 @@ pytestmark = pytest.mark.gpu
 
 PRODUCER, MMA, EPILOGUE, DRAIN = 0x1, 0x2, 0x4, 0x8
 PAIR = 4   # launch-trace flag: the GEMM ran on CTA pairs
+CLUSTER = 128   # launch-trace flag: the token splits were reduced inside a cluster
 
 
 @pytest.fixture(scope="module", autouse=True)
@@ -111,3 +115,30 @@ def test_pair_selftest_argument_errors():
     assert lib.cola_selftest_wait_timeout_pair(None, 1 << 20, 1, None) == 1
     assert lib.cola_selftest_wait_timeout_pair(ws.data_ptr(), ws.numel(), 3, None) == 1    # no such variant
     assert lib.cola_selftest_wait_timeout_pair(ws.data_ptr(), 4096, 1, None) == 4          # too small
+
+
+def test_cluster_wait_runs_out_and_exchange_completes():
+    from paper_2502_10940_gb300 import cola
+    ws = torch.zeros(1 << 20, dtype=torch.uint8, device="cuda")
+    cola.cola_workspace_init(ws)
+    assert cola.cola_check_status(ws)[0] == 0
+    t0 = time.perf_counter()
+    with cola.Trace(4) as tr:
+        cola.cola_selftest_wait_timeout_cluster(ws)
+    st, code = cola.cola_check_status(ws)
+    dt = time.perf_counter() - t0
+    recs = tr.records()
+    assert len(recs) == 1 and recs[0][3] & CLUSTER and recs[0][2] == 2, recs
+    assert st == 6  # COLA_ERR_DEVICE_TIMEOUT
+    assert code & (PRODUCER | MMA | EPILOGUE), hex(code)
+    assert not code & ~(PRODUCER | MMA | EPILOGUE), hex(code)   # the exchange completed: no drain timeout
+    assert 1.5 < dt < 30.0
+    assert cola.cola_check_status(ws)[0] == 0
+    # the context still runs cluster-reduced weight gradients correctly
+    inp = make_inputs(2048, 512, 512, 128, seed=23)
+    with cola.Trace(16) as tr:
+        g = gpu_layer(inp, "silu", "cola")
+    assert any(rec[0] == "wgrad" and rec[3] & CLUSTER for rec in tr.records()), tr.records()
+    o = oracle_layer(inp, "silu", "cola")
+    for k in ["Y", "dX", "dA", "dB"]:
+        assert_close(k, to64(g[k]), o[k])
