@@ -435,25 +435,30 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) fused_layer_kernel(const __gri
                         z[4 * j + 3] = t.w;
                     }
                     tmem_ld_wait();
-                    // dZ = bf16(acc * sigma'(Z)), as the B1 epilogue of the two-GEMM backward
+                    // dZ = bf16(acc * sigma'(Z)), as the B1 epilogue of the two-GEMM backward;
+                    // under CoLA-M also H = sigma(Z), from the same logistic
+                    uint32_t h[16];
+                    const bool want_h = P.store_s2 && first;
                     with_sigma(P.sigma, [&](auto tag) {
                         constexpr int S = decltype(tag)::value;
+                        if (want_h) {
 #pragma unroll
-                        for (int j = 0; j < 16; ++j)
-                            w[j] = pack_bf16x2(__uint_as_float(v[2 * j]) * act_dsigma<S>(bf16_lo(z[j])),
-                                               __uint_as_float(v[2 * j + 1]) * act_dsigma<S>(bf16_hi(z[j])));
-                    });
-                    if (P.store_s1 && first) emit(&P.map_s1, w, c * 32, row0);
-                    if (P.store_s2 && first) {   // CoLA-M: H = sigma(Z) for the weight gradient of B
-                        uint32_t h[16];
-                        with_sigma(P.sigma, [&](auto tag) {
-                            constexpr int S = decltype(tag)::value;
+                            for (int j = 0; j < 16; ++j) {
+                                float hl, dl, hh, dh;
+                                act_both<S>(bf16_lo(z[j]), hl, dl);
+                                act_both<S>(bf16_hi(z[j]), hh, dh);
+                                w[j] = pack_bf16x2(__uint_as_float(v[2 * j]) * dl, __uint_as_float(v[2 * j + 1]) * dh);
+                                h[j] = pack_bf16x2(hl, hh);
+                            }
+                        } else {
 #pragma unroll
                             for (int j = 0; j < 16; ++j)
-                                h[j] = pack_bf16x2(act_sigma<S>(bf16_lo(z[j])), act_sigma<S>(bf16_hi(z[j])));
-                        });
-                        emit(&P.map_s2, h, c * 32, row0);
-                    }
+                                w[j] = pack_bf16x2(__uint_as_float(v[2 * j]) * act_dsigma<S>(bf16_lo(z[j])),
+                                                   __uint_as_float(v[2 * j + 1]) * act_dsigma<S>(bf16_hi(z[j])));
+                        }
+                    });
+                    if (P.store_s1 && first) emit(&P.map_s1, w, c * 32, row0);
+                    if (want_h) emit(&P.map_s2, h, c * 32, row0);   // for the weight gradient of B
                 } else {
                     tmem_ld_wait();
 #pragma unroll

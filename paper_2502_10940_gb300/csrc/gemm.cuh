@@ -205,6 +205,26 @@ __device__ __forceinline__ float act_dsigma(float z)
     return 1.0f;
 }
 
+// sigma(z) and sigma'(z) together, sharing the logistic (SiLU) or the normal
+// CDF and density (GELU): the same values as act_sigma and act_dsigma.
+template <int SIG>
+__device__ __forceinline__ void act_both(float z, float& h, float& d)
+{
+    if (SIG == SIG_SILU) {
+        const float s = logistic_fast(z);
+        h = z * s;
+        d = s * (1.0f + z * (1.0f - s));
+    } else if (SIG == SIG_GELU) {
+        const float Phi = 0.5f * erfcf(-z * 0.70710678118654752f);
+        const float phi = 0.39894228040143268f * __expf(-0.5f * z * z);
+        h = 0.5f * z * erfcf(-z * 0.70710678118654752f);
+        d = Phi + z * phi;
+    } else {
+        h = z;
+        d = 1.0f;
+    }
+}
+
 template <int SIG>
 struct SigTag {
     static constexpr int value = SIG;
@@ -1102,26 +1122,32 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                         z[4 * j + 2] = t.z;
                         z[4 * j + 3] = t.w;
                     }
+                    uint32_t hw[16];   // CoLA-M: H = sigma(Z), formed with sigma'(Z)
                     with_sigma(p.sigma, [&](auto tag) {
                         constexpr int S = decltype(tag)::value;
+                        if (p.has_d2) {
 #pragma unroll
-                        for (int j = 0; j < 16; ++j)
-                            w[j] = pack_bf16x2(__uint_as_float(v[2 * j]) * act_dsigma<S>(bf16_lo(z[j])),
-                                               __uint_as_float(v[2 * j + 1]) * act_dsigma<S>(bf16_hi(z[j])));
+                            for (int j = 0; j < 16; ++j) {
+                                float hl, dl, hh, dh;
+                                act_both<S>(bf16_lo(z[j]), hl, dl);
+                                act_both<S>(bf16_hi(z[j]), hh, dh);
+                                w[j] = pack_bf16x2(__uint_as_float(v[2 * j]) * dl, __uint_as_float(v[2 * j + 1]) * dh);
+                                hw[j] = pack_bf16x2(hl, hh);
+                            }
+                        } else {
+#pragma unroll
+                            for (int j = 0; j < 16; ++j)
+                                w[j] = pack_bf16x2(__uint_as_float(v[2 * j]) * act_dsigma<S>(bf16_lo(z[j])),
+                                                   __uint_as_float(v[2 * j + 1]) * act_dsigma<S>(bf16_hi(z[j])));
+                        }
                     });
                     stage_row(box, lane, w);        // dZ in place of this row's Z
                     fence_proxy_async_smem();
                     store_box(map_d, box, col0, row0);
-                    if (p.has_d2) {                 // CoLA-M: H = sigma(Z) through the same box
-                        with_sigma(p.sigma, [&](auto tag) {
-                            constexpr int S = decltype(tag)::value;
-#pragma unroll
-                            for (int j = 0; j < 16; ++j)
-                                w[j] = pack_bf16x2(act_sigma<S>(bf16_lo(z[j])), act_sigma<S>(bf16_hi(z[j])));
-                        });
+                    if (p.has_d2) {                 // CoLA-M: H through the same box
                         if (lane == 0) bulk_wait_group_read<0>();
                         __syncwarp();
-                        stage_row(box, lane, w);
+                        stage_row(box, lane, hw);
                         fence_proxy_async_smem();
                         store_box(map_d2, box, col0, row0);
                     }
