@@ -217,7 +217,7 @@ __device__ __forceinline__ void act_both(float z, float& h, float& d)
     } else if (SIG == SIG_GELU) {
         const float Phi = 0.5f * erfcf(-z * 0.70710678118654752f);
         const float phi = 0.39894228040143268f * __expf(-0.5f * z * z);
-        h = 0.5f * z * erfcf(-z * 0.70710678118654752f);
+        h = z * Phi;   // = (0.5 z) erfc(...) of act_sigma: scaling by 0.5 is exact
         d = Phi + z * phi;
     } else {
         h = z;
