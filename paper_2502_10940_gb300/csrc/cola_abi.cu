@@ -663,7 +663,8 @@ cola_status_t run_b1(const Shape& s, int sigma, int count, const void* const* dY
         mnk[j][1] = s.r;
         mnk[j][2] = s.d_out;
     }
-    return run_batch<false, true, EPI_DSIGMA>(COLA_KERNEL_BWD_DZ, bn, ms, pr, mnk, count, Hout != nullptr, sms, st);
+    if (Hout) return run_batch<false, true, EPI_DSIGMA_H>(COLA_KERNEL_BWD_DZ, bn, ms, pr, mnk, count, 1, sms, st);
+    return run_batch<false, true, EPI_DSIGMA>(COLA_KERNEL_BWD_DZ, bn, ms, pr, mnk, count, 0, sms, st);
 }
 
 // Weight gradients of one backward call, in one launch: D_j[M_j x N_j] =

@@ -34,7 +34,7 @@
 // intermediate makes no extra HBM round trip):
 //   EPI_STORE   D = bf16(acc)                                  (Y, dX)
 //   EPI_ZH      Z = bf16(acc), H = bf16(sigma(Z))              (forward A-GEMM)
-//   EPI_DSIGMA  dZ = bf16(acc * sigma'(Z_saved)); with CoLA-M also
+//   EPI_DSIGMA  dZ = bf16(acc * sigma'(Z_saved)); EPI_DSIGMA_H (CoLA-M) also
 //               H = bf16(sigma(Z_saved)) for the weight gradient of B
 //   EPI_F32     fp32 split-K partial slab, reduced (in a fixed order) by the
 //               reduce kernel: fp32-accumulated weight gradients, and the
@@ -92,7 +92,10 @@ enum : unsigned int {
     ST_TIMEOUT_DRAIN = 1u << 3,
 };
 
-enum Epi : int { EPI_STORE = 0, EPI_ZH = 1, EPI_DSIGMA = 2, EPI_F32 = 3, EPI_TAIL = 4, EPI_GLU = 5, EPI_GLU_BWD = 6 };
+enum Epi : int {
+    EPI_STORE = 0, EPI_ZH = 1, EPI_DSIGMA = 2, EPI_F32 = 3, EPI_TAIL = 4, EPI_GLU = 5, EPI_GLU_BWD = 6,
+    EPI_DSIGMA_H = 7
+};
 enum Sigma : int { SIG_IDENTITY = 0, SIG_SILU = 1, SIG_GELU = 2 };
 
 struct GemmParams {
@@ -104,7 +107,7 @@ struct GemmParams {
     void* D;               // EPI_F32: fp32 partial slabs (bf16 outputs go through map_d / map_d2)
     long long ldd;         // EPI_F32: row pitch of a slab in elements
     long long part_stride; // EPI_F32: elements per split slab
-    int has_d2;            // EPI_ZH / EPI_DSIGMA: also store H through map_d2
+    int has_d2;            // EPI_ZH: also store H through map_d2 (EPI_DSIGMA_H always does)
     int h_only;            // EPI_ZH: store H = sigma(bf16(acc)) through map_d and nothing else
     // tile order within the problem: 0 = row-major (n_blk fastest), 1 =
     // column-major (m_blk fastest).  A wave of CTAs walking the reduction in
@@ -445,6 +448,12 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     // the single-CTA GEMMs of the LLaMA-60M block 5-7 % slower, which keep
     // freeing it after their stores)
     constexpr bool EARLY_FREE = EPI == EPI_STORE && PAIR;
+    // the dZ epilogue: EPI_DSIGMA_H (CoLA-M) also stores H = sigma(Z), formed
+    // with sigma'(Z) from one logistic; a kind of its own so that the
+    // register budget of the CoLA form (dZ alone) is unaffected (measured:
+    // a run-time switch between the two made the LLaMA-60M dZ GEMMs 4-10 %
+    // slower)
+    constexpr bool DSIG = EPI == EPI_DSIGMA || EPI == EPI_DSIGMA_H;
     using C = GemmCfg<BN, MSUB, PAIR, EPI == EPI_GLU ? 2 : 1, GLU_SPLIT ? 1 : 2>;
     constexpr int STAGES = C::STAGES;
     constexpr int TILE_M = C::TILE_M;
@@ -496,7 +505,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             tma_prefetch_desc(&batch.prob[g].map_a);
             tma_prefetch_desc(&batch.prob[g].map_b);
             if (EPI != EPI_F32) tma_prefetch_desc(&batch.prob[g].map_d);
-            if (EPI == EPI_DSIGMA) tma_prefetch_desc(&batch.prob[g].map_z);
+            if (DSIG) tma_prefetch_desc(&batch.prob[g].map_z);
             if (EPI == EPI_GLU) {
                 tma_prefetch_desc(&batch.prob[g].map_b2);
                 tma_prefetch_desc(&batch.prob[g].map_d2);
@@ -878,7 +887,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             zc += C_STEP;
             z_advance();
         };
-        if (EPI == EPI_DSIGMA) {
+        if (DSIG) {
             z_advance();
             z_issue();
         }
@@ -1006,7 +1015,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 #pragma unroll 1
             for (int c = c_first; c < nch; c += C_STEP) {
                 const int col0 = n_blk * BN + c * 32;
-                if (EPI == EPI_DSIGMA) z_issue();   // the next item's Z box, while this one is processed
+                if (DSIG) z_issue();   // the next item's Z box, while this one is processed
                 // EPI_GLU_BWD: this row's Y_gate and Y_up chunk, loaded ahead of the accumulator
                 uint4 yg[4], yu[4];
                 if constexpr (EPI == EPI_GLU_BWD) {
@@ -1103,7 +1112,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                         });
                         emit(p.h_only ? map_d : map_d2, w, col0, row0);
                     }
-                } else if (EPI == EPI_DSIGMA) {
+                } else if (DSIG) {
                     const int b = zuse & 1;
                     const bool zok = wait_bounded(&zbar[b], (zphase >> b) & 1u, wc, ST_TIMEOUT_EPILOGUE);
                     zphase ^= 1u << b;
@@ -1122,10 +1131,11 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                         z[4 * j + 2] = t.z;
                         z[4 * j + 3] = t.w;
                     }
-                    uint32_t hw[16];   // CoLA-M: H = sigma(Z), formed with sigma'(Z)
-                    with_sigma(p.sigma, [&](auto tag) {
-                        constexpr int S = decltype(tag)::value;
-                        if (p.has_d2) {
+                    if constexpr (EPI == EPI_DSIGMA_H) {
+                        // CoLA-M: H = sigma(Z) formed with sigma'(Z), stored through the same box
+                        uint32_t hw[16];
+                        with_sigma(p.sigma, [&](auto tag) {
+                            constexpr int S = decltype(tag)::value;
 #pragma unroll
                             for (int j = 0; j < 16; ++j) {
                                 float hl, dl, hh, dh;
@@ -1134,22 +1144,26 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                                 w[j] = pack_bf16x2(__uint_as_float(v[2 * j]) * dl, __uint_as_float(v[2 * j + 1]) * dh);
                                 hw[j] = pack_bf16x2(hl, hh);
                             }
-                        } else {
-#pragma unroll
-                            for (int j = 0; j < 16; ++j)
-                                w[j] = pack_bf16x2(__uint_as_float(v[2 * j]) * act_dsigma<S>(bf16_lo(z[j])),
-                                                   __uint_as_float(v[2 * j + 1]) * act_dsigma<S>(bf16_hi(z[j])));
-                        }
-                    });
-                    stage_row(box, lane, w);        // dZ in place of this row's Z
-                    fence_proxy_async_smem();
-                    store_box(map_d, box, col0, row0);
-                    if (p.has_d2) {                 // CoLA-M: H through the same box
+                        });
+                        stage_row(box, lane, w);    // dZ in place of this row's Z
+                        fence_proxy_async_smem();
+                        store_box(map_d, box, col0, row0);
                         if (lane == 0) bulk_wait_group_read<0>();
                         __syncwarp();
                         stage_row(box, lane, hw);
                         fence_proxy_async_smem();
                         store_box(map_d2, box, col0, row0);
+                    } else {
+                        with_sigma(p.sigma, [&](auto tag) {
+                            constexpr int S = decltype(tag)::value;
+#pragma unroll
+                            for (int j = 0; j < 16; ++j)
+                                w[j] = pack_bf16x2(__uint_as_float(v[2 * j]) * act_dsigma<S>(bf16_lo(z[j])),
+                                                   __uint_as_float(v[2 * j + 1]) * act_dsigma<S>(bf16_hi(z[j])));
+                        });
+                        stage_row(box, lane, w);    // dZ in place of this row's Z
+                        fence_proxy_async_smem();
+                        store_box(map_d, box, col0, row0);
                     }
                 }
             }

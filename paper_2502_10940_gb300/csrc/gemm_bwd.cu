@@ -1,4 +1,5 @@
-// Backward activation-gradient GEMMs: dZ = (dY B) * sigma'(Z) (EPI_DSIGMA) and
+// Backward activation-gradient GEMMs: dZ = (dY B) * sigma'(Z) (EPI_DSIGMA; with
+// H = sigma(Z) for CoLA-M, EPI_DSIGMA_H) and
 // dX = dZ A (EPI_STORE); A operand K-major, B operand (a weight read
 // transposed) MN-major.
 #define COLA_DEFINE_LAUNCHERS
@@ -9,6 +10,10 @@ template cudaError_t launch_gemm<128, 1, false, true, EPI_DSIGMA>(const GemmBatc
 template cudaError_t launch_gemm<256, 1, false, true, EPI_DSIGMA>(const GemmBatch&, int, bool, cudaStream_t);
 template cudaError_t launch_gemm<128, 2, false, true, EPI_DSIGMA>(const GemmBatch&, int, bool, cudaStream_t);
 template cudaError_t launch_gemm<256, 1, false, true, EPI_DSIGMA, true>(const GemmBatch&, int, bool, cudaStream_t);
+template cudaError_t launch_gemm<128, 1, false, true, EPI_DSIGMA_H>(const GemmBatch&, int, bool, cudaStream_t);
+template cudaError_t launch_gemm<256, 1, false, true, EPI_DSIGMA_H>(const GemmBatch&, int, bool, cudaStream_t);
+template cudaError_t launch_gemm<128, 2, false, true, EPI_DSIGMA_H>(const GemmBatch&, int, bool, cudaStream_t);
+template cudaError_t launch_gemm<256, 1, false, true, EPI_DSIGMA_H, true>(const GemmBatch&, int, bool, cudaStream_t);
 template cudaError_t launch_gemm<128, 1, false, true, EPI_STORE>(const GemmBatch&, int, bool, cudaStream_t);
 template cudaError_t launch_gemm<256, 1, false, true, EPI_STORE>(const GemmBatch&, int, bool, cudaStream_t);
 template cudaError_t launch_gemm<128, 2, false, true, EPI_STORE>(const GemmBatch&, int, bool, cudaStream_t);
