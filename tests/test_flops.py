@@ -84,3 +84,30 @@ def test_saved_activations_app_c(name):
     assert W.saved_activation_elems(wl, "cola") == 14 * wl.n * r
     assert W.saved_activation_elems(wl, "cola_m") == 7 * wl.n * r
     assert W.saved_activation_elems(wl, "infer") == 0
+
+
+@pytest.mark.parametrize("n,d_in,d_out,r", [(2048, 512, 512, 128), (19456, 1376, 512, 64), (300, 200, 328, 128)])
+@pytest.mark.parametrize("with_h", [False, True])
+def test_fused_launch_accounting_matches_the_two_gemms(n, d_in, d_out, r, with_h):
+    # bench.py's algorithmic bytes of a single-kernel pass are those of the two
+    # GEMMs it replaces less the rank-r intermediate's round trip (written by
+    # the first, read by the second: here it never leaves the chip); the FLOPs
+    # are the two GEMMs' FLOPs
+    import sys
+    sys.path.insert(0, os.path.join(os.path.dirname(__file__), ".."))
+    import bench
+    e = 2
+    # forward: the two-GEMM form always writes Z and H (H kept, or in the
+    # workspace to feed F2); the single kernel stores Z, and H only when kept
+    fz, ff = bench.launch_cost("fwd_zh", [(n, r, d_in)], 1, 1)
+    yz, yf = bench.launch_cost("fwd_y", [(n, d_out, r)], 1, 0)
+    fb, fl = bench.launch_cost("fwd_fused", [(n, r, d_in), (n, d_out, r)], 1, (1 if with_h else 0) | 64)
+    saved = e * n * r * (1 if with_h else 2)      # H not re-read (and, when not kept, not written)
+    assert fb == fz + yz - saved
+    assert fl == ff + yf
+    # backward: dZ (and H under CoLA-M) stored; dX from dZ on chip
+    dz, dzf = bench.launch_cost("bwd_dz", [(n, r, d_out)], 1, 1 if with_h else 0)
+    dx, dxf = bench.launch_cost("bwd_dx", [(n, d_in, r)], 1, 0)
+    bb, bf = bench.launch_cost("bwd_fused", [(n, r, d_out), (n, d_in, r)], 1, 1 if with_h else 0)
+    assert bb == dz + dx - e * n * r
+    assert bf == dzf + dxf
