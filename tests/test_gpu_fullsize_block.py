@@ -1,6 +1,7 @@
 """GPU parity of the whole LLaMA-shaped CoLA block in the launch configuration
-bench.py times, at 1B and 7B widths, against the fp64 oracle on sampled
-outputs it computes one by one.
+bench.py times, at 1B and 7B widths (and at 60M and 350M widths, the bench's
+token counts), against the fp64 oracle on sampled outputs it computes one by
+one.
 
 The block runs q/k/v through the shared-input entry points with count 3
 (one Z/H GEMM with N = 3r, the three Y GEMMs and the three dZ GEMMs as one
@@ -73,11 +74,12 @@ def _block(name, n, mode):
     return bench.Block(wl, mode, "cuda:0", seed=5)
 
 
-def _check_trace(records, groups):
+def _check_trace(records, groups, pair=True):
     gemms = [r for r in records if r[0] in ("fwd_zh", "fwd_y", "bwd_dz", "wgrad", "bwd_dx")]
     assert len(gemms) == 5 * len(groups), [r[0] for r in records]
-    for kind, shapes, splits, flags, _ in gemms:
-        assert flags & PAIR, (kind, shapes, flags)
+    if pair:
+        for kind, shapes, splits, flags, _ in gemms:
+            assert flags & PAIR, (kind, shapes, flags)
     counts = {k: sorted(len(s) for kk, s, *_ in gemms if kk == k) for k in ("fwd_y", "bwd_dz", "wgrad")}
     # q/k/v (3 problems; weight gradients 3 dB + dA_qkv) and gate/up (2; 2 dB + dA)
     assert counts["fwd_y"] == [1, 1, 2, 3], counts
@@ -98,7 +100,28 @@ def test_block_groups_sampled(case):
     records = tr.records()
     blk.check()
     _check_trace(records, blk.groups)
+    _sample_groups(blk, n)
 
+
+# The LLaMA-60M and 350M blocks at the bench's token counts: their GEMMs are
+# HBM-bound single-CTA launches (60M), or a mix of CTA-pair launches (the
+# compute-heavy Z/H, dZ and weight-gradient GEMMs) and single-CTA ones (the
+# rank-256 Y and dX GEMMs, K = 256) at 350M; the launch structure is the same.
+@pytest.mark.parametrize("case", [("60m", 65536, "cola"), ("350m", 131072, "cola")],
+                         ids=lambda c: f"{c[0]}-n{c[1]}-{c[2]}")
+def test_block_groups_sampled_smaller_widths(case):
+    from paper_2502_10940_gb300 import cola
+    name, n, mode = case
+    blk = _block(name, n, mode)
+    with cola.Trace(64) as tr:
+        blk.step()
+    records = tr.records()
+    blk.check()
+    _check_trace(records, blk.groups, pair=False)
+    _sample_groups(blk, n)
+
+
+def _sample_groups(blk, n):
     rng = np.random.default_rng(2024)
     tail = [n - 1 - k for k in (0, 1, 63, 64, 127, 128, 200, 255, 256)]
     for g in blk.groups:
