@@ -441,20 +441,29 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) fused_layer_kernel(const __gri
                     const bool want_h = P.store_s2 && first;
                     with_sigma(P.sigma, [&](auto tag) {
                         constexpr int S = decltype(tag)::value;
+                        if constexpr (S == SIG_SILU) {
+                            if (below_tanh_floor(z)) {
+                                if (want_h)
+                                    dsilu_silu_chunk_fallback(z, v, w, h);
+                                else
+                                    dsilu_chunk_fallback(z, v, w);
+                                return;
+                            }
+                        }
                         if (want_h) {
 #pragma unroll
                             for (int j = 0; j < 16; ++j) {
                                 float hl, dl, hh, dh;
-                                act_both<S>(bf16_lo(z[j]), hl, dl);
-                                act_both<S>(bf16_hi(z[j]), hh, dh);
+                                act_both<S, LOGI_TANH>(bf16_lo(z[j]), hl, dl);
+                                act_both<S, LOGI_TANH>(bf16_hi(z[j]), hh, dh);
                                 w[j] = pack_bf16x2(__uint_as_float(v[2 * j]) * dl, __uint_as_float(v[2 * j + 1]) * dh);
                                 h[j] = pack_bf16x2(hl, hh);
                             }
                         } else {
 #pragma unroll
                             for (int j = 0; j < 16; ++j)
-                                w[j] = pack_bf16x2(__uint_as_float(v[2 * j]) * act_dsigma<S>(bf16_lo(z[j])),
-                                                   __uint_as_float(v[2 * j + 1]) * act_dsigma<S>(bf16_hi(z[j])));
+                                w[j] = pack_bf16x2(__uint_as_float(v[2 * j]) * act_dsigma<S, LOGI_TANH>(bf16_lo(z[j])),
+                                                   __uint_as_float(v[2 * j + 1]) * act_dsigma<S, LOGI_TANH>(bf16_hi(z[j])));
                         }
                     });
                     if (P.store_s1 && first) emit(&P.map_s1, w, c * 32, row0);
@@ -467,8 +476,16 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) fused_layer_kernel(const __gri
                     if (P.store_s1 && first) emit(&P.map_s1, w, c * 32, row0);
                     with_sigma(P.sigma, [&](auto tag) {
                         constexpr int S = decltype(tag)::value;
+                        if constexpr (S == SIG_SILU) {
+                            if (below_tanh_floor(w)) {
+                                silu_chunk_fallback(w);
+                                return;
+                            }
+                        }
 #pragma unroll
-                        for (int j = 0; j < 16; ++j) w[j] = pack_bf16x2(act_sigma<S>(bf16_lo(w[j])), act_sigma<S>(bf16_hi(w[j])));
+                        for (int j = 0; j < 16; ++j)
+                            w[j] = pack_bf16x2(act_sigma<S, LOGI_TANH>(bf16_lo(w[j])),
+                                               act_sigma<S, LOGI_TANH>(bf16_hi(w[j])));
                     });
                     if (P.store_s2 && first) emit(&P.map_s2, w, c * 32, row0);
                 }

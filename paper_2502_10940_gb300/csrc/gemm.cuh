@@ -176,28 +176,86 @@ struct GemmCfg {
     static_assert(SMEM_BYTES <= SMEM_LIMIT, "shared memory budget");
 };
 
+// two bf16 values packed in a 32-bit word (low half first) and back
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi)
+{
+    __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+    return *reinterpret_cast<uint32_t*>(&v);
+}
+
+__device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
+__device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
+
 // ------------------------------------------------------------ activations
-// logistic(z) with the fast exponential and divide (a few ulp of fp32, far
-// below the bf16 rounding every result goes through); exactly 0 below -87,
-// where e^{-z} would leave the range of the fast divide.
-__device__ __forceinline__ float logistic_fast(float z)
+// The logistic s(z) = 1 / (1 + e^{-z}) of SiLU, in two forms:
+//   tanh form         s = 1/2 + tanh(z/2)/2 with tanh from the special-function
+//   (logistic_tanh)   unit's approximation: one MUFU operation per element.
+//                     For z < 0 the sum cancels (s -> 0 while tanh -> -1), so
+//                     this form serves only z >= -TANH_FLOOR, where its
+//                     relative error stays below 1e-4 (measured on every bf16
+//                     input: a twentieth of half a bf16 ulp).
+//   exponential form  s = 1 / (1 + e^{-z}) with the fast exponential and
+//   (logistic_exp)    divide (a few ulp of fp32): two MUFU operations; exactly
+//                     0 below -87, where e^{-z} would leave the range of the
+//                     fast divide.
+// The value of every element is logistic_of<LOGI_SELECT>(z): the exponential
+// form below -TANH_FLOOR, the tanh form elsewhere.  The epilogues evaluate a
+// chunk of a row (32 values) with no input below the floor (under N(0, 1)
+// inputs, all but about 1 in 10^9) by the tanh form alone
+// (logistic_of<LOGI_TANH>), and any other chunk element by element with the
+// choice, out of line (the *_chunk_select functions below), so a result never
+// depends on its neighbours.  The SFU rate bounds the sigma epilogues of the
+// HBM-bound launches, which the single-operation form relieves.  Every sigma
+// input is a bf16 value (the stored Z); over all of them the result is
+// checked through the library against the oracle.
+constexpr float TANH_FLOOR = 6.0f;
+constexpr uint32_t TANH_FLOOR_BF16_NEG = 0xC0C0u;   // bf16 bit pattern of -6.0
+enum { LOGI_TANH = 0, LOGI_SELECT = 1 };
+
+__device__ __forceinline__ float logistic_tanh(float z)
+{
+    float t;
+    asm("tanh.approx.f32 %0, %1;" : "=f"(t) : "f"(0.5f * z));
+    return fmaf(0.5f, t, 0.5f);
+}
+
+__device__ __forceinline__ float logistic_exp(float z)
 {
     return z < -87.0f ? 0.0f : __fdividef(1.0f, 1.0f + __expf(-z));
 }
 
-template <int SIG>
+template <int L>
+__device__ __forceinline__ float logistic_of(float z)
+{
+    if (L == LOGI_TANH) return logistic_tanh(z);
+    return z < -TANH_FLOOR ? logistic_exp(z) : logistic_tanh(z);
+}
+
+// Whether any of the 2N bf16 values packed in w lies below -TANH_FLOOR
+// (negative with a magnitude above the floor's: as unsigned 16-bit patterns,
+// above -6.0's; NaN patterns with the sign bit set count too, harmlessly).
+template <int N>
+__device__ __forceinline__ bool below_tanh_floor(const uint32_t (&w)[N])
+{
+    uint32_t m = 0;
+#pragma unroll
+    for (int j = 0; j < N; ++j) m = __vmaxu2(m, w[j]);
+    return (m & 0xFFFFu) > TANH_FLOOR_BF16_NEG || (m >> 16) > TANH_FLOOR_BF16_NEG;
+}
+
+template <int SIG, int L = LOGI_SELECT>
 __device__ __forceinline__ float act_sigma(float z)
 {
-    if (SIG == SIG_SILU) return z * logistic_fast(z);
+    if (SIG == SIG_SILU) return z * logistic_of<L>(z);
     if (SIG == SIG_GELU) return 0.5f * z * erfcf(-z * 0.70710678118654752f);
     return z;
 }
 
-template <int SIG>
+template <int SIG, int L = LOGI_SELECT>
 __device__ __forceinline__ float act_dsigma(float z)
 {
     if (SIG == SIG_SILU) {
-        const float s = logistic_fast(z);
+        const float s = logistic_of<L>(z);
         return s * (1.0f + z * (1.0f - s));
     }
     if (SIG == SIG_GELU) {
@@ -210,11 +268,11 @@ __device__ __forceinline__ float act_dsigma(float z)
 
 // sigma(z) and sigma'(z) together, sharing the logistic (SiLU) or the normal
 // CDF and density (GELU): the same values as act_sigma and act_dsigma.
-template <int SIG>
+template <int SIG, int L = LOGI_SELECT>
 __device__ __forceinline__ void act_both(float z, float& h, float& d)
 {
     if (SIG == SIG_SILU) {
-        const float s = logistic_fast(z);
+        const float s = logistic_of<L>(z);
         h = z * s;
         d = s * (1.0f + z * (1.0f - s));
     } else if (SIG == SIG_GELU) {
@@ -244,6 +302,95 @@ __device__ __forceinline__ void with_sigma(int sigma, Fn&& fn)
         fn(SigTag<SIG_GELU>{});
     else
         fn(SigTag<SIG_IDENTITY>{});
+}
+
+// The SiLU steps of one epilogue chunk (a row's 32 values, 16 packed bf16
+// pairs) that holds an input below the tanh form's floor: every element
+// takes logistic_of<LOGI_SELECT>.  Out of line, so that the unrolled loops of
+// the common chunk (LOGI_TANH) stay compact: measured, inlining both forms
+// cost the small launches more in cold instruction fetches than the rare
+// call costs here.  Arguments and results pass by value.
+struct Words16 {
+    uint32_t w[16];
+};
+struct Words32 {
+    uint32_t w[32];
+};
+
+static __device__ __noinline__ Words16 silu_chunk_select(Words16 z)
+{
+    Words16 h;
+#pragma unroll
+    for (int j = 0; j < 16; ++j)
+        h.w[j] = pack_bf16x2(act_sigma<SIG_SILU>(bf16_lo(z.w[j])), act_sigma<SIG_SILU>(bf16_hi(z.w[j])));
+    return h;
+}
+
+// dZ = bf16(acc * sigma'(Z)) for a chunk of fp32 accumulators acc
+static __device__ __noinline__ Words16 dsilu_chunk_select(Words16 z, Words32 acc)
+{
+    Words16 d;
+#pragma unroll
+    for (int j = 0; j < 16; ++j)
+        d.w[j] = pack_bf16x2(__uint_as_float(acc.w[2 * j]) * act_dsigma<SIG_SILU>(bf16_lo(z.w[j])),
+                             __uint_as_float(acc.w[2 * j + 1]) * act_dsigma<SIG_SILU>(bf16_hi(z.w[j])));
+    return d;
+}
+
+// dZ (words 0..15) and H = sigma(Z) (words 16..31) together
+static __device__ __noinline__ Words32 dsilu_silu_chunk_select(Words16 z, Words32 acc)
+{
+    Words32 o;
+#pragma unroll
+    for (int j = 0; j < 16; ++j) {
+        float hl, dl, hh, dh;
+        act_both<SIG_SILU>(bf16_lo(z.w[j]), hl, dl);
+        act_both<SIG_SILU>(bf16_hi(z.w[j]), hh, dh);
+        o.w[j] = pack_bf16x2(__uint_as_float(acc.w[2 * j]) * dl, __uint_as_float(acc.w[2 * j + 1]) * dh);
+        o.w[16 + j] = pack_bf16x2(hl, hh);
+    }
+    return o;
+}
+
+// In-register front ends of the three: w = sigma(w); w = dZ; w = dZ, h = H.
+__device__ __forceinline__ void silu_chunk_fallback(uint32_t (&w)[16])
+{
+    Words16 a;
+#pragma unroll
+    for (int j = 0; j < 16; ++j) a.w[j] = w[j];
+    a = silu_chunk_select(a);
+#pragma unroll
+    for (int j = 0; j < 16; ++j) w[j] = a.w[j];
+}
+
+__device__ __forceinline__ void dsilu_chunk_fallback(const uint32_t (&z)[16], const uint32_t (&v)[32], uint32_t (&w)[16])
+{
+    Words16 a;
+    Words32 b;
+#pragma unroll
+    for (int j = 0; j < 16; ++j) a.w[j] = z[j];
+#pragma unroll
+    for (int j = 0; j < 32; ++j) b.w[j] = v[j];
+    a = dsilu_chunk_select(a, b);
+#pragma unroll
+    for (int j = 0; j < 16; ++j) w[j] = a.w[j];
+}
+
+__device__ __forceinline__ void dsilu_silu_chunk_fallback(const uint32_t (&z)[16], const uint32_t (&v)[32],
+                                                          uint32_t (&w)[16], uint32_t (&h)[16])
+{
+    Words16 a;
+    Words32 b;
+#pragma unroll
+    for (int j = 0; j < 16; ++j) a.w[j] = z[j];
+#pragma unroll
+    for (int j = 0; j < 32; ++j) b.w[j] = v[j];
+    b = dsilu_silu_chunk_select(a, b);
+#pragma unroll
+    for (int j = 0; j < 16; ++j) {
+        w[j] = b.w[j];
+        h[j] = b.w[16 + j];
+    }
 }
 
 // --------------------------------------------------------- bounded waits
@@ -396,15 +543,6 @@ __device__ __forceinline__ bool work_next(const GemmBatch& b, int unit_step, Wor
     }
     return true;
 }
-
-__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi)
-{
-    __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
-    return *reinterpret_cast<uint32_t*>(&v);
-}
-
-__device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
-__device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
 
 // Byte offset of 16-byte chunk j of row i inside a 32 x 32 bf16 box laid out
 // with the TMA 64-byte swizzle (chunk bits 4-5 XOR address bits 7-8).
@@ -1106,9 +1244,16 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                     if (p.has_d2 || p.h_only) {
                         with_sigma(p.sigma, [&](auto tag) {
                             constexpr int S = decltype(tag)::value;
+                            if constexpr (S == SIG_SILU) {
+                                if (below_tanh_floor(w)) {
+                                    silu_chunk_fallback(w);
+                                    return;
+                                }
+                            }
 #pragma unroll
                             for (int j = 0; j < 16; ++j)
-                                w[j] = pack_bf16x2(act_sigma<S>(bf16_lo(w[j])), act_sigma<S>(bf16_hi(w[j])));
+                                w[j] = pack_bf16x2(act_sigma<S, LOGI_TANH>(bf16_lo(w[j])),
+                                                   act_sigma<S, LOGI_TANH>(bf16_hi(w[j])));
                         });
                         emit(p.h_only ? map_d : map_d2, w, col0, row0);
                     }
@@ -1136,11 +1281,17 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                         uint32_t hw[16];
                         with_sigma(p.sigma, [&](auto tag) {
                             constexpr int S = decltype(tag)::value;
+                            if constexpr (S == SIG_SILU) {
+                                if (below_tanh_floor(z)) {
+                                    dsilu_silu_chunk_fallback(z, v, w, hw);
+                                    return;
+                                }
+                            }
 #pragma unroll
                             for (int j = 0; j < 16; ++j) {
                                 float hl, dl, hh, dh;
-                                act_both<S>(bf16_lo(z[j]), hl, dl);
-                                act_both<S>(bf16_hi(z[j]), hh, dh);
+                                act_both<S, LOGI_TANH>(bf16_lo(z[j]), hl, dl);
+                                act_both<S, LOGI_TANH>(bf16_hi(z[j]), hh, dh);
                                 w[j] = pack_bf16x2(__uint_as_float(v[2 * j]) * dl, __uint_as_float(v[2 * j + 1]) * dh);
                                 hw[j] = pack_bf16x2(hl, hh);
                             }
@@ -1156,10 +1307,16 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                     } else {
                         with_sigma(p.sigma, [&](auto tag) {
                             constexpr int S = decltype(tag)::value;
+                            if constexpr (S == SIG_SILU) {
+                                if (below_tanh_floor(z)) {
+                                    dsilu_chunk_fallback(z, v, w);
+                                    return;
+                                }
+                            }
 #pragma unroll
                             for (int j = 0; j < 16; ++j)
-                                w[j] = pack_bf16x2(__uint_as_float(v[2 * j]) * act_dsigma<S>(bf16_lo(z[j])),
-                                                   __uint_as_float(v[2 * j + 1]) * act_dsigma<S>(bf16_hi(z[j])));
+                                w[j] = pack_bf16x2(__uint_as_float(v[2 * j]) * act_dsigma<S, LOGI_TANH>(bf16_lo(z[j])),
+                                                   __uint_as_float(v[2 * j + 1]) * act_dsigma<S, LOGI_TANH>(bf16_hi(z[j])));
                         });
                         stage_row(box, lane, w);    // dZ in place of this row's Z
                         fence_proxy_async_smem();

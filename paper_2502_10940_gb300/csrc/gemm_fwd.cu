@@ -17,6 +17,17 @@ template cudaError_t launch_gemm<256, 1, false, false, EPI_STORE, true>(const Ge
 // H = bf16(sigma(Z)) over `vecs` groups of 8 bf16, each a 16-byte vector;
 // sigma is evaluated exactly as in the Z/H epilogue (same function on the
 // same bf16 inputs), so the result is bit-identical to the forward's H.
+template <int S, int L>
+__device__ __forceinline__ uint4 sigma8(const uint4 z)
+{
+    uint4 h;
+    h.x = pack_bf16x2(act_sigma<S, L>(bf16_lo(z.x)), act_sigma<S, L>(bf16_hi(z.x)));
+    h.y = pack_bf16x2(act_sigma<S, L>(bf16_lo(z.y)), act_sigma<S, L>(bf16_hi(z.y)));
+    h.z = pack_bf16x2(act_sigma<S, L>(bf16_lo(z.z)), act_sigma<S, L>(bf16_hi(z.z)));
+    h.w = pack_bf16x2(act_sigma<S, L>(bf16_lo(z.w)), act_sigma<S, L>(bf16_hi(z.w)));
+    return h;
+}
+
 template <int S>
 __global__ void __launch_bounds__(256) sigma_kernel(const uint4* __restrict__ Z, uint4* __restrict__ H, long long vecs)
 {
@@ -25,12 +36,9 @@ __global__ void __launch_bounds__(256) sigma_kernel(const uint4* __restrict__ Z,
     const long long stride = static_cast<long long>(gridDim.x) * blockDim.x;
     for (long long i = static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x; i < vecs; i += stride) {
         const uint4 z = __ldg(Z + i);
-        uint4 h;
-        h.x = pack_bf16x2(act_sigma<S>(bf16_lo(z.x)), act_sigma<S>(bf16_hi(z.x)));
-        h.y = pack_bf16x2(act_sigma<S>(bf16_lo(z.y)), act_sigma<S>(bf16_hi(z.y)));
-        h.z = pack_bf16x2(act_sigma<S>(bf16_lo(z.z)), act_sigma<S>(bf16_hi(z.z)));
-        h.w = pack_bf16x2(act_sigma<S>(bf16_lo(z.w)), act_sigma<S>(bf16_hi(z.w)));
-        H[i] = h;
+        const uint32_t zw[4] = {z.x, z.y, z.z, z.w};
+        // the logistic's tanh form alone where no input lies below its floor
+        H[i] = (S == SIG_SILU && !below_tanh_floor(zw)) ? sigma8<S, LOGI_TANH>(z) : sigma8<S, LOGI_SELECT>(z);
     }
 }
 

@@ -1,0 +1,161 @@
+"""sigma and sigma' through the library on every finite bf16 input (Sec. 3.2,
+h = B sigma(A x) with SiLU; Sec. 3.4, the chain rule through sigma).
+
+Every input of sigma in the kernels is a stored bf16 Z, so the 65,280 finite
+bf16 values are all the inputs the activation can ever see.  A layer whose Z
+enumerates them: n = 512 tokens, X = [I | 0] (the identity, then zero
+columns), so that Z = X A^T is A's first 512 columns transposed, exactly
+(one nonzero product per sum); A (r = 128 rows) holds every finite bit
+pattern once in those columns.  B is the identity (d_out = r) and dY is all
+ones, so Y = H B^T = H and dH = dY B = 1: dZ = sigma'(Z), and dA = dZ^T X
+holds dZ transposed in its first 512 columns, again exactly.
+
+Each epilogue that evaluates sigma runs once: the single-kernel forward and
+backward (CoLA, and CoLA-M where sigma and sigma' are formed together), the
+two-GEMM forward (its Z/H epilogue at d_in = 512; at d_in = 1024 the launch
+splits over K and sigma is applied in the reduce) and backward (the dZ
+epilogue, and CoLA-M's with H), and the recompute's elementwise sigma launch
+(Sec. 4.2).  The results are compared with the oracle's fp64 sigma and
+sigma' of the same inputs: every result lies within one bf16 ulp of the
+exactly rounded value (or 1e-6 from it, near the zero of sigma' where an ulp
+is finer than the fp32 evaluation of the logistic resolves), and equals the
+exactly rounded value at all but a small fraction of the inputs.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+
+pytestmark = pytest.mark.gpu
+
+N_TOK, R = 512, 128
+ABS_FLOOR = 1e-6
+# results that are not the exactly rounded value: about half the 254 subnormal
+# inputs (sigma(z) = z/2 + z^2/4 lands on a tie of the bf16 grid that the
+# fp32 product z * 1/2 rounds to even while the exact value breaks it), the
+# few inputs below -87 where the fast divide underflows to 0 (|error| < 1e-36),
+# and rounding flips of the logistic's fp32 error
+MISMATCH_MAX = 5e-3
+
+
+@pytest.fixture(scope="module")
+def cola():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2502_10940_gb300 import build
+    build.build()
+    from paper_2502_10940_gb300 import cola as c
+    yield c
+    c.cola_set_fused_forward(True)
+    c.cola_set_fused_backward(True)
+
+
+def _all_finite_bf16():
+    """(N_TOK x R) bf16 values: every finite bit pattern once, then zeros."""
+    bits = np.arange(65536, dtype=np.uint32)
+    finite = ((bits >> 7) & 0xFF) != 0xFF
+    vals = bits[finite].astype(np.uint16)
+    grid = np.zeros(N_TOK * R, dtype=np.uint16)
+    grid[:vals.size] = vals
+    return torch.from_numpy(grid.view(np.int16).reshape(N_TOK, R).copy()).view(torch.bfloat16), vals.size
+
+
+def _bf16_round(x64):
+    """Round fp64 values to bf16, to nearest with ties to even, in one step:
+    the fp64 significand is cut to bf16's 8 bits (45 bits dropped, the carry
+    running into the exponent), and below 2^-126 the value is rounded to a
+    multiple of bf16's subnormal step 2^-133."""
+    x = np.asarray(x64, dtype=np.float64)
+    u = x.view(np.uint64)
+    lsb = (u >> np.uint64(45)) & np.uint64(1)
+    r = ((u + np.uint64((1 << 44) - 1) + lsb) >> np.uint64(45)) << np.uint64(45)
+    sub = np.abs(x) < 2.0 ** -126
+    return np.where(sub, np.round(x / 2.0 ** -133) * 2.0 ** -133, r.view(np.float64))
+
+
+def _bf16_ulp(v):
+    """Spacing of the bf16 grid at each (bf16) value: 2^(e-7) for a normal
+    value with exponent e, 2^-133 for subnormals and zero."""
+    a = np.abs(v)
+    e = np.floor(np.log2(np.where(a > 0, a, 1.0)))
+    return np.where(a >= 2.0 ** -126, 2.0 ** (e - 7), 2.0 ** -133)
+
+
+def _check(name, got, exact64):
+    ref = _bf16_round(exact64)
+    diff = np.abs(got - ref)
+    tol = np.maximum(_bf16_ulp(ref), ABS_FLOOR)
+    bad = diff > tol
+    assert not bad.any(), (f"{name}: {int(bad.sum())} inputs beyond one ulp, e.g. got {got[bad][:4]} "
+                           f"exact {exact64[bad][:4]}")
+    frac = float((got != ref).mean())
+    print(f"{name}: {frac:.2e} of the inputs not exactly rounded, max |error| {diff.max():.3e}")
+    assert frac <= MISMATCH_MAX, f"{name}: {frac:.2e} of the inputs not exactly rounded"
+    return frac
+
+
+def _layer(cola, d_in, mode, fused):
+    zt, count = _all_finite_bf16()                 # Z's intended values, token-major [N_TOK x R]
+    dev = "cuda"
+    X = torch.zeros((N_TOK, d_in), dtype=torch.bfloat16, device=dev)
+    X[:, :N_TOK] = torch.eye(N_TOK, dtype=torch.bfloat16, device=dev)
+    A = torch.zeros((R, d_in), dtype=torch.bfloat16, device=dev)
+    A[:, :N_TOK] = zt.t().to(dev)
+    B = torch.eye(R, dtype=torch.bfloat16, device=dev)
+    dY = torch.ones((N_TOK, R), dtype=torch.bfloat16, device=dev)
+    d = cola.desc(N_TOK, d_in, R, R, sigma="silu", mode=mode)
+    ws = cola.workspace(d)
+    Y = torch.empty((N_TOK, R), dtype=torch.bfloat16, device=dev)
+    Z = torch.empty((N_TOK, R), dtype=torch.bfloat16, device=dev)
+    H = torch.empty((N_TOK, R), dtype=torch.bfloat16, device=dev) if mode == "cola" else None
+    dX = torch.empty((N_TOK, d_in), dtype=torch.bfloat16, device=dev)
+    dA = torch.empty((R, d_in), dtype=torch.bfloat16, device=dev)
+    dB = torch.empty((R, R), dtype=torch.bfloat16, device=dev)
+    cola.cola_set_fused_forward(fused)
+    cola.cola_set_fused_backward(fused)
+    try:
+        with cola.Trace(16) as tr:
+            cola.cola_fwd(d, X, A, B, Y, Z, H, ws)
+            cola.cola_bwd(d, X, A, B, dY, Z, H, dX, dA, dB, ws)
+    finally:
+        cola.cola_set_fused_forward(True)
+        cola.cola_set_fused_backward(True)
+    assert cola.cola_check_status(ws)[0] == 0
+    recs = tr.records()
+    z = zt.double().numpy().reshape(-1)[:count]
+    assert torch.equal(Z.cpu(), zt), "Z = X A^T must reproduce the enumerated inputs exactly"
+    h = Y.cpu().double().numpy().reshape(-1)[:count]
+    dz = dA[:, :N_TOK].t().cpu().double().numpy().reshape(-1)[:count]
+    return z, h, dz, recs
+
+
+@pytest.mark.parametrize("mode", ["cola", "cola_m"])
+@pytest.mark.parametrize("d_in,fused,fwd_kind,bwd_kind", [
+    (512, True, "fwd_fused", "bwd_fused"),
+    (512, False, "fwd_zh", "bwd_dz"),
+    (1024, False, "fwd_zh", "bwd_dz"),     # the forward splits over K: sigma in the reduce
+], ids=["fused", "two_gemm", "two_gemm_split_k"])
+def test_sigma_every_bf16_input(cola, mode, d_in, fused, fwd_kind, bwd_kind):
+    z, h, dz, recs = _layer(cola, d_in, mode, fused)
+    kinds = [rec[0] for rec in recs]
+    assert fwd_kind in kinds and bwd_kind in kinds, kinds
+    fwd_splits = [rec[2] for rec in recs if rec[0] == fwd_kind][0]
+    assert (fwd_splits > 1) == (d_in == 1024), recs
+    _check("sigma", h, oracle.sigma("silu", z))
+    _check("sigma'", dz, oracle.dsigma("silu", z))
+
+
+def test_recompute_sigma_every_bf16_input(cola):
+    zt, count = _all_finite_bf16()
+    Z = zt.cuda()
+    B = torch.eye(R, dtype=torch.bfloat16, device="cuda")
+    d = cola.desc(N_TOK, R, R, R, sigma="silu", mode="cola_m")
+    ws = cola.workspace(d)
+    Y = torch.empty((N_TOK, R), dtype=torch.bfloat16, device="cuda")
+    with cola.Trace(8) as tr:
+        cola.cola_recompute_up(d, Z, [B], [Y], ws)
+    assert cola.cola_check_status(ws)[0] == 0
+    assert "sigma" in [rec[0] for rec in tr.records()]
+    z = zt.double().numpy().reshape(-1)[:count]
+    _check("sigma (recompute)", Y.cpu().double().numpy().reshape(-1)[:count], oracle.sigma("silu", z))
