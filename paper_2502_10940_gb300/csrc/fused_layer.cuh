@@ -110,7 +110,7 @@ __device__ __forceinline__ uint64_t fused_operand_desc(uint32_t base, int ks)
               : smem_desc_sw128(base + ks * UMMA_K * 2, 16, 1024);
 }
 
-template <int R, bool BWD>
+template <int R, bool BWD, int SIG>
 __global__ void __launch_bounds__(NUM_THREADS, 1) fused_layer_kernel(const __grid_constant__ FusedParams P)
 {
     using C = FusedCfg<R>;
@@ -439,7 +439,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) fused_layer_kernel(const __gri
                     // under CoLA-M also H = sigma(Z), from the same logistic
                     uint32_t h[16];
                     const bool want_h = P.store_s2 && first;
-                    with_sigma(P.sigma, [&](auto tag) {
+                    with_sigma_fixed<SIG>([&](auto tag) {
                         constexpr int S = decltype(tag)::value;
                         if constexpr (S == SIG_SILU) {
                             if (below_tanh_floor(z)) {
@@ -474,7 +474,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) fused_layer_kernel(const __gri
                     for (int j = 0; j < 16; ++j)
                         w[j] = pack_bf16x2(__uint_as_float(v[2 * j]), __uint_as_float(v[2 * j + 1]));
                     if (P.store_s1 && first) emit(&P.map_s1, w, c * 32, row0);
-                    with_sigma(P.sigma, [&](auto tag) {
+                    with_sigma_fixed<SIG>([&](auto tag) {
                         constexpr int S = decltype(tag)::value;
                         if constexpr (S == SIG_SILU) {
                             if (below_tanh_floor(w)) {

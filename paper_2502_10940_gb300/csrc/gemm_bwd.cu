@@ -6,14 +6,54 @@
 #include "gemm_launch.cuh"
 
 namespace cola {
-template cudaError_t launch_gemm<128, 1, false, true, EPI_DSIGMA>(const GemmBatch&, int, bool, cudaStream_t);
-template cudaError_t launch_gemm<256, 1, false, true, EPI_DSIGMA>(const GemmBatch&, int, bool, cudaStream_t);
-template cudaError_t launch_gemm<128, 2, false, true, EPI_DSIGMA>(const GemmBatch&, int, bool, cudaStream_t);
-template cudaError_t launch_gemm<256, 1, false, true, EPI_DSIGMA, true>(const GemmBatch&, int, bool, cudaStream_t);
-template cudaError_t launch_gemm<128, 1, false, true, EPI_DSIGMA_H>(const GemmBatch&, int, bool, cudaStream_t);
-template cudaError_t launch_gemm<256, 1, false, true, EPI_DSIGMA_H>(const GemmBatch&, int, bool, cudaStream_t);
-template cudaError_t launch_gemm<128, 2, false, true, EPI_DSIGMA_H>(const GemmBatch&, int, bool, cudaStream_t);
-template cudaError_t launch_gemm<256, 1, false, true, EPI_DSIGMA_H, true>(const GemmBatch&, int, bool, cudaStream_t);
+template cudaError_t launch_gemm<128, 1, false, true, EPI_DSIGMA, false, SIG_IDENTITY>(
+    const GemmBatch&, int, bool, cudaStream_t);
+template cudaError_t launch_gemm<128, 1, false, true, EPI_DSIGMA, false, SIG_SILU>(
+    const GemmBatch&, int, bool, cudaStream_t);
+template cudaError_t launch_gemm<128, 1, false, true, EPI_DSIGMA, false, SIG_GELU>(
+    const GemmBatch&, int, bool, cudaStream_t);
+template cudaError_t launch_gemm<256, 1, false, true, EPI_DSIGMA, false, SIG_IDENTITY>(
+    const GemmBatch&, int, bool, cudaStream_t);
+template cudaError_t launch_gemm<256, 1, false, true, EPI_DSIGMA, false, SIG_SILU>(
+    const GemmBatch&, int, bool, cudaStream_t);
+template cudaError_t launch_gemm<256, 1, false, true, EPI_DSIGMA, false, SIG_GELU>(
+    const GemmBatch&, int, bool, cudaStream_t);
+template cudaError_t launch_gemm<128, 2, false, true, EPI_DSIGMA, false, SIG_IDENTITY>(
+    const GemmBatch&, int, bool, cudaStream_t);
+template cudaError_t launch_gemm<128, 2, false, true, EPI_DSIGMA, false, SIG_SILU>(
+    const GemmBatch&, int, bool, cudaStream_t);
+template cudaError_t launch_gemm<128, 2, false, true, EPI_DSIGMA, false, SIG_GELU>(
+    const GemmBatch&, int, bool, cudaStream_t);
+template cudaError_t launch_gemm<256, 1, false, true, EPI_DSIGMA, true, SIG_IDENTITY>(
+    const GemmBatch&, int, bool, cudaStream_t);
+template cudaError_t launch_gemm<256, 1, false, true, EPI_DSIGMA, true, SIG_SILU>(
+    const GemmBatch&, int, bool, cudaStream_t);
+template cudaError_t launch_gemm<256, 1, false, true, EPI_DSIGMA, true, SIG_GELU>(
+    const GemmBatch&, int, bool, cudaStream_t);
+template cudaError_t launch_gemm<128, 1, false, true, EPI_DSIGMA_H, false, SIG_IDENTITY>(
+    const GemmBatch&, int, bool, cudaStream_t);
+template cudaError_t launch_gemm<128, 1, false, true, EPI_DSIGMA_H, false, SIG_SILU>(
+    const GemmBatch&, int, bool, cudaStream_t);
+template cudaError_t launch_gemm<128, 1, false, true, EPI_DSIGMA_H, false, SIG_GELU>(
+    const GemmBatch&, int, bool, cudaStream_t);
+template cudaError_t launch_gemm<256, 1, false, true, EPI_DSIGMA_H, false, SIG_IDENTITY>(
+    const GemmBatch&, int, bool, cudaStream_t);
+template cudaError_t launch_gemm<256, 1, false, true, EPI_DSIGMA_H, false, SIG_SILU>(
+    const GemmBatch&, int, bool, cudaStream_t);
+template cudaError_t launch_gemm<256, 1, false, true, EPI_DSIGMA_H, false, SIG_GELU>(
+    const GemmBatch&, int, bool, cudaStream_t);
+template cudaError_t launch_gemm<128, 2, false, true, EPI_DSIGMA_H, false, SIG_IDENTITY>(
+    const GemmBatch&, int, bool, cudaStream_t);
+template cudaError_t launch_gemm<128, 2, false, true, EPI_DSIGMA_H, false, SIG_SILU>(
+    const GemmBatch&, int, bool, cudaStream_t);
+template cudaError_t launch_gemm<128, 2, false, true, EPI_DSIGMA_H, false, SIG_GELU>(
+    const GemmBatch&, int, bool, cudaStream_t);
+template cudaError_t launch_gemm<256, 1, false, true, EPI_DSIGMA_H, true, SIG_IDENTITY>(
+    const GemmBatch&, int, bool, cudaStream_t);
+template cudaError_t launch_gemm<256, 1, false, true, EPI_DSIGMA_H, true, SIG_SILU>(
+    const GemmBatch&, int, bool, cudaStream_t);
+template cudaError_t launch_gemm<256, 1, false, true, EPI_DSIGMA_H, true, SIG_GELU>(
+    const GemmBatch&, int, bool, cudaStream_t);
 template cudaError_t launch_gemm<128, 1, false, true, EPI_STORE>(const GemmBatch&, int, bool, cudaStream_t);
 template cudaError_t launch_gemm<256, 1, false, true, EPI_STORE>(const GemmBatch&, int, bool, cudaStream_t);
 template cudaError_t launch_gemm<128, 2, false, true, EPI_STORE>(const GemmBatch&, int, bool, cudaStream_t);

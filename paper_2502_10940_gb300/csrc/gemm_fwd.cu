@@ -5,10 +5,30 @@
 #include "gemm_launch.cuh"
 
 namespace cola {
-template cudaError_t launch_gemm<128, 1, false, false, EPI_ZH>(const GemmBatch&, int, bool, cudaStream_t);
-template cudaError_t launch_gemm<256, 1, false, false, EPI_ZH>(const GemmBatch&, int, bool, cudaStream_t);
-template cudaError_t launch_gemm<128, 2, false, false, EPI_ZH>(const GemmBatch&, int, bool, cudaStream_t);
-template cudaError_t launch_gemm<256, 1, false, false, EPI_ZH, true>(const GemmBatch&, int, bool, cudaStream_t);
+template cudaError_t launch_gemm<128, 1, false, false, EPI_ZH, false, SIG_IDENTITY>(
+    const GemmBatch&, int, bool, cudaStream_t);
+template cudaError_t launch_gemm<128, 1, false, false, EPI_ZH, false, SIG_SILU>(
+    const GemmBatch&, int, bool, cudaStream_t);
+template cudaError_t launch_gemm<128, 1, false, false, EPI_ZH, false, SIG_GELU>(
+    const GemmBatch&, int, bool, cudaStream_t);
+template cudaError_t launch_gemm<256, 1, false, false, EPI_ZH, false, SIG_IDENTITY>(
+    const GemmBatch&, int, bool, cudaStream_t);
+template cudaError_t launch_gemm<256, 1, false, false, EPI_ZH, false, SIG_SILU>(
+    const GemmBatch&, int, bool, cudaStream_t);
+template cudaError_t launch_gemm<256, 1, false, false, EPI_ZH, false, SIG_GELU>(
+    const GemmBatch&, int, bool, cudaStream_t);
+template cudaError_t launch_gemm<128, 2, false, false, EPI_ZH, false, SIG_IDENTITY>(
+    const GemmBatch&, int, bool, cudaStream_t);
+template cudaError_t launch_gemm<128, 2, false, false, EPI_ZH, false, SIG_SILU>(
+    const GemmBatch&, int, bool, cudaStream_t);
+template cudaError_t launch_gemm<128, 2, false, false, EPI_ZH, false, SIG_GELU>(
+    const GemmBatch&, int, bool, cudaStream_t);
+template cudaError_t launch_gemm<256, 1, false, false, EPI_ZH, true, SIG_IDENTITY>(
+    const GemmBatch&, int, bool, cudaStream_t);
+template cudaError_t launch_gemm<256, 1, false, false, EPI_ZH, true, SIG_SILU>(
+    const GemmBatch&, int, bool, cudaStream_t);
+template cudaError_t launch_gemm<256, 1, false, false, EPI_ZH, true, SIG_GELU>(
+    const GemmBatch&, int, bool, cudaStream_t);
 template cudaError_t launch_gemm<128, 1, false, false, EPI_STORE>(const GemmBatch&, int, bool, cudaStream_t);
 template cudaError_t launch_gemm<256, 1, false, false, EPI_STORE>(const GemmBatch&, int, bool, cudaStream_t);
 template cudaError_t launch_gemm<128, 2, false, false, EPI_STORE>(const GemmBatch&, int, bool, cudaStream_t);

@@ -14,7 +14,9 @@ namespace cola {
 // launch with programmatic stream serialization (the prologue overlaps the
 // previous kernel's tail).  PAIR: clusters of two CTAs (grid even), each
 // pair running one 256-row tile with tcgen05 cta_group::2.
-template <int BN, int MSUB, bool A_MN, bool B_MN, int EPI, bool PAIR = false>
+// SIG: the activation the epilogue applies (EPI_ZH, EPI_DSIGMA, EPI_DSIGMA_H
+// are compiled once per activation; the other kinds take SIG_IDENTITY).
+template <int BN, int MSUB, bool A_MN, bool B_MN, int EPI, bool PAIR = false, int SIG = SIG_IDENTITY>
 cudaError_t launch_gemm(const GemmBatch& batch, int grid, bool pdl, cudaStream_t stream);
 
 // One fixed-order reduction of fp32 split partials into a result: a weight
@@ -72,11 +74,11 @@ cudaError_t launch_tail_reduce(const TailReduce& r, int sms, cudaStream_t stream
 cudaError_t launch_sigma(const void* Z, void* H, long long elems, int sigma, int sms, cudaStream_t stream);
 
 #ifdef COLA_DEFINE_LAUNCHERS
-template <int BN, int MSUB, bool A_MN, bool B_MN, int EPI, bool PAIR>
+template <int BN, int MSUB, bool A_MN, bool B_MN, int EPI, bool PAIR, int SIG>
 cudaError_t launch_gemm(const GemmBatch& batch, int grid, bool pdl, cudaStream_t stream)
 {
     constexpr int smem = GemmCfg<BN, MSUB, PAIR>::SMEM_BYTES;
-    auto kern = gemm_kernel<BN, MSUB, A_MN, B_MN, EPI, PAIR>;
+    auto kern = gemm_kernel<BN, MSUB, A_MN, B_MN, EPI, PAIR, SIG>;
     // the opt-in shared-memory size is a per-device function attribute; host
     // threads may launch concurrently, so the set of configured devices is atomic
     static std::atomic<unsigned long long> configured{0};   // bit d: set on device d

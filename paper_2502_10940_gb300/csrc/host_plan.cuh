@@ -360,8 +360,8 @@ int tile_flags(int bn, int msub)
 // dependent launch hides launch latency and the prologue of short GEMMs
 // (measured: -8 % step time on the HBM-bound 60M block) but costs ~1 % on
 // long ones, so it is used below 64 GFLOP per launch.
-template <bool A_MN, bool B_MN, int EPI>
-cudaError_t dispatch(int bn, int msub, GemmBatch& b, int sms, cudaStream_t s)
+template <bool A_MN, bool B_MN, int EPI, int SIG>
+cudaError_t dispatch_sig(int bn, int msub, GemmBatch& b, int sms, cudaStream_t s)
 {
     double flops = 0.0;
     int units = 0;
@@ -379,16 +379,34 @@ cudaError_t dispatch(int bn, int msub, GemmBatch& b, int sms, cudaStream_t s)
     if constexpr (!small_only) {
         if (msub == TILE_PAIR && bn == 256) {
             const int pairs = units < sms / 2 ? units : sms / 2;
-            return launch_gemm<256, 1, A_MN, B_MN, EPI, true>(b, 2 * pairs, pdl, s);
+            return launch_gemm<256, 1, A_MN, B_MN, EPI, true, SIG>(b, 2 * pairs, pdl, s);
         }
     }
     if (msub != 1 && (bn == 256 || small_only)) return cudaErrorInvalidValue;   // planned tiles exist as above only
     const int grid = units < sms ? units : sms;
-    if (bn == 256) return launch_gemm<256, 1, A_MN, B_MN, EPI>(b, grid, pdl, s);
+    if (bn == 256) return launch_gemm<256, 1, A_MN, B_MN, EPI, false, SIG>(b, grid, pdl, s);
     if constexpr (!small_only) {
-        if (msub != 1) return launch_gemm<128, 2, A_MN, B_MN, EPI>(b, grid, pdl, s);
+        if (msub != 1) return launch_gemm<128, 2, A_MN, B_MN, EPI, false, SIG>(b, grid, pdl, s);
     }
-    return launch_gemm<128, 1, A_MN, B_MN, EPI>(b, grid, pdl, s);
+    return launch_gemm<128, 1, A_MN, B_MN, EPI, false, SIG>(b, grid, pdl, s);
+}
+
+// The launch of a batch whose epilogue applies sigma (EPI_ZH, EPI_DSIGMA,
+// EPI_DSIGMA_H) goes to the kernel compiled for its activation (the problems
+// of one batch share it); the other kinds have one kernel.
+template <bool A_MN, bool B_MN, int EPI>
+cudaError_t dispatch(int bn, int msub, GemmBatch& b, int sms, cudaStream_t s)
+{
+    if constexpr (EPI == EPI_ZH || EPI == EPI_DSIGMA || EPI == EPI_DSIGMA_H) {
+        switch (b.prob[0].p.sigma) {
+        case SIG_SILU: return dispatch_sig<A_MN, B_MN, EPI, SIG_SILU>(bn, msub, b, sms, s);
+        case SIG_GELU: return dispatch_sig<A_MN, B_MN, EPI, SIG_GELU>(bn, msub, b, sms, s);
+        case SIG_IDENTITY: return dispatch_sig<A_MN, B_MN, EPI, SIG_IDENTITY>(bn, msub, b, sms, s);
+        default: return cudaErrorInvalidValue;
+        }
+    } else {
+        return dispatch_sig<A_MN, B_MN, EPI, SIG_IDENTITY>(bn, msub, b, sms, s);
+    }
 }
 
 // The gated-MLP forward launch (EPI_GLU) with `bn`-column tiles: on CTA
