@@ -292,30 +292,16 @@ struct SigTag {
 };
 
 // Run fn(SigTag<SIG>{}): the activation of a kernel specialised for one
-// sigma.  The GEMM and fused-layer kernels whose epilogues evaluate sigma are
-// compiled once per activation: a kernel then holds only its own
-// activation's code, and the small launches, whose code runs once per CTA
-// from a cold instruction cache, fetch less of it (measured: the 2048-token
-// layer step 12 % faster than with the three activations behind a run-time
-// switch in one kernel).
+// sigma, so the unrolled elementwise loops carry no branch on the activation
+// kind.  Every kernel whose epilogue evaluates sigma is compiled once per
+// activation: a kernel then holds only its own activation's code, and the
+// small launches, whose code runs once per CTA from a cold instruction cache,
+// fetch less of it (measured: the 2048-token layer step 12 % faster than with
+// the three activations behind a run-time switch in one kernel).
 template <int SIG, class Fn>
 __device__ __forceinline__ void with_sigma_fixed(Fn&& fn)
 {
     fn(SigTag<SIG>{});
-}
-
-// Run fn(SigTag<sigma>{}) with sigma fixed at compile time, so the unrolled
-// elementwise loops carry no per-element branch on the activation kind (the
-// kernels that are not specialised per activation).
-template <class Fn>
-__device__ __forceinline__ void with_sigma(int sigma, Fn&& fn)
-{
-    if (sigma == SIG_SILU)
-        fn(SigTag<SIG_SILU>{});
-    else if (sigma == SIG_GELU)
-        fn(SigTag<SIG_GELU>{});
-    else
-        fn(SigTag<SIG_IDENTITY>{});
 }
 
 // The SiLU steps of one epilogue chunk (a row's 32 values, 16 packed bf16

@@ -26,6 +26,9 @@ namespace cola {
 constexpr int RED_THREADS = 256;
 constexpr int RED_BATCH = 4;
 
+// ZH: the Z/H epilogue of a split-K Z GEMM with activation SIG (one kernel
+// per activation, as the GEMM epilogues); without it the plain sums.
+template <bool ZH, int SIG>
 __global__ void __launch_bounds__(RED_THREADS) splitk_reduce_kernel(const __grid_constant__ ReduceBatch rb)
 {
     grid_dependency_wait();            // the partials come from the GEMM launched just before
@@ -60,15 +63,11 @@ __global__ void __launch_bounds__(RED_THREADS) splitk_reduce_kernel(const __grid
         }
         const float v[4] = {acc.x, acc.y, acc.z, acc.w};
         const int valid = min(4, job.N - j);
-        if (rb.zh) {
+        if (ZH) {
             // Z = bf16(sum), H = bf16(sigma(bf16 Z)): the split-K form of the Z/H epilogue
             const uint32_t z01 = pack_bf16x2(v[0], v[1]), z23 = pack_bf16x2(v[2], v[3]);
-            uint32_t h01 = 0, h23 = 0;
-            with_sigma(rb.sigma, [&](auto tag) {
-                constexpr int S = decltype(tag)::value;
-                h01 = pack_bf16x2(act_sigma<S>(bf16_lo(z01)), act_sigma<S>(bf16_hi(z01)));
-                h23 = pack_bf16x2(act_sigma<S>(bf16_lo(z23)), act_sigma<S>(bf16_hi(z23)));
-            });
+            const uint32_t h01 = pack_bf16x2(act_sigma<SIG>(bf16_lo(z01)), act_sigma<SIG>(bf16_hi(z01)));
+            const uint32_t h23 = pack_bf16x2(act_sigma<SIG>(bf16_lo(z23)), act_sigma<SIG>(bf16_hi(z23)));
             const long long off = static_cast<long long>(i) * job.ldo + j;   // N = count r: 4 | N
             if (job.out) *reinterpret_cast<uint2*>(reinterpret_cast<__nv_bfloat16*>(job.out) + off) = make_uint2(z01, z23);
             *reinterpret_cast<uint2*>(reinterpret_cast<__nv_bfloat16*>(job.out2) + off) = make_uint2(h01, h23);
@@ -206,7 +205,13 @@ cudaError_t launch_splitk_reduce(ReduceBatch& rb, cudaStream_t stream)
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, splitk_reduce_kernel, rb);
+    if (!rb.zh) return cudaLaunchKernelEx(&cfg, splitk_reduce_kernel<false, SIG_IDENTITY>, rb);
+    switch (rb.sigma) {
+    case SIG_SILU: return cudaLaunchKernelEx(&cfg, splitk_reduce_kernel<true, SIG_SILU>, rb);
+    case SIG_GELU: return cudaLaunchKernelEx(&cfg, splitk_reduce_kernel<true, SIG_GELU>, rb);
+    case SIG_IDENTITY: return cudaLaunchKernelEx(&cfg, splitk_reduce_kernel<true, SIG_IDENTITY>, rb);
+    default: return cudaErrorInvalidValue;
+    }
 }
 
 }  // namespace cola
