@@ -98,7 +98,15 @@ bool heavy_gemm(int64_t M, int64_t N, int64_t K)
     return M > 128 && (flops >= 64e9 || (flops >= 16e9 && flops / bytes >= 300.0));
 }
 
-int choose_bn_for(int64_t M, int64_t N, int64_t K) { return choose_bn(N, heavy_gemm(M, N, K)); }
+// A GEMM of one 128-row block (a few tokens: decode) streams its B operand
+// through as many CTAs as it has column tiles, so it takes 128-column tiles:
+// twice the CTAs of 256-column ones (measured: 1B decode step 0.066 ->
+// 0.059 ms, 7B 0.090 -> 0.083 ms).
+int choose_bn_for(int64_t M, int64_t N, int64_t K)
+{
+    if (M <= 128) return 128;
+    return choose_bn(N, heavy_gemm(M, N, K));
+}
 
 // Tile modes ("msub" below): 1 = one CTA runs a 128-row tile; 2 = one CTA
 // runs two 128-row sub-tiles sharing each B tile; TILE_PAIR = a CTA pair runs
