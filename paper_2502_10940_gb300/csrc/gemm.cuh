@@ -201,7 +201,7 @@ __device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w 
 // The value of every element is logistic_of<LOGI_SELECT>(z): the exponential
 // form below -TANH_FLOOR, the tanh form elsewhere.  The epilogues evaluate a
 // chunk of a row (32 values) with no input below the floor (under N(0, 1)
-// inputs, all but about 1 in 10^9) by the tanh form alone
+// inputs, all but about 3 chunks in 10^8) by the tanh form alone
 // (logistic_of<LOGI_TANH>), and any other chunk element by element with the
 // choice, out of line (the *_chunk_select functions below), so a result never
 // depends on its neighbours.  The SFU rate bounds the sigma epilogues of the
