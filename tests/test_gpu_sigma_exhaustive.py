@@ -161,3 +161,50 @@ def test_recompute_sigma_every_bf16_input(cola, sigma):
     assert "sigma" in [rec[0] for rec in tr.records()]
     z = zt.double().numpy().reshape(-1)[:count]
     _check(f"{sigma} (recompute)", Y.cpu().double().numpy().reshape(-1)[:count], oracle.sigma(sigma, z))
+
+
+@pytest.mark.parametrize("mode", ["cola", "cola_m"])
+@pytest.mark.parametrize("fused", [True, False], ids=["fused", "two_gemm"])
+def test_silu_value_independent_of_its_chunk(cola, mode, fused):
+    # SiLU evaluates a 32-value chunk with no input below the tanh form's
+    # floor by that form alone, and any other chunk element by element with
+    # the exponential form below the floor: every value must depend on its own
+    # input only.  All 512 rows of Z hold the same 128 values, except that odd
+    # rows replace one of them (a different column per row) with -20; sigma
+    # and sigma' of every other element must equal row 0's bit for bit.
+    g = torch.Generator().manual_seed(5)
+    u = (torch.randn(R, generator=g) * 2).to(torch.bfloat16)
+    zt = u.repeat(N_TOK, 1)
+    odd = torch.arange(1, N_TOK, 2)
+    cols = odd % R
+    zt[odd, cols] = -20.0
+    dev = "cuda"
+    X = torch.eye(N_TOK, dtype=torch.bfloat16, device=dev)
+    A = zt.t().contiguous().to(dev)
+    B = torch.eye(R, dtype=torch.bfloat16, device=dev)
+    dY = torch.ones((N_TOK, R), dtype=torch.bfloat16, device=dev)
+    d = cola.desc(N_TOK, N_TOK, R, R, sigma="silu", mode=mode)
+    ws = cola.workspace(d)
+    Y = torch.empty((N_TOK, R), dtype=torch.bfloat16, device=dev)
+    Z = torch.empty((N_TOK, R), dtype=torch.bfloat16, device=dev)
+    H = torch.empty((N_TOK, R), dtype=torch.bfloat16, device=dev) if mode == "cola" else None
+    dX = torch.empty((N_TOK, N_TOK), dtype=torch.bfloat16, device=dev)
+    dA = torch.empty((R, N_TOK), dtype=torch.bfloat16, device=dev)
+    dB = torch.empty((R, R), dtype=torch.bfloat16, device=dev)
+    cola.cola_set_fused_forward(fused)
+    cola.cola_set_fused_backward(fused)
+    try:
+        cola.cola_fwd(d, X, A, B, Y, Z, H, ws)
+        cola.cola_bwd(d, X, A, B, dY, Z, H, dX, dA, dB, ws)
+    finally:
+        cola.cola_set_fused_forward(True)
+        cola.cola_set_fused_backward(True)
+    assert cola.cola_check_status(ws)[0] == 0
+    assert torch.equal(Z.cpu(), zt)
+    h = Y.cpu().view(torch.int16)
+    dz = dA.t().cpu().view(torch.int16)
+    keep = torch.ones((N_TOK, R), dtype=torch.bool)
+    keep[odd, cols] = False
+    for out in (h, dz):
+        ref = out[0].expand(N_TOK, R)
+        assert torch.equal(out[keep], ref[keep])
