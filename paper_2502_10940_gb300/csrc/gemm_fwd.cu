@@ -34,9 +34,7 @@ template cudaError_t launch_gemm<256, 1, false, false, EPI_STORE>(const GemmBatc
 template cudaError_t launch_gemm<128, 2, false, false, EPI_STORE>(const GemmBatch&, int, bool, cudaStream_t);
 template cudaError_t launch_gemm<256, 1, false, false, EPI_STORE, true>(const GemmBatch&, int, bool, cudaStream_t);
 
-// H = bf16(sigma(Z)) over `vecs` groups of 8 bf16, each a 16-byte vector;
-// sigma is evaluated exactly as in the Z/H epilogue (same function on the
-// same bf16 inputs), so the result is bit-identical to the forward's H.
+// sigma of 8 bf16 values (one 16-byte vector), with the logistic's form L
 template <int S, int L>
 __device__ __forceinline__ uint4 sigma8(const uint4 z)
 {
@@ -48,6 +46,9 @@ __device__ __forceinline__ uint4 sigma8(const uint4 z)
     return h;
 }
 
+// H = bf16(sigma(Z)) over `vecs` groups of 8 bf16, each a 16-byte vector;
+// sigma is evaluated exactly as in the Z/H epilogue (same function on the
+// same bf16 inputs), so the result is bit-identical to the forward's H.
 template <int S>
 __global__ void __launch_bounds__(256) sigma_kernel(const uint4* __restrict__ Z, uint4* __restrict__ H, long long vecs)
 {

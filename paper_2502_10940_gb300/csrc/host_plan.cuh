@@ -100,9 +100,9 @@ bool heavy_gemm(int64_t M, int64_t N, int64_t K)
 
 // A GEMM of one 128-row block (a few tokens: decode) streams its B operand
 // through as many CTAs as it has column tiles, so it takes 128-column tiles:
-// twice the CTAs of 256-column ones (measured: 1B decode step 0.066 ->
-// 0.059 ms, 7B 0.090 -> 0.083 ms), up to N = 8192 (64 tiles; wider ones,
-// often batched in twos, would spill into a second wave of CTAs).
+// twice the CTAs of 256-column ones, up to N = 8192 (64 tiles; wider ones,
+// often batched in twos, would spill into a second wave of CTAs).  Measured:
+// 1B decode step 0.066 -> 0.059 ms, 7B 0.090 -> 0.081 ms.
 int choose_bn_for(int64_t M, int64_t N, int64_t K)
 {
     if (M <= 128 && N <= 8192) return 128;
