@@ -674,11 +674,14 @@ def whole_job_tflops(flops_per_rank_step, world, ms_per_step):
     return flops_per_rank_step * world / (ms_per_step / 1e3) / 1e12
 
 
-def full_rank_baseline(wl, device, steps, warmup, seed=0, flush=None, settle=0.0):
+def full_rank_baseline(wl, device, steps, warmup, seed=0, flush=None, settle=0.0, graph=False):
     """Same-shape full-rank layers (fwd Y = X W^T, bwd dX = dY W, dW = dY^T X;
     forward only for an inference workload) with torch.matmul (cuBLAS);
     layers reading one input (q/k/v, gate/up) are fused into one GEMM with
-    their output widths concatenated."""
+    their output widths concatenated.  With `graph`, the step is captured
+    once as a CUDA graph and replayed, as the CoLA step is, so that both
+    sides pay the same launch costs (which set the time of the small
+    workloads)."""
     import torch
 
     n = wl.n
@@ -719,11 +722,20 @@ def full_rank_baseline(wl, device, steps, warmup, seed=0, flush=None, settle=0.0
 
     for _ in range(warmup):
         step()
-    st = settle_steps(step, settle)
-    ms = time_steps(step, steps, torch.cuda.current_stream(), flush=flush)
+    run = step
+    if graph:
+        torch.cuda.synchronize()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            step()
+        run = g.replay
+        for _ in range(warmup):
+            run()
+    st = settle_steps(run, settle)
+    ms = time_steps(run, steps, torch.cuda.current_stream(), flush=flush)
     del bufs
     return {"ms_per_step": round(ms, 4), "tflops": round(flops / (ms / 1e3) / 1e12, 1), "flops": flops,
-            "impl": "torch.matmul (cuBLAS) bf16", "settle": st}
+            "impl": "torch.matmul (cuBLAS) bf16", "cuda_graph": bool(graph), "settle": st}
 
 
 def timed_block(wl, mode, args, device, stream, dist=None, seed=0, **block_kw):
@@ -963,7 +975,7 @@ def run_cola(args, wl):
             del g1
         if rank == 0 and world == 1:
             fr = full_rank_baseline(wl, device, max(3, args.steps // 2), 3, seed=args.seed, flush=flush,
-                                    settle=args.settle)
+                                    settle=args.settle, graph=use_graph)
             fr["speedup_cola_vs_full_rank"] = round(fr["ms_per_step"] / ms, 3)
             line["full_rank"] = fr
             mr = modes_ratio(wl, mode, blk, args, device, stream, seed=args.seed + rank)
